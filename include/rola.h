@@ -1,0 +1,186 @@
+/*
+ * rola.h -- C ABI of the RoLA hybrid-attention library for one GB300 (sm_103a).
+ *
+ * RoLA ("Rotary-Positioned Low-Rank Linear Attention") replaces dense 3D-RoPE
+ * self-attention in a video DiT layer with
+ *   - a block-sparse softmax branch over the kept 64-token key blocks of each
+ *     64-token query block (Alg. 1, sparse-branch steps; Sec. 3 for the
+ *     softmax form), and
+ *   - a low-rank linear-attention branch whose features are rotated by the
+ *     truncated 3D RoPE *after* the SiLU feature map (Eq. qklr), so one
+ *     summary C = sum_q k~_q v_q^T per head (Eq. ctx) serves every query,
+ * merged by the RMS-referenced token gate of Eq. (gate).
+ *
+ * Conventions shared by every entry point
+ *   Memory     every tensor pointer is a DEVICE pointer owned by the caller,
+ *              16-byte aligned and densely packed in the layout stated.  The
+ *              library allocates nothing and keeps no global mutable state;
+ *              scratch lives in the caller's workspace (see
+ *              rola_workspace_bytes).
+ *   Element    q, k, v, o, o_s, P_q, P_k are bf16 when cfg->dtype ==
+ *   types      ROLA_BF16 and fp32 when cfg->dtype == ROLA_FP32 (validation
+ *              mode: fp32 arithmetic everywhere, no bf16/tf32 rounding).
+ *              C, z and gate are always fp32; kv_idx is int32.
+ *   Layouts    q, k, v, o_s, o : [B][H][N][d_h]
+ *              P_q, P_k        : [H][r][d_h]   (one r x d_h projection per head)
+ *              C               : [B][H][r][d_h]
+ *              z               : [B][H][r]
+ *              gate            : [B][N]        (one scalar per token, shared by heads)
+ *              kv_idx          : [B][H][nQB][n_keep], ascending block ids
+ *   Tokens     token n of the flattened video sits at (t, x, y) with
+ *              t = n / (Hh*Ww), x = (n / Ww) % Hh, y = n % Ww (t-major), plus
+ *              cfg->pos_offset (Sec. 3 notation).
+ *   Inputs     q and k are the backbone's normalised, PRE-RoPE vectors
+ *              (q^n, k^n of Sec. 4.1 / Alg. 1); the library applies both the
+ *              full RoPE (sparse branch) and the truncated RoPE (low-rank
+ *              branch) itself.
+ *   Streams    `stream` is a cudaStream_t (NULL = legacy default stream).  All
+ *              calls are asynchronous on it.  Calls that share a workspace
+ *              must be ordered on one stream.
+ *   Errors     argument validation happens on the host before any launch
+ *              and returns ROLA_ERR_INVALID_ARG / ROLA_ERR_UNSUPPORTED /
+ *              ROLA_ERR_WORKSPACE with nothing launched; a launch failure
+ *              returns ROLA_ERR_CUDA.  A device-side bounded wait that gives
+ *              up records ROLA_ERR_TIMEOUT in the workspace status word,
+ *              which rola_get_device_status reads.  No C++ exception
+ *              crosses this ABI.
+ */
+#ifndef ROLA_H_
+#define ROLA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    ROLA_OK = 0,
+    ROLA_ERR_INVALID_ARG = 1,  /* bad pointer, shape, alignment or value */
+    ROLA_ERR_UNSUPPORTED = 2,  /* valid but not built here (e.g. d_h != 128) */
+    ROLA_ERR_WORKSPACE = 3,    /* workspace NULL, misaligned or too small */
+    ROLA_ERR_CUDA = 4,         /* a CUDA launch or runtime call failed */
+    ROLA_ERR_TIMEOUT = 5       /* a device-side bounded wait expired */
+} rola_status_t;
+
+typedef enum {
+    ROLA_BF16 = 0,             /* bf16 storage, tensor-core MMAs, fp32 accumulation */
+    ROLA_FP32 = 1              /* fp32 storage and fp32 arithmetic (validation mode) */
+} rola_dtype_t;
+
+/*
+ * Layer configuration (plain old data).  Fill with rola_config_init, then
+ * set the shape.  Defaults follow the paper where it gives a value and the
+ * stated reading where it does not.
+ */
+typedef struct {
+    int32_t B, H, N, d_h;      /* batch, heads, tokens, head dim (d_h == 128) */
+    int32_t T, Hh, Ww;         /* latent grid; N == T*Hh*Ww (Sec. 3) */
+    int32_t pos_offset[3];     /* added to (t, x, y); 0 normally */
+    int32_t rope_split[3];     /* d_t, d_x, d_y; each even, sum == d_h (Sec. 3); default 44,42,42 */
+    double rope_theta;         /* RoPE base; default 10000 */
+    int32_t block;             /* block size for queries and keys; 64 */
+    float keep_ratio;          /* n_keep = clamp(floor(keep_ratio*nKB + 0.5), 1, nKB) */
+    int32_t r;                 /* low-rank width, even, 16 <= r <= d_h, r % 16 == 0 */
+    float eps_lr;              /* RMSNorm epsilon of the low-rank readout; default 1e-6 */
+    float eps_fuse;            /* epsilon of the sparse-output RMS r_p, Eq. (gate); default 1e-6 */
+    float gate_bias;           /* g = sigmoid(gate_bias) when gate == NULL; default -1.946 */
+    rola_dtype_t dtype;        /* ROLA_BF16 (default) or ROLA_FP32 */
+} rola_config_t;
+
+/* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
+rola_status_t rola_config_init(rola_config_t* cfg);
+
+/* ceil(N / block): the number of query blocks nQB, equal to the number of key blocks nKB. */
+int32_t rola_num_blocks(const rola_config_t* cfg);
+
+/* Kept key blocks per query block, clamp(floor(keep_ratio*nKB + 0.5), 1, nKB); 0 if cfg is invalid. */
+int32_t rola_num_keep(const rola_config_t* cfg);
+
+/* Bytes of workspace every entry point below accepts for this cfg (the
+ * largest any of them needs); 0 if cfg is invalid.  The workspace must be
+ * 256-byte aligned.  Its first bytes hold the device status word. */
+size_t rola_workspace_bytes(const rola_config_t* cfg);
+
+/*
+ * Kernel (1): block mask.  Rotates q and k by the full 3D RoPE R(p)
+ * (Sec. 3, Eq. shiftinv), mean-pools each 64-token block, scores every
+ * (query block, key block) pair as q_bar . k_bar / sqrt(d_h) and keeps the
+ * n_keep highest-scoring key blocks of each query block (Alg. 1, "topk
+ * ratio"; the pooling / scoring rule is this library's reading of the
+ * unspecified selection of the sparse engine).  Ties go to the lower block
+ * id.  Pooled means and scores are fp32.
+ *   q, k    : [B][H][N][d_h] pre-RoPE, dtype
+ *   kv_idx  : out, int32 [B][H][nQB][n_keep], ascending within each row
+ */
+rola_status_t rola_block_mask(const rola_config_t* cfg, const void* q, const void* k,
+                              int32_t* kv_idx, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Kernel (2): block-sparse softmax attention (Alg. 1, sparse branch):
+ *   O^s_p = sum_{q in kept(i)} softmax_q(<R(p) q_p, R(q) k_q> / sqrt(d_h)) v_q
+ * for p in query block i, over the key blocks kv_idx lists for block i.
+ * Softmax is evaluated online in fp32.
+ *   q, k, v : [B][H][N][d_h] (q, k pre-RoPE), dtype
+ *   kv_idx  : int32 [B][H][nQB][n_keep], each row ascending, ids < nKB
+ *   o_s     : out, [B][H][N][d_h], dtype
+ */
+rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                               const int32_t* kv_idx, void* o_s, void* ws, size_t ws_bytes,
+                               void* stream);
+
+/*
+ * Kernel (3): low-rank summary, Eq. (qklr) and Eq. (ctx):
+ *   k~_q = R_r(q) SiLU(P_k k^n_q),   C = sum_q k~_q v_q^T,   z = sum_q k~_q.
+ * R_r keeps the first r coordinates (r/2 complete pairs) of the native RoPE
+ * ordering (Sec. 4.2).  The reduction over N is split across CTAs and
+ * combined in a fixed order, so results are bitwise reproducible.
+ *   k, v    : [B][H][N][d_h] (k pre-RoPE), dtype;  P_k : [H][r][d_h], dtype
+ *   C       : out, fp32 [B][H][r][d_h];   z : out, fp32 [B][H][r], or NULL
+ */
+rola_status_t rola_lowrank_summary(const rola_config_t* cfg, const void* k, const void* v,
+                                   const void* P_k, float* C, float* z, void* ws, size_t ws_bytes,
+                                   void* stream);
+
+/*
+ * Kernel (4): low-rank readout and gated fusion, Eq. (ctx) and Eq. (gate):
+ *   q~_p   = R_r(p) SiLU(P_q q^n_p)
+ *   O^lr_p = y_p / sqrt(mean_i y_{p,i}^2 + eps_lr),   y_p = q~_p^T C
+ *   r_p    = sqrt(mean_i (O^s_{p,i})^2 + eps_fuse)
+ *   O_p    = (O^s_p / r_p + g_p O^lr_p) r_p
+ * q~ never leaves the chip.
+ *   q       : [B][H][N][d_h] pre-RoPE, dtype;  P_q : [H][r][d_h], dtype
+ *   C       : fp32 [B][H][r][d_h];  gate : fp32 [B][N] or NULL (sigmoid(gate_bias))
+ *   o_s     : [B][H][N][d_h], dtype;  o : out, same layout, may alias o_s
+ */
+rola_status_t rola_lowrank_apply(const rola_config_t* cfg, const void* q, const void* P_q,
+                                 const float* C, const float* gate, const void* o_s, void* o,
+                                 void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * The whole module (Alg. 1, the per-head steps between the QKV projection
+ * and W_o): block mask, sparse branch, low-rank summary, readout and fusion.
+ *   o          : out, [B][H][N][d_h] fused per-head output O^fused, dtype
+ *   kv_idx_out : out, the mask used (int32 [B][H][nQB][n_keep]), or NULL
+ */
+rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                           const void* P_q, const void* P_k, const float* gate, void* o,
+                           int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Synchronises `stream`, then reads the device status word at the start of
+ * ws: ROLA_OK, or ROLA_ERR_TIMEOUT if a bounded device wait expired since the
+ * workspace was last cleared by an entry point.  ROLA_ERR_CUDA if the
+ * synchronisation or copy fails.
+ */
+rola_status_t rola_get_device_status(const void* ws, void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* rola_status_string(rola_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ROLA_H_ */

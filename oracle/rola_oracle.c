@@ -1,0 +1,545 @@
+/*
+ * RoLA hybrid attention -- plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously-correct
+ * reference the CUDA library is checked against.  Only the tests, the smoke
+ * check and the bench's CPU-baseline leg may load it; the product path never
+ * does.  It shares no code, header, table or constant with the CUDA library.
+ *
+ * Every input arrives as float32 (an exact copy of the bf16 / fp32 device
+ * inputs) and is upcast to double on read.  All arithmetic is fp64, each
+ * step written in the order the paper states it, with no blocking, fusion
+ * or reordering:
+ *
+ *   positions        Sec. 3 (Preliminary, notation): p = (t, x, y), token n
+ *                    of the flattened video is t-major.
+ *   full 3D RoPE     Sec. 3, Eq. (shiftinv): block-diagonal rotation R(p),
+ *                    d_h = d_t + d_x + d_y, pairs (2m, 2m+1) (Sec. 4.5,
+ *                    even/odd split), frequency theta^(-2i/d_axis).
+ *   truncated RoPE   Sec. 4.2: R_r(p) keeps the first r coordinates (r/2
+ *                    complete pairs) of the native ordering.
+ *   block mask       Alg. 1 "SparseAttn ... with topk ratio"; the selection
+ *                    rule itself is not given by the paper -- this oracle
+ *                    mean-pools the rotated q / k over each block, scores
+ *                    q_bar . k_bar / sqrt(d_h) and keeps the n_keep largest
+ *                    per query block (ties -> lower block index).
+ *   sparse branch    Sec. 3 (softmax(QK^T / sqrt d_h) V) restricted to the
+ *                    kept key blocks; Alg. 1 sparse-branch steps.
+ *   low-rank branch  Eq. (qklr): q~ = R_r(p) SiLU(P_q q^n), k~ = R_r(q)
+ *                    SiLU(P_k k^n); Eq. (ctx): C = sum_q k~_q v_q^T,
+ *                    O^lr = RMSNorm(q~^T C) with no gain.
+ *   fusion           Eq. (gate): r_p = sqrt(mean_i O^s_{p,i}^2 + eps),
+ *                    O = (O^s / r_p + g_p O^lr) r_p.
+ *   variants         Prop. (inside): SiLU(R_r(p) P x) ("inside"), and the
+ *                    no-RoPE ablation (Sec. 5.2) SiLU(P x).
+ *
+ * Layouts: q, k, v, o: [B][H][N][d_h]; P_q, P_k: [H][r][d_h];
+ * C: [B][H][r][d_h]; z: [B][H][r]; gate: [B][N] (NULL -> sigmoid(gate_bias));
+ * kv_idx: [B][H][nQB][n_keep] ascending.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+    int32_t B, H, N, dh;
+    int32_t T, Hh, Ww;
+    int32_t pos_offset[3];
+    int32_t split[3];
+    double theta;
+    int32_t block;
+    double keep;          /* keep ratio; n_keep = clamp(floor(keep*nKB+0.5), 1, nKB) */
+    int32_t r;
+    double eps_lr, eps_f;
+    double gate_bias;     /* g = sigmoid(gate_bias) when gate == NULL */
+    int32_t rope_mode;    /* 0: RoPE outside SiLU (RoLA), 1: inside, 2: none */
+} orc_cfg;
+
+/* ------------------------------------------------------------------ */
+/* sizes                                                              */
+/* ------------------------------------------------------------------ */
+
+int orc_num_blocks(const orc_cfg* c) { return (c->N + c->block - 1) / c->block; }
+
+int orc_num_keep(const orc_cfg* c)
+{
+    int nkb = orc_num_blocks(c);
+    double x = floor(c->keep * (double)nkb + 0.5);
+    int n = (int)x;
+    if (n < 1) n = 1;
+    if (n > nkb) n = nkb;
+    return n;
+}
+
+/* ------------------------------------------------------------------ */
+/* positions and RoPE (Sec. 3, Sec. 4.2)                              */
+/* ------------------------------------------------------------------ */
+
+/* token n -> (t, x, y), t-major flattening, plus the configured offset. */
+void orc_position(const orc_cfg* c, int n, double pos[3])
+{
+    int hw = c->Hh * c->Ww;
+    int t = n / hw;
+    int x = (n / c->Ww) % c->Hh;
+    int y = n % c->Ww;
+    pos[0] = (double)(t + c->pos_offset[0]);
+    pos[1] = (double)(x + c->pos_offset[1]);
+    pos[2] = (double)(y + c->pos_offset[2]);
+}
+
+/* Rotation angle of pair m (coordinates 2m, 2m+1) at position pos. */
+double orc_pair_angle(const orc_cfg* c, int m, const double pos[3])
+{
+    int pt = c->split[0] / 2, px = c->split[1] / 2;
+    int axis, i, d_axis;
+    if (m < pt) { axis = 0; i = m; d_axis = c->split[0]; }
+    else if (m < pt + px) { axis = 1; i = m - pt; d_axis = c->split[1]; }
+    else { axis = 2; i = m - pt - px; d_axis = c->split[2]; }
+    double freq = pow(c->theta, -2.0 * (double)i / (double)d_axis);
+    return pos[axis] * freq;
+}
+
+/* out = R(pos) restricted to the first 2*npairs coordinates, applied to in.
+ * Coordinates beyond 2*npairs are copied unchanged.  in / out of length len
+ * may alias. */
+void orc_rotate(const orc_cfg* c, int npairs, const double pos[3], const double* in,
+                double* out, int len)
+{
+    for (int m = 0; m < npairs; ++m) {
+        double a = orc_pair_angle(c, m, pos);
+        double ca = cos(a), sa = sin(a);
+        double x = in[2 * m], y = in[2 * m + 1];
+        out[2 * m] = x * ca - y * sa;
+        out[2 * m + 1] = x * sa + y * ca;
+    }
+    for (int i = 2 * npairs; i < len; ++i) out[i] = in[i];
+}
+
+static double silu(double x) { return x / (1.0 + exp(-x)); }
+
+/* ------------------------------------------------------------------ */
+/* low-rank features, Eq. (qklr) and its two ablations                */
+/* ------------------------------------------------------------------ */
+
+/* feat[r] for one token: x [dh] (float input), P [r][dh] (one head). */
+static void lowrank_feature(const orc_cfg* c, int n, const float* x, const float* P, double* feat)
+{
+    int r = c->r, dh = c->dh;
+    double pos[3];
+    orc_position(c, n, pos);
+    double* u = (double*)malloc(sizeof(double) * (size_t)r);
+    for (int a = 0; a < r; ++a) {
+        double s = 0.0;
+        for (int d = 0; d < dh; ++d) s += (double)P[(size_t)a * dh + d] * (double)x[d];
+        u[a] = s;
+    }
+    if (c->rope_mode == 0) {            /* R_r(p) SiLU(P x) */
+        for (int a = 0; a < r; ++a) u[a] = silu(u[a]);
+        orc_rotate(c, r / 2, pos, u, feat, r);
+    } else if (c->rope_mode == 1) {     /* SiLU(R_r(p) P x) */
+        orc_rotate(c, r / 2, pos, u, feat, r);
+        for (int a = 0; a < r; ++a) feat[a] = silu(feat[a]);
+    } else {                            /* SiLU(P x) */
+        for (int a = 0; a < r; ++a) feat[a] = silu(u[a]);
+    }
+    free(u);
+}
+
+/* Low-rank features of every token of every head: out [B][H][N][r]. */
+void orc_lowrank_features(const orc_cfg* c, const float* x, const float* P, double* out)
+{
+    int BH = c->B * c->H;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int h = bh % c->H;
+        for (int n = 0; n < c->N; ++n)
+            lowrank_feature(c, n, x + ((size_t)bh * c->N + n) * c->dh,
+                            P + (size_t)h * c->r * c->dh, out + ((size_t)bh * c->N + n) * c->r);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* summary C = sum_q k~_q v_q^T and z = sum_q k~_q, Eq. (ctx)         */
+/* ------------------------------------------------------------------ */
+
+void orc_lowrank_summary(const orc_cfg* c, const float* k, const float* v, const float* Pk,
+                         double* C, double* z)
+{
+    int BH = c->B * c->H, r = c->r, dh = c->dh;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int h = bh % c->H;
+        double* Cb = C + (size_t)bh * r * dh;
+        double* zb = z ? z + (size_t)bh * r : NULL;
+        double* kt = (double*)malloc(sizeof(double) * (size_t)r);
+        memset(Cb, 0, sizeof(double) * (size_t)r * dh);
+        if (zb) memset(zb, 0, sizeof(double) * (size_t)r);
+        for (int n = 0; n < c->N; ++n) {
+            lowrank_feature(c, n, k + ((size_t)bh * c->N + n) * dh, Pk + (size_t)h * r * dh, kt);
+            const float* vn = v + ((size_t)bh * c->N + n) * dh;
+            for (int a = 0; a < r; ++a) {
+                for (int d = 0; d < dh; ++d) Cb[(size_t)a * dh + d] += kt[a] * (double)vn[d];
+                if (zb) zb[a] += kt[a];
+            }
+        }
+        free(kt);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* readout, RMSNorm and fusion, Eq. (ctx) and Eq. (gate)             */
+/* ------------------------------------------------------------------ */
+
+static double gate_value(const orc_cfg* c, const float* gate, int b, int n)
+{
+    if (gate) return (double)gate[(size_t)b * c->N + n];
+    return 1.0 / (1.0 + exp(-c->gate_bias));
+}
+
+/* O^lr for token n of head bh into olr[dh]; y (pre-RMSNorm) into y if non-NULL. */
+static void lowrank_readout(const orc_cfg* c, int bh, int n, const float* q, const float* Pq,
+                            const double* C, double* olr, double* y)
+{
+    int r = c->r, dh = c->dh, h = bh % c->H;
+    double* qt = (double*)malloc(sizeof(double) * (size_t)r);
+    double* yy = (double*)malloc(sizeof(double) * (size_t)dh);
+    lowrank_feature(c, n, q + ((size_t)bh * c->N + n) * dh, Pq + (size_t)h * r * dh, qt);
+    const double* Cb = C + (size_t)bh * r * dh;
+    double ss = 0.0;
+    for (int d = 0; d < dh; ++d) {
+        double s = 0.0;
+        for (int a = 0; a < r; ++a) s += qt[a] * Cb[(size_t)a * dh + d];
+        yy[d] = s;
+        ss += s * s;
+    }
+    double inv = 1.0 / sqrt(ss / (double)dh + c->eps_lr);
+    for (int d = 0; d < dh; ++d) {
+        if (olr) olr[d] = yy[d] * inv;
+        if (y) y[d] = yy[d];
+    }
+    free(qt);
+    free(yy);
+}
+
+/* Fusion of one token: o_s [dh] (double), olr [dh], gate g -> out [dh]. */
+static void fuse(const orc_cfg* c, const double* os, const double* olr, double g, double* out)
+{
+    int dh = c->dh;
+    double ss = 0.0;
+    for (int d = 0; d < dh; ++d) ss += os[d] * os[d];
+    double rp = sqrt(ss / (double)dh + c->eps_f);
+    for (int d = 0; d < dh; ++d) out[d] = (os[d] / rp + g * olr[d]) * rp;
+}
+
+/* Token list helper: the tokens of the selected query blocks (all if NULL). */
+static int token_in_selection(const orc_cfg* c, int n, const uint8_t* qb_sel)
+{
+    return qb_sel == NULL || qb_sel[n / c->block];
+}
+
+/* O = fusion(O^s, RMSNorm(q~^T C)) for the tokens of the selected query
+ * blocks (qb_sel[nQB] flags, NULL = all).  o_s is float [B][H][N][dh]. */
+void orc_lowrank_apply(const orc_cfg* c, const float* q, const float* Pq, const double* C,
+                       const float* gate, const float* o_s, const uint8_t* qb_sel, double* o)
+{
+    int BH = c->B * c->H, dh = c->dh;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int b = bh / c->H;
+        double* olr = (double*)malloc(sizeof(double) * (size_t)dh);
+        double* os = (double*)malloc(sizeof(double) * (size_t)dh);
+        for (int n = 0; n < c->N; ++n) {
+            if (!token_in_selection(c, n, qb_sel)) continue;
+            size_t off = ((size_t)bh * c->N + n) * dh;
+            lowrank_readout(c, bh, n, q, Pq, C, olr, NULL);
+            for (int d = 0; d < dh; ++d) os[d] = (double)o_s[off + d];
+            fuse(c, os, olr, gate_value(c, gate, b, n), o + off);
+        }
+        free(olr);
+        free(os);
+    }
+}
+
+/* Pre-RMSNorm readout y_p = q~_p^T C for every token: y [B][H][N][dh]. */
+void orc_lowrank_readout(const orc_cfg* c, const float* q, const float* Pq, const double* C, double* y)
+{
+    int BH = c->B * c->H;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh)
+        for (int n = 0; n < c->N; ++n)
+            lowrank_readout(c, bh, n, q, Pq, C, NULL, y + ((size_t)bh * c->N + n) * c->dh);
+}
+
+/* Explicit O(N^2) form of the pre-RMSNorm low-rank output,
+ * y_p = sum_q (q~_p . k~_q) v_q  (Prop. exact, Step 2, read right to left). */
+void orc_lowrank_explicit(const orc_cfg* c, const float* q, const float* k, const float* v,
+                          const float* Pq, const float* Pk, double* y)
+{
+    int BH = c->B * c->H, r = c->r, dh = c->dh, N = c->N;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int h = bh % c->H;
+        double* kt = (double*)malloc(sizeof(double) * (size_t)N * r);
+        double* qt = (double*)malloc(sizeof(double) * (size_t)r);
+        for (int n = 0; n < N; ++n)
+            lowrank_feature(c, n, k + ((size_t)bh * N + n) * dh, Pk + (size_t)h * r * dh,
+                            kt + (size_t)n * r);
+        for (int p = 0; p < N; ++p) {
+            lowrank_feature(c, p, q + ((size_t)bh * N + p) * dh, Pq + (size_t)h * r * dh, qt);
+            double* yp = y + ((size_t)bh * N + p) * dh;
+            for (int d = 0; d < dh; ++d) yp[d] = 0.0;
+            for (int n = 0; n < N; ++n) {
+                double w = 0.0;
+                for (int a = 0; a < r; ++a) w += qt[a] * kt[(size_t)n * r + a];
+                const float* vn = v + ((size_t)bh * N + n) * dh;
+                for (int d = 0; d < dh; ++d) yp[d] += w * (double)vn[d];
+            }
+        }
+        free(kt);
+        free(qt);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* full RoPE of q / k for the sparse branch (Alg. 1, sparse steps)    */
+/* ------------------------------------------------------------------ */
+
+/* Rotated copy of x [B][H][N][dh] into xr (double). */
+void orc_rope_full(const orc_cfg* c, const float* x, double* xr)
+{
+    int BH = c->B * c->H, dh = c->dh;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        double* tmp = (double*)malloc(sizeof(double) * (size_t)dh);
+        for (int n = 0; n < c->N; ++n) {
+            double pos[3];
+            orc_position(c, n, pos);
+            size_t off = ((size_t)bh * c->N + n) * dh;
+            for (int d = 0; d < dh; ++d) tmp[d] = (double)x[off + d];
+            orc_rotate(c, dh / 2, pos, tmp, xr + off, dh);
+        }
+        free(tmp);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* block mask: pooled scores + per-row top-n_keep                     */
+/* ------------------------------------------------------------------ */
+
+typedef struct { double s; int j; } scored;
+
+static int cmp_scored(const void* a, const void* b)
+{
+    const scored* x = (const scored*)a;
+    const scored* y = (const scored*)b;
+    if (x->s > y->s) return -1;
+    if (x->s < y->s) return 1;
+    return (x->j < y->j) ? -1 : (x->j > y->j);   /* ties: lower block first */
+}
+
+static int cmp_int(const void* a, const void* b)
+{
+    int x = *(const int*)a, y = *(const int*)b;
+    return (x > y) - (x < y);
+}
+
+/*
+ * Block mask.  Outputs (any may be NULL except kv_idx):
+ *   kv_idx [B][H][nQB][n_keep]   kept key blocks, ascending
+ *   scores [B][H][nQB][nKB]      s_ij = q_bar_i . k_bar_j / sqrt(dh)
+ *   gap    [B][H][nQB]           s_(n_keep) - s_(n_keep+1) in descending order
+ *                                (+inf when n_keep == nKB)
+ *   tau    [B][H][nQB]           an upper bound on the difference between this
+ *                                score row and one evaluated in fp32 arithmetic
+ *                                (u = 2^-24) in any summation order, times 2
+ *                                (two scores enter a comparison) times a safety
+ *                                factor 4.  A row with gap <= tau is a
+ *                                near-tie row: more than one kept set is a
+ *                                correct fp32 answer there.
+ */
+void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* kv_idx,
+                    double* scores, double* gap, double* tau)
+{
+    int BH = c->B * c->H, dh = c->dh, N = c->N, bs = c->block;
+    int nB = orc_num_blocks(c), nk = orc_num_keep(c);
+    double isd = 1.0 / sqrt((double)dh);
+    const double u = ldexp(1.0, -24);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        size_t nbd = (size_t)nB * dh;
+        double* qb = (double*)calloc(nbd, sizeof(double));   /* pooled means */
+        double* kb = (double*)calloc(nbd, sizeof(double));
+        double* qa = (double*)calloc(nbd, sizeof(double));   /* pooled |pair| magnitudes */
+        double* ka = (double*)calloc(nbd, sizeof(double));
+        double* xr = (double*)malloc(sizeof(double) * (size_t)dh);
+        double* xi = (double*)malloc(sizeof(double) * (size_t)dh);
+        scored* row = (scored*)malloc(sizeof(scored) * (size_t)nB);
+        for (int which = 0; which < 2; ++which) {
+            const float* x = which == 0 ? q : k;
+            double* mean = which == 0 ? qb : kb;
+            double* mag = which == 0 ? qa : ka;
+            for (int n = 0; n < N; ++n) {
+                double pos[3];
+                orc_position(c, n, pos);
+                size_t off = ((size_t)bh * N + n) * dh;
+                for (int d = 0; d < dh; ++d) xi[d] = (double)x[off + d];
+                orc_rotate(c, dh / 2, pos, xi, xr, dh);
+                int blk = n / bs;
+                for (int d = 0; d < dh; ++d) {
+                    mean[(size_t)blk * dh + d] += xr[d];
+                    mag[(size_t)blk * dh + d] += fabs(xi[d & ~1]) + fabs(xi[d | 1]);
+                }
+            }
+            for (int blk = 0; blk < nB; ++blk) {
+                int cnt = (blk + 1) * bs <= N ? bs : N - blk * bs;
+                for (int d = 0; d < dh; ++d) {
+                    mean[(size_t)blk * dh + d] /= (double)cnt;
+                    mag[(size_t)blk * dh + d] /= (double)cnt;
+                }
+            }
+        }
+        for (int i = 0; i < nB; ++i) {
+            const double* qi = qb + (size_t)i * dh;
+            const double* qm = qa + (size_t)i * dh;
+            double tmax = 0.0;
+            for (int j = 0; j < nB; ++j) {
+                const double* kj = kb + (size_t)j * dh;
+                const double* km = ka + (size_t)j * dh;
+                double s = 0.0, a1 = 0.0, a2 = 0.0;
+                for (int d = 0; d < dh; ++d) {
+                    s += qi[d] * kj[d];
+                    a1 += fabs(qi[d]) * fabs(kj[d]);
+                    a2 += qm[d] * fabs(kj[d]) + fabs(qi[d]) * km[d];
+                }
+                row[j].s = s * isd;
+                row[j].j = j;
+                if (scores) scores[((size_t)bh * nB + i) * nB + j] = s * isd;
+                /* rotation (3u) + pooling over <= bs terms + 1 divide, per
+                 * operand; dot product over dh terms; final scale. */
+                double e = u * ((double)(dh + 2) * a1 + (double)(bs + 4) * a2) * isd;
+                if (e > tmax) tmax = e;
+            }
+            qsort(row, (size_t)nB, sizeof(scored), cmp_scored);
+            int32_t* out = kv_idx + ((size_t)bh * nB + i) * nk;
+            for (int t = 0; t < nk; ++t) out[t] = row[t].j;
+            qsort(out, (size_t)nk, sizeof(int32_t), cmp_int);
+            if (gap) gap[(size_t)bh * nB + i] = nk < nB ? row[nk - 1].s - row[nk].s : INFINITY;
+            if (tau) tau[(size_t)bh * nB + i] = 2.0 * 4.0 * tmax;
+        }
+        free(qb); free(kb); free(qa); free(ka); free(xr); free(xi); free(row);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* block-sparse softmax attention                                     */
+/* ------------------------------------------------------------------ */
+
+/* O^s for the tokens of the selected query blocks (qb_sel flags, NULL =
+ * all).  qr, kr: rotated q / k (double) [B][H][N][dh]; v float; kv_idx
+ * [B][H][nQB][n_keep]; o_s out double [B][H][N][dh] (rows outside the
+ * selection untouched). */
+void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const float* v,
+                     const int32_t* kv_idx, int n_keep, const uint8_t* qb_sel, double* o_s)
+{
+    int BH = c->B * c->H, dh = c->dh, N = c->N, bs = c->block;
+    int nB = orc_num_blocks(c);
+    double isd = 1.0 / sqrt((double)dh);
+    int ntask = BH * nB;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int task = 0; task < ntask; ++task) {
+        int bh = task / nB, i = task % nB;
+        if (qb_sel && !qb_sel[i]) continue;
+        const int32_t* kept = kv_idx + ((size_t)bh * nB + i) * n_keep;
+        int nkeys = 0;
+        for (int t = 0; t < n_keep; ++t) {
+            int j = kept[t];
+            nkeys += (j + 1) * bs <= N ? bs : N - j * bs;
+        }
+        int* keys = (int*)malloc(sizeof(int) * (size_t)nkeys);
+        double* s = (double*)malloc(sizeof(double) * (size_t)nkeys);
+        int kk = 0;
+        for (int t = 0; t < n_keep; ++t)
+            for (int qn = kept[t] * bs; qn < (kept[t] + 1) * bs && qn < N; ++qn) keys[kk++] = qn;
+        for (int p = i * bs; p < (i + 1) * bs && p < N; ++p) {
+            const double* qp = qr + ((size_t)bh * N + p) * dh;
+            double mx = -INFINITY;
+            for (int t = 0; t < nkeys; ++t) {
+                const double* kq = kr + ((size_t)bh * N + keys[t]) * dh;
+                double acc = 0.0;
+                for (int d = 0; d < dh; ++d) acc += qp[d] * kq[d];
+                s[t] = acc * isd;
+                if (s[t] > mx) mx = s[t];
+            }
+            double den = 0.0;
+            for (int t = 0; t < nkeys; ++t) { s[t] = exp(s[t] - mx); den += s[t]; }
+            double* op = o_s + ((size_t)bh * N + p) * dh;
+            for (int d = 0; d < dh; ++d) op[d] = 0.0;
+            for (int t = 0; t < nkeys; ++t) {
+                const float* vq = v + ((size_t)bh * N + keys[t]) * dh;
+                double w = s[t] / den;
+                for (int d = 0; d < dh; ++d) op[d] += w * (double)vq[d];
+            }
+        }
+        free(keys);
+        free(s);
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* full forward (Alg. 1, the per-head steps between QKV and W_o)      */
+/* ------------------------------------------------------------------ */
+
+/*
+ * o [B][H][N][dh] for the tokens of the selected query blocks.  The mask is
+ * computed here (kv_idx_out receives it if non-NULL), unless mask_override is
+ * given.  Intermediates (o_s_out, C_out, z_out) are returned when non-NULL.
+ */
+void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* v,
+                 const float* Pq, const float* Pk, const float* gate,
+                 const int32_t* mask_override, const uint8_t* qb_sel,
+                 double* o, int32_t* kv_idx_out, double* o_s_out, double* C_out, double* z_out)
+{
+    size_t nel = (size_t)c->B * c->H * c->N * c->dh;
+    int nB = orc_num_blocks(c), nk = orc_num_keep(c);
+    size_t nmask = (size_t)c->B * c->H * nB * nk;
+    int32_t* mask = (int32_t*)malloc(sizeof(int32_t) * nmask);
+    if (mask_override) memcpy(mask, mask_override, sizeof(int32_t) * nmask);
+    else orc_block_mask(c, q, k, mask, NULL, NULL, NULL);
+    if (kv_idx_out) memcpy(kv_idx_out, mask, sizeof(int32_t) * nmask);
+
+    double* qr = (double*)malloc(sizeof(double) * nel);
+    double* kr = (double*)malloc(sizeof(double) * nel);
+    orc_rope_full(c, q, qr);
+    orc_rope_full(c, k, kr);
+    double* os = (double*)calloc(nel, sizeof(double));
+    orc_sparse_attn(c, qr, kr, v, mask, nk, qb_sel, os);
+    free(qr);
+    free(kr);
+
+    size_t nC = (size_t)c->B * c->H * c->r * c->dh;
+    double* C = (double*)malloc(sizeof(double) * nC);
+    double* z = (double*)malloc(sizeof(double) * (size_t)c->B * c->H * c->r);
+    orc_lowrank_summary(c, k, v, Pk, C, z);
+
+    int BH = c->B * c->H, dh = c->dh;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int b = bh / c->H;
+        double* olr = (double*)malloc(sizeof(double) * (size_t)dh);
+        for (int n = 0; n < c->N; ++n) {
+            if (!token_in_selection(c, n, qb_sel)) continue;
+            size_t off = ((size_t)bh * c->N + n) * dh;
+            lowrank_readout(c, bh, n, q, Pq, C, olr, NULL);
+            fuse(c, os + off, olr, gate_value(c, gate, b, n), o + off);
+        }
+        free(olr);
+    }
+    if (o_s_out) memcpy(o_s_out, os, sizeof(double) * nel);
+    if (C_out) memcpy(C_out, C, sizeof(double) * nC);
+    if (z_out) memcpy(z_out, z, sizeof(double) * (size_t)c->B * c->H * c->r);
+    free(os);
+    free(C);
+    free(z);
+    free(mask);
+}

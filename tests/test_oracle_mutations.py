@@ -1,0 +1,57 @@
+"""Plants plausible mistakes in a copy of the oracle and checks the pins catch each.
+
+Each mutation edits one line of ``oracle/rola_oracle.c`` (a sign, an index, a
+divisor, a dropped factor, a swapped order), compiles it to a temporary
+library and runs the pin suite against it in a subprocess: the suite must
+fail.  CPU only; nothing here touches the CUDA library.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "rola_oracle.c")
+
+MUTATIONS = {
+    "rotation_sign": ("out[2 * m] = x * ca - y * sa;", "out[2 * m] = x * ca + y * sa;"),
+    "rotation_pair_swap": ("out[2 * m + 1] = x * sa + y * ca;", "out[2 * m + 1] = y * sa + x * ca;"),
+    "frequency_exponent": ("pow(c->theta, -2.0 * (double)i / (double)d_axis)",
+                           "pow(c->theta, -1.0 * (double)i / (double)d_axis)"),
+    "axis_boundary": ("if (m < pt) { axis = 0;", "if (m <= pt) { axis = 0;"),
+    "position_row_index": ("int x = (n / c->Ww) % c->Hh;", "int x = (n / c->Hh) % c->Ww;"),
+    "silu_sign": ("return x / (1.0 + exp(-x));", "return x / (1.0 + exp(x));"),
+    "truncation_pairs": ("orc_rotate(c, r / 2, pos, u, feat, r);\n    } else if",
+                         "orc_rotate(c, r / 2 - 1, pos, u, feat, r);\n    } else if"),
+    "summary_transposed": ("Cb[(size_t)a * dh + d] += kt[a] * (double)vn[d];",
+                           "Cb[(size_t)a * dh + d] += kt[a] * (double)vn[(d + 1) % dh];"),
+    "mask_tie_order": ("return (x->j < y->j) ? -1 : (x->j > y->j);",
+                       "return (x->j > y->j) ? -1 : (x->j < y->j);"),
+    "pool_divisor": ("mean[(size_t)blk * dh + d] /= (double)cnt;", "mean[(size_t)blk * dh + d] /= (double)bs;"),
+    "pool_unrotated": ("mean[(size_t)blk * dh + d] += xr[d];", "mean[(size_t)blk * dh + d] += xi[d];"),
+    "softmax_scale": ("double isd = 1.0 / sqrt((double)dh);\n    int ntask",
+                      "double isd = 1.0;\n    int ntask"),
+    "ragged_keys": ("nkeys += (j + 1) * bs <= N ? bs : N - j * bs;", "nkeys += bs <= N ? bs : N;"),
+    "fusion_norm": ("out[d] = (os[d] / rp + g * olr[d]) * rp;", "out[d] = (os[d] + g * olr[d]) * rp;"),
+    "rmsnorm_mean": ("double inv = 1.0 / sqrt(ss / (double)dh + c->eps_lr);",
+                     "double inv = 1.0 / sqrt(ss + c->eps_lr);"),
+    "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    old, new = MUTATIONS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor for {name} not unique"
+    mutated = tmp_path / "mut.c"
+    mutated.write_text(src.replace(old, new))
+    lib = tmp_path / "libmut.so"
+    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c99", "-o", str(lib),
+                           str(mutated), "-lm"])
+    env = dict(os.environ, ORACLE_LIB=str(lib), OMP_NUM_THREADS="4")
+    res = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                          os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                         cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert res.returncode != 0, f"mutation {name} survived the pins:\n{res.stdout[-2000:]}"

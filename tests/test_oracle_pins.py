@@ -1,0 +1,374 @@
+"""Pins of the fp64 oracle to facts outside itself (CPU only).
+
+Each test checks the oracle against something the paper or the mathematics
+fixes: closed forms, exact identities the paper proves, special cases that
+reduce to a library routine (torch SDPA, torch rms_norm, torch silu), brute
+force on tiny inputs, and invariants.  See the per-test docstrings for the
+passage each one follows.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_06712_gb300 import configs, inputs
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def small_cfg(**kw):
+    """A small ragged layer: 3 x 5 x 7 grid = 105 tokens -> blocks of 64 and 41."""
+    c = configs.get("tiny")
+    c.update(T=3, Hh=5, Ww=7, H=2, r=16, keep=0.5, seed=11)
+    c.update(kw)
+    c["N"] = c["T"] * c["Hh"] * c["Ww"]
+    return c
+
+
+def draw(cfg, dtype=torch.float32):
+    x = inputs.make_inputs(cfg, dtype=dtype)
+    return {n: (None if t is None else t.float().numpy()) for n, t in x.items()}
+
+
+# ---------------------------------------------------------------- RoPE --------
+
+def rot_matrix(O, cfg, npairs, pos, dim):
+    return np.stack([O.rotate(cfg, npairs, pos, e) for e in np.eye(dim)], axis=1)
+
+
+def test_rope_orthogonal_and_group_property(oracle):
+    """Sec. 3 (R(p) orthogonal) and App. B (R_r(p)^T R_r(q) = R_r(q - p), R(0) = I)."""
+    O = oracle
+    cfg = configs.get("tiny")
+    rng = np.random.default_rng(0)
+    for npairs in (8, 16, 32, 64):
+        dim = 2 * npairs
+        for _ in range(3):
+            p = rng.integers(-40, 90, size=3).astype(float)
+            q = rng.integers(-40, 90, size=3).astype(float)
+            Rp = rot_matrix(O, cfg, npairs, p, dim)
+            Rq = rot_matrix(O, cfg, npairs, q, dim)
+            Rqp = rot_matrix(O, cfg, npairs, q - p, dim)
+            np.testing.assert_allclose(Rp.T @ Rp, np.eye(dim), atol=1e-13)
+            np.testing.assert_allclose(Rp.T @ Rq, Rqp, atol=1e-12)
+        np.testing.assert_allclose(rot_matrix(O, cfg, npairs, np.zeros(3), dim), np.eye(dim), atol=0)
+
+
+def test_rope_closed_forms(oracle):
+    """Sec. 3 / Sec. 4.2 with the 44/42/42 split and theta = 10^4: the first pair of
+    each axis turns by exactly its position (frequency theta^0 = 1), frequencies
+    fall geometrically by theta^(-2/d_axis) within an axis, and the pair ->
+    axis assignment follows the native ordering t | x | y."""
+    O = oracle
+    cfg = configs.get("tiny")
+    pos = np.array([3.0, 5.0, 7.0])
+    assert O.pair_angle(cfg, 0, pos) == 3.0           # first temporal pair
+    assert O.pair_angle(cfg, 22, pos) == 5.0          # first height pair
+    assert O.pair_angle(cfg, 43, pos) == 7.0          # first width pair
+    for m in range(1, 22):
+        ratio = O.pair_angle(cfg, m, pos) / O.pair_angle(cfg, m - 1, pos)
+        assert ratio == pytest.approx(10000.0 ** (-2.0 / 44.0), rel=1e-14)
+    for m in range(23, 43):
+        ratio = O.pair_angle(cfg, m, pos) / O.pair_angle(cfg, m - 1, pos)
+        assert ratio == pytest.approx(10000.0 ** (-2.0 / 42.0), rel=1e-14)
+    # the truncated schedule at r = 32 is purely temporal: moving x, y does nothing
+    assert all(O.pair_angle(cfg, m, [3, 0, 0]) == O.pair_angle(cfg, m, pos) for m in range(16))
+
+
+def test_rope_is_complex_multiplication(oracle):
+    """Sec. 4.5: RoPE acts on adjacent (even, odd) coordinate pairs; each pair is the
+    complex number x + iy multiplied by exp(i angle) (a counter-clockwise turn)."""
+    O = oracle
+    cfg = configs.get("tiny")
+    rng = np.random.default_rng(1)
+    x = rng.standard_normal(128)
+    pos = np.array([2.0, 9.0, 4.0])
+    got = O.rotate(cfg, 64, pos, x)
+    ang = np.array([O.pair_angle(cfg, m, pos) for m in range(64)])
+    z = (x[0::2] + 1j * x[1::2]) * np.exp(1j * ang)
+    np.testing.assert_allclose(got[0::2], z.real, atol=1e-14)
+    np.testing.assert_allclose(got[1::2], z.imag, atol=1e-14)
+    # coordinates past the truncation are untouched
+    got_r = O.rotate(cfg, 8, pos, x)
+    np.testing.assert_array_equal(got_r[16:], x[16:])
+    np.testing.assert_allclose(got_r[:16], got[:16], atol=0)
+
+
+def test_positions_t_major(oracle):
+    """Sec. 3 notation: p = (t, x, y), L = T H W; flattening is t-major."""
+    O = oracle
+    cfg = small_cfg()
+    for n in (0, 1, 6, 7, 34, 35, 36, 104):
+        t, x, y = np.unravel_index(n, (cfg["T"], cfg["Hh"], cfg["Ww"]))
+        np.testing.assert_array_equal(O.position(cfg, n), [t, x, y])
+    cfg2 = small_cfg(pos_offset=(2, -1, 5))
+    np.testing.assert_array_equal(O.position(cfg2, 36), np.array([1, 0, 1]) + [2, -1, 5])
+
+
+# ---------------------------------------------------------------- mask --------
+
+def test_num_keep_rounding(oracle):
+    """n_keep = clamp(floor(keep * nKB + 0.5), 1, nKB) at the layer shapes."""
+    O = oracle
+    assert O.num_keep(configs.get("tiny")) == 2
+    assert O.num_keep(configs.get("wan13b_480p")) == 51
+    assert O.num_keep(configs.get("wan14b_720p")) == 118
+    assert O.num_keep(configs.get("wan14b_720p_long")) == 231
+    assert O.num_blocks(configs.get("wan14b_720p")) == 1182
+    assert O.num_keep(small_cfg(keep=0.0)) == 1
+    assert O.num_keep(small_cfg(keep=1.0)) == 2
+
+
+def test_mask_is_the_best_subset_by_brute_force(oracle):
+    """Top-k by exhaustive search: on distinct scores, the kept set is the unique
+    n_keep-subset with the largest score sum."""
+    O = oracle
+    cfg = configs.get("tiny")
+    x = draw(cfg)
+    idx, scores, gap, tau = O.block_mask(cfg, x["q"], x["k"])
+    nb, nk = scores.shape[-1], idx.shape[-1]
+    for h in range(cfg["H"]):
+        for i in range(nb):
+            s = scores[0, h, i]
+            best = max(itertools.combinations(range(nb), nk), key=lambda S: sum(s[list(S)]))
+            assert list(best) == list(idx[0, h, i])
+            srt = np.sort(s)[::-1]
+            assert gap[0, h, i] == pytest.approx(srt[nk - 1] - srt[nk], abs=1e-15)
+
+
+def test_mask_closed_form_single_token(oracle):
+    """Pooling divides by the block's own token count (the ragged last block too);
+    ties go to the lower key block.  q and k are zero except one token whose
+    position is moved to the origin (R = I), so every score is known."""
+    O = oracle
+    cfg = small_cfg(keep=0.5)          # 2 blocks of 64 and 41 tokens, n_keep = 1
+    n = 70                             # a token of the partial block
+    t, xx, y = np.unravel_index(n, (cfg["T"], cfg["Hh"], cfg["Ww"]))
+    cfg["pos_offset"] = (-int(t), -int(xx), -int(y))
+    q = np.zeros((1, cfg["H"], cfg["N"], 128), np.float32)
+    k = np.zeros_like(q)
+    a = np.linspace(-1, 1, 128).astype(np.float32)
+    q[0, :, n] = a
+    k[0, :, n] = a
+    idx, scores, gap, tau = O.block_mask(cfg, q, k)
+    expect = float(a.astype(np.float64) @ a.astype(np.float64)) / 41 ** 2 / math.sqrt(128)
+    assert scores[0, 0, 1, 1] == pytest.approx(expect, rel=1e-14)
+    assert scores[0, 0, 0, 0] == 0 and scores[0, 0, 0, 1] == 0
+    assert idx[0, 0, 1, 0] == 1        # the one positive score wins
+    assert idx[0, 0, 0, 0] == 0        # all-zero row: the tie goes to block 0
+    # a negative pooled score loses to the zero score of the other block
+    k[0, :, n] = -a
+    idx, scores, _, _ = O.block_mask(cfg, q, k)
+    assert scores[0, 0, 1, 1] == pytest.approx(-expect, rel=1e-14)
+    assert idx[0, 0, 1, 0] == 0
+    # pooling acts on the ROTATED vectors: a query token and a key token at
+    # different positions score a^T R(p_k - p_q) b (Eq. shiftinv)
+    cfg["pos_offset"] = (0, 0, 0)
+    nq, nk = 10, 100                   # blocks 0 (64 tokens) and 1 (41 tokens)
+    q[:] = 0
+    k[:] = 0
+    b = np.cos(np.arange(128)).astype(np.float32)
+    q[0, :, nq] = a
+    k[0, :, nk] = b
+    _, scores, _, _ = O.block_mask(cfg, q, k)
+    rel = O.position(cfg, nk) - O.position(cfg, nq)
+    expect = float(a.astype(np.float64) @ O.rotate(cfg, 64, rel, b)) / (64 * 41) / math.sqrt(128)
+    assert scores[0, 0, 0, 1] == pytest.approx(expect, rel=1e-12)
+    assert abs(expect - float(a @ b) / (64 * 41) / math.sqrt(128)) > 1e-3 * abs(expect)
+
+
+def test_mask_keep_all_and_shift_invariance(oracle):
+    """keep = 1 keeps every block in order; the pooled scores depend only on relative
+    positions (Eq. shiftinv: each block mean turns by the same R(delta))."""
+    O = oracle
+    cfg = small_cfg(keep=1.0)
+    x = draw(cfg)
+    idx, _, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    assert (idx == np.arange(2)).all()
+    cfg = configs.get("tiny")
+    x = draw(cfg)
+    _, s0, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    _, s1, _, _ = O.block_mask(dict(cfg, pos_offset=(5, -3, 11)), x["q"], x["k"])
+    np.testing.assert_allclose(s1, s0, atol=1e-13)
+
+
+# ---------------------------------------------------------------- sparse ------
+
+def sdpa64(qr, kr, v, mask=None):
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float64))
+    return torch.nn.functional.scaled_dot_product_attention(
+        t(qr), t(kr), t(v), attn_mask=None if mask is None else torch.from_numpy(mask)).numpy()
+
+
+@pytest.mark.parametrize("grid", [(4, 16, 16), (3, 5, 7)])
+def test_sparse_keep_all_is_dense_sdpa(oracle, grid):
+    """T4: at keep ratio 1 the block-sparse branch is dense softmax attention
+    softmax(Q K^T / sqrt d_h) V (Sec. 3), here torch's fp64 SDPA."""
+    O = oracle
+    cfg = small_cfg(T=grid[0], Hh=grid[1], Ww=grid[2], keep=1.0)
+    x = draw(cfg)
+    qr, kr = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"])
+    idx, _, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    got = O.sparse_attn(cfg, qr, kr, x["v"], idx)
+    np.testing.assert_allclose(got, sdpa64(qr, kr, x["v"]), rtol=1e-11, atol=1e-12)
+
+
+def test_sparse_with_mask_is_masked_sdpa(oracle):
+    """The sparse branch with a block mask equals SDPA with the equivalent boolean
+    token mask; query rows of the ragged block use only real keys."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=9, Ww=10, keep=0.34)     # 360 tokens: 6 blocks, last has 40
+    x = draw(cfg)
+    qr, kr = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"])
+    idx, _, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    N, bs = cfg["N"], cfg["block"]
+    mask = np.zeros((1, cfg["H"], N, N), dtype=bool)
+    for h in range(cfg["H"]):
+        for i in range(idx.shape[2]):
+            for j in idx[0, h, i]:
+                mask[0, h, i * bs:(i + 1) * bs, j * bs:(j + 1) * bs] = True
+    got = O.sparse_attn(cfg, qr, kr, x["v"], idx)
+    np.testing.assert_allclose(got, sdpa64(qr, kr, x["v"], mask), rtol=1e-11, atol=1e-12)
+    sel = O.sparse_attn(cfg, qr, kr, x["v"], idx, qblocks=[1, 5])
+    np.testing.assert_array_equal(sel[:, :, 64:128], got[:, :, 64:128])
+    assert np.isnan(sel[:, :, :64]).all()
+
+
+# ---------------------------------------------------------------- low-rank ----
+
+def test_summary_form_equals_explicit_quadratic_form(oracle):
+    """T2 / Prop. exact, Step 2: q~_p^T C equals sum_q (q~_p . k~_q) v_q."""
+    O = oracle
+    cfg = small_cfg(T=2, Hh=6, Ww=9, r=32)
+    x = draw(cfg)
+    C, z = O.lowrank_summary(cfg, x["k"], x["v"], x["P_k"])
+    y = O.lowrank_readout(cfg, x["q"], x["P_q"], C)
+    y2 = O.lowrank_explicit(cfg, x["q"], x["k"], x["v"], x["P_q"], x["P_k"])
+    np.testing.assert_allclose(y, y2, rtol=1e-10, atol=1e-10)
+    kt = O.lowrank_features(cfg, x["k"], x["P_k"])
+    np.testing.assert_allclose(z, kt.sum(axis=2), rtol=1e-12, atol=1e-12)
+
+
+def test_features_identity_projection_reduces_to_silu_then_rope(oracle):
+    """With r = d_h and P = I the feature map of Eq. (qklr) is R(p) SiLU(x): torch's
+    SiLU, then the full RoPE; the inside variant is SiLU(R(p) x)."""
+    O = oracle
+    cfg = small_cfg(r=128)
+    x = draw(cfg)
+    P = np.broadcast_to(np.eye(128, dtype=np.float32), (cfg["H"], 128, 128)).copy()
+    silu = torch.nn.functional.silu(torch.from_numpy(x["k"]).double()).numpy()
+    got = O.lowrank_features(cfg, x["k"], P)
+    want = np.stack([np.stack([O.rotate(cfg, 64, O.position(cfg, n), silu[0, h, n])
+                               for n in range(cfg["N"])]) for h in range(cfg["H"])])[None]
+    np.testing.assert_allclose(got, want, rtol=1e-13, atol=1e-14)
+    inside = O.lowrank_features(cfg, x["k"], P, rope_mode=O.ROPE_INSIDE)
+    want_in = torch.nn.functional.silu(torch.from_numpy(O.rope_full(cfg, x["k"]))).numpy()
+    np.testing.assert_allclose(inside, want_in, rtol=1e-13, atol=1e-14)
+    none = O.lowrank_features(cfg, x["k"], P, rope_mode=O.ROPE_NONE)
+    np.testing.assert_allclose(none, silu, rtol=1e-13, atol=1e-14)
+
+
+def test_projection_is_a_matmul(oracle):
+    """With RoPE removed the feature map is SiLU(x P^T) (torch matmul + silu)."""
+    O = oracle
+    cfg = small_cfg(r=48)
+    x = draw(cfg)
+    got = O.lowrank_features(cfg, x["q"], x["P_q"], rope_mode=O.ROPE_NONE)
+    q = torch.from_numpy(x["q"]).double()
+    P = torch.from_numpy(x["P_q"]).double()
+    want = torch.nn.functional.silu(torch.einsum("bhnd,hrd->bhnr", q, P)).numpy()
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-13)
+
+
+def shift_residual(O, cfg, x, rope_mode, delta):
+    a = O.forward(cfg, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], rope_mode=rope_mode)
+    b = O.forward(dict(cfg, pos_offset=delta), x["q"], x["k"], x["v"], x["P_q"], x["P_k"],
+                  x["gate"], rope_mode=rope_mode)
+    assert (a["kv_idx"] == b["kv_idx"]).all()
+    return np.linalg.norm(a["o"] - b["o"]) / np.linalg.norm(a["o"])
+
+
+def test_module_shift_invariance_outside_vs_inside(oracle):
+    """T5 / T6 (Eq. shiftinv, Prop. exact vs Prop. inside, Sec. 5.2 shift test): with
+    RoPE outside SiLU the whole module is invariant under a uniform shift of all
+    positions; with RoPE inside it is not; with no RoPE the low-rank branch is
+    position-blind.  The shift moves t, the only axis the r = 16 schedule sees."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=6, Ww=8, r=16, keep=0.25)
+    x = draw(cfg)
+    x["gate"] = np.full((1, cfg["N"]), 0.9, np.float32)   # make the low-rank branch matter
+    out = shift_residual(O, cfg, x, O.ROPE_OUTSIDE, (7, 3, -2))
+    ins = shift_residual(O, cfg, x, O.ROPE_INSIDE, (7, 3, -2))
+    non = shift_residual(O, cfg, x, O.ROPE_NONE, (7, 3, -2))
+    assert out < 1e-12
+    assert non < 1e-12
+    assert ins > 1e-3
+
+
+def test_truncation_bound(oracle):
+    """T7 / Prop. truncation-bound: for full-dimensional position-free features,
+    |Phi^T R(q-p) Psi - Phi_<=r^T R_r(q-p) Psi_<=r| <= ||Phi_>r|| ||Psi_>r||,
+    with equality to zero at r = d_h."""
+    O = oracle
+    cfg = configs.get("tiny")
+    rng = np.random.default_rng(3)
+    for _ in range(20):
+        phi, psi = rng.standard_normal(128), rng.standard_normal(128)
+        d = rng.integers(-20, 20, size=3).astype(float)
+        full = phi @ O.rotate(cfg, 64, d, psi)
+        for r in (16, 32, 64, 128):
+            tr = phi[:r] @ O.rotate(cfg, r // 2, d, psi[:r].copy())[:r]
+            bound = np.linalg.norm(phi[r:]) * np.linalg.norm(psi[r:])
+            assert abs(full - tr) <= bound + 1e-12
+            if r == 128:
+                assert abs(full - tr) < 1e-12
+
+
+# ---------------------------------------------------------------- fusion ------
+
+def test_fusion_identities(oracle):
+    """T8 / Eq. (gate): g = 0 gives O = O^s exactly; O is affine in g with slope
+    r_p O^lr, r_p = sqrt(mean O^s^2 + eps), and O^lr = RMSNorm(y) is torch's
+    rms_norm of the readout; O^s = 0 leaves g sqrt(eps) O^lr."""
+    O = oracle
+    cfg = small_cfg(T=2, Hh=6, Ww=9, r=32)
+    x = draw(cfg)
+    C, _ = O.lowrank_summary(cfg, x["k"], x["v"], x["P_k"])
+    rng = np.random.default_rng(4)
+    o_s = (0.05 * rng.standard_normal(x["q"].shape)).astype(np.float32)
+    N = cfg["N"]
+    g0, g1, gh = (np.full((1, N), g, np.float32) for g in (0.0, 1.0, 0.5))
+    o0 = O.lowrank_apply(cfg, x["q"], x["P_q"], C, g0, o_s)
+    o1 = O.lowrank_apply(cfg, x["q"], x["P_q"], C, g1, o_s)
+    oh = O.lowrank_apply(cfg, x["q"], x["P_q"], C, gh, o_s)
+    np.testing.assert_allclose(o0, o_s.astype(np.float64), rtol=1e-15, atol=0)
+    np.testing.assert_allclose(oh, 0.5 * (o0 + o1), rtol=1e-13, atol=1e-15)
+    y = torch.from_numpy(O.lowrank_readout(cfg, x["q"], x["P_q"], C))
+    olr = torch.nn.functional.rms_norm(y, (128,), eps=float(np.float32(1e-6))).numpy()
+    osd = torch.from_numpy(o_s).double()
+    rp = torch.sqrt(osd.pow(2).mean(-1, keepdim=True) + float(np.float32(1e-6))).numpy()
+    np.testing.assert_allclose(o1 - o0, rp * olr, rtol=1e-11, atol=1e-14)
+    zero = O.lowrank_apply(cfg, x["q"], x["P_q"], C, gh, np.zeros_like(o_s))
+    np.testing.assert_allclose(zero, 0.5 * math.sqrt(float(np.float32(1e-6))) * olr, rtol=1e-11)
+
+
+def test_default_gate_is_one_eighth(oracle):
+    """Tab. (hyper) initialises the gate bias at -1.946, i.e. -ln 7 to 3 decimals, so the
+    default gate sigmoid(b_g) is 1/8; gate = NULL must use it."""
+    with open(os.path.join(GOLDEN, "paper_constants.json")) as f:
+        gold = json.load(f)
+    b = gold["gate_bias_init"]["value"]
+    assert b == pytest.approx(-math.log(7.0), abs=5e-4)
+    O = oracle
+    cfg = small_cfg(T=1, Hh=8, Ww=8, r=16)
+    x = draw(cfg)
+    C, _ = O.lowrank_summary(cfg, x["k"], x["v"], x["P_k"])
+    o_s = np.full(x["q"].shape, 0.1, np.float32)
+    g = np.full((1, cfg["N"]), 1.0 / (1.0 + math.exp(-np.float32(b))), np.float32)
+    a = O.lowrank_apply(cfg, x["q"], x["P_q"], C, None, o_s)
+    bb = O.lowrank_apply(cfg, x["q"], x["P_q"], C, g, o_s)
+    np.testing.assert_allclose(a, bb, rtol=1e-7)
