@@ -1,0 +1,399 @@
+"""Benchmark of the RoLA attention layer on GB300.
+
+One step = one pass of the whole module (block mask, low-rank summary, sparse
+branch, readout + fusion) over one Wan2.1-14B 720p-shaped layer (B=1, 40 heads,
+21 x 45 x 80 = 75600 tokens, d_h=128, 90 % block sparsity, r=32) with seeded
+synthetic bf16 inputs already resident in HBM.  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload wan14b_720p] [--no-dense] [--no-cpu]
+
+Under torchrun each rank runs its own replica layer (the module shards by
+(batch, head) with no exchange, so there is no data-path collective); value is
+the tokens of all ranks divided by the slowest rank's time.
+`--impl reference` times the fp64 CPU oracle on a bounded sample of the same
+workload on the host cores (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "RoLA attn layer ms & tokens/s (Wan2.1-14B 720p shape); % of TC/HBM roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- accounting
+
+def sparse_flops_from_mask(kv_idx, N, block=64, d_h=128):
+    """Algorithmic FLOPs of the sparse branch: 4 d_h sum_{h,i} |Q_i| sum_{j kept} |K_j|
+    (QK^T and PV, 2 flops per multiply-add), with the ragged last block counted
+    at its real size (App. D, C_sparse = 4 B H L^2 (1-S) d_h)."""
+    import torch
+    nB = kv_idx.shape[-2]
+    sizes = torch.full((nB,), block, dtype=torch.float64, device=kv_idx.device)
+    sizes[-1] = N - (nB - 1) * block
+    keys = sizes[kv_idx.long()].sum(dim=-1)            # [B,H,nQB] kept keys per query block
+    return float(4.0 * d_h * (keys * sizes).sum().item())
+
+
+def lowrank_flops(B, H, N, d_h, r):
+    """App. D: C_lowrank = 8 B H L d_h r (projections, context, readout)."""
+    return 8.0 * B * H * N * d_h * r
+
+
+def summary_bytes(B, H, N, d_h, esize=2):
+    """HBM bytes the summary must move: read k and v once."""
+    return 2.0 * B * H * N * d_h * esize
+
+
+# ----------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.tmp = None
+
+    def start(self):
+        try:
+            self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.tmp, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.tmp.flush()
+        self.tmp.seek(0)
+        rows = [r for r in csv.reader(io.StringIO(self.tmp.read())) if len(r) >= 9]
+        os.unlink(self.tmp.name)
+        sm, smax, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+                power.append(float(r[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        load = [x for x in sm if x > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(load), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# ----------------------------------------------------------------- CPU oracle baseline
+
+def oracle_sample_time(cfg, heads, qblocks):
+    """Wall time of the oracle forward on `heads` heads of the layer and the given
+    query blocks (mask, summary and RoPE over the whole sequence of those heads)."""
+    import torch
+    from oracle import oracle as O
+    from paper_2609_06712_gb300 import inputs
+    sub = dict(cfg, H=heads)
+    x = inputs.make_inputs(sub, dtype=torch.bfloat16)
+    h = {k: (None if v is None else v.float().numpy()) for k, v in x.items()}
+    t0 = time.perf_counter()
+    O.forward(sub, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], qblocks=qblocks)
+    return time.perf_counter() - t0
+
+
+def cpu_oracle_estimate(cfg, heads=None, q_lo=2, q_hi=6):
+    """Layer time of the oracle extrapolated from a bounded sample: `heads` heads in
+    parallel with q_lo and q_hi query blocks each; the difference gives the
+    per-query-block cost, the rest the per-head fixed cost (mask, summary)."""
+    from oracle import oracle as O
+    O.build()
+    cores = os.cpu_count() or 1
+    heads = heads or min(cfg["H"], cores)
+    nB = (cfg["N"] + cfg["block"] - 1) // cfg["block"]
+    t_lo = oracle_sample_time(cfg, heads, list(range(q_lo)))
+    t_hi = oracle_sample_time(cfg, heads, list(range(q_hi)))
+    per_block = max(t_hi - t_lo, 0.0) / (q_hi - q_lo)
+    fixed = max(t_lo - q_lo * per_block, 0.0)
+    layer_s = (cfg["H"] / heads) * (fixed + nB * per_block)
+    tokens_s = cfg["B"] * cfg["N"] / layer_s
+    sample = (f"fp64 oracle on {heads} of {cfg['H']} heads (full-sequence mask, RoPE and summary) with "
+              f"{q_lo} and {q_hi} of {nB} query blocks; layer time extrapolated per query block and per head")
+    return {"value": tokens_s, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample,
+            "layer_s_est": layer_s, "sample_s": t_lo + t_hi}
+
+
+# ----------------------------------------------------------------- main
+
+def dist_setup(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        import torch
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return ws, rank, local
+
+
+def reduce_max(x, ws):
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def run_reference(args, cfg, ws, rank):
+    if rank != 0:
+        return
+    from oracle import oracle as O
+    O.build()
+    times = []
+    est = None
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        est = cpu_oracle_estimate(cfg, q_lo=1, q_hi=3)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": est["value"], "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * est["layer_s_est"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg["name"], "B": cfg["B"], "H": cfg["H"], "N": cfg["N"],
+                   "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "keep": cfg["keep"], "r": cfg["r"]},
+        "cpu_baseline": {"value": est["value"], "unit": "tokens/s", "cores": est["cores"], "kind": "oracle",
+                         "sample": est["sample"], "wall_s_per_step": statistics.median(times)},
+        "e2e": {"value": est["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="wan14b_720p")
+    ap.add_argument("--keep", type=float, default=None)
+    ap.add_argument("--r", type=int, default=None)
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    from paper_2609_06712_gb300 import configs
+    over = {}
+    if args.keep is not None:
+        over["keep"] = args.keep
+    if args.r is not None:
+        over["r"] = args.r
+    cfg = configs.get(args.workload, **over)
+    ws, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, cfg, ws, rank)
+        return
+
+    import torch
+    from paper_2609_06712_gb300 import build as rbuild
+    rbuild.build()
+    from paper_2609_06712_gb300 import inputs, rola
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    x = inputs.make_inputs(cfg, dtype=torch.bfloat16, device=dev, seed=cfg["seed"] + 1000 * rank)
+    c = rola.make_config(cfg)
+    wsb = rola.workspace(c, dev)
+    nB, nk = rola.num_blocks(c), rola.num_keep(c)
+    o = torch.empty_like(x["q"])
+    kv = torch.empty((cfg["B"], cfg["H"], nB, nk), dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    for row in evs:
+        for e in row:
+            e.record(stream)
+    args_fw = (c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kv, wsb)
+
+    for _ in range(args.warmup):
+        rola.forward(*args_fw)
+    torch.cuda.synchronize()
+    assert rola.get_device_status(wsb) == rola.ROLA_OK
+
+    # ---- device-timed region: inputs resident in HBM (each of q, k, v > L2)
+    clocks = ClockSampler(local)
+    barrier(ws)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(K):
+        rola.forward_timed(*args_fw, evs[i])
+    stop.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(ws)
+    ms_total = start.elapsed_time(stop)
+    ms_step = reduce_max(ms_total / K, ws)
+    stage_names = ["mask", "summary", "sparse_attn", "apply_fuse"]
+    stage_ms = {n: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K))
+                for j, n in enumerate(stage_names)}
+    assert rola.get_device_status(wsb) == rola.ROLA_OK
+    tokens = cfg["B"] * cfg["N"]
+    value = ws * tokens / (ms_step * 1e-3)
+
+    # ---- roofline of the dominant kernel (the sparse branch: tensor-core bound)
+    peaks, peak_src = load_peaks()
+    fl = sparse_flops_from_mask(kv, cfg["N"])
+    sp_ms = stage_ms["sparse_attn"]
+    achieved = fl / (sp_ms * 1e-3) / 1e12
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    roofline = {"bound": "tensor", "kernel": "sparse_attn", "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "peak_source": f"{peak_src} bf16_tflops_sustained",
+                "algorithmic_flops_per_launch": fl, "ms_per_launch": sp_ms}
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    sb = summary_bytes(cfg["B"], cfg["H"], cfg["N"], 128)
+    secondary = {
+        "summary": {"bound": "hbm", "achieved_gbs": sb / (stage_ms["summary"] * 1e-3) / 1e9, "peak_gbs": hbm,
+                    "frac": sb / (stage_ms["summary"] * 1e-3) / 1e9 / hbm, "bytes": sb},
+        "mask": {"bound": "hbm", "achieved_gbs": sb / (stage_ms["mask"] * 1e-3) / 1e9, "peak_gbs": hbm,
+                 "frac": sb / (stage_ms["mask"] * 1e-3) / 1e9 / hbm, "bytes": sb,
+                 "note": "algorithmic bytes = read q and k once"},
+        "apply_fuse": {"bound": "hbm",
+                       "achieved_gbs": 1.5 * sb / (stage_ms["apply_fuse"] * 1e-3) / 1e9, "peak_gbs": hbm,
+                       "frac": 1.5 * sb / (stage_ms["apply_fuse"] * 1e-3) / 1e9 / hbm, "bytes": 1.5 * sb,
+                       "note": "read q and O^s, write O"},
+    }
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        host = {k: (None if v is None else v.cpu().pin_memory()) for k, v in x.items()}
+        o_host = torch.empty(o.shape, dtype=o.dtype, pin_memory=True)
+        dbuf = {k: (None if v is None else torch.empty_like(v)) for k, v in x.items()}
+        h2d = sum(v.numel() * v.element_size() for v in host.values() if v is not None)
+        d2h = o_host.numel() * o_host.element_size()
+
+        def e2e_step():
+            for kk, v in host.items():
+                if v is not None:
+                    dbuf[kk].copy_(v, non_blocking=True)
+            rola.forward(c, dbuf["q"], dbuf["k"], dbuf["v"], dbuf["P_q"], dbuf["P_k"], dbuf["gate"], o, kv, wsb)
+            o_host.copy_(o, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(ws)
+        s2, t2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        ke = max(2, K // 2)
+        for _ in range(ke):
+            e2e_step()
+        t2.record(stream)
+        torch.cuda.synchronize()
+        e_ms = reduce_max(s2.elapsed_time(t2) / ke, ws)
+        e2e = {"value": ws * tokens / (e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e_ms,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+        del dbuf
+
+    # ---- dense comparator: the same kernels with every block kept
+    dense = None
+    if not args.no_dense:
+        cd = rola.make_config(dict(cfg, keep=1.0))
+        wsd = rola.workspace(cd, dev)
+        kvd = torch.empty((cfg["B"], cfg["H"], nB, nB), dtype=torch.int32, device=dev)
+        rola.forward(cd, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kvd, wsd)
+        torch.cuda.synchronize()
+        s3, t3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s3.record(stream)
+        for _ in range(2):
+            rola.forward(cd, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kvd, wsd)
+        t3.record(stream)
+        torch.cuda.synchronize()
+        d_ms = s3.elapsed_time(t3) / 2
+        flop_ratio = (sparse_flops_from_mask(kvd, cfg["N"]) + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"])) / \
+            (fl + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"]))
+        dense = {"dense_ms": d_ms, "speedup": d_ms / ms_step, "flop_ratio": flop_ratio,
+                 "target_speedup": 0.85 * flop_ratio}
+        del wsd, kvd
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        cpu = cpu_oracle_estimate(cfg)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": K, "warmup": args.warmup,
+            "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": cfg["name"], "B": cfg["B"], "H": cfg["H"], "N": cfg["N"],
+                       "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "block": 64, "keep": cfg["keep"],
+                       "n_keep": nk, "r": cfg["r"], "d_h": 128,
+                       "l2": "no flush: q, k, v are each larger than L2 (774 MB vs 129 MB)",
+                       "parallelism": f"replica per GPU x{ws}"},
+            "stage_ms": stage_ms,
+            "roofline": roofline,
+            "roofline_other": secondary,
+            "dense": dense,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": 8 * K,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

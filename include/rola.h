@@ -169,6 +169,19 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
                            int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * rola_forward with stage timing: identical computation and launches, plus
+ * cudaEventRecord(stage_events[i], stream) at five stage boundaries --
+ *   [0] start  [1] after the block mask  [2] after the low-rank summary
+ *   [3] after the sparse branch  [4] after the readout + fusion.
+ * stage_events: array of 5 cudaEvent_t created by the caller (owned by the
+ * caller), or NULL (then this is rola_forward).
+ */
+rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                                 const void* P_q, const void* P_k, const float* gate, void* o,
+                                 int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream,
+                                 void* const* stage_events);
+
+/*
  * Synchronises `stream`, then reads the device status word at the start of
  * ws: ROLA_OK, or ROLA_ERR_TIMEOUT if a bounded device wait expired since the
  * workspace was last cleared by an entry point.  ROLA_ERR_CUDA if the

@@ -100,20 +100,52 @@ double orc_pair_angle(const orc_cfg* c, int m, const double pos[3])
     return pos[axis] * freq;
 }
 
-/* out = R(pos) restricted to the first 2*npairs coordinates, applied to in.
- * Coordinates beyond 2*npairs are copied unchanged.  in / out of length len
- * may alias. */
-void orc_rotate(const orc_cfg* c, int npairs, const double pos[3], const double* in,
-                double* out, int len)
+/* Turn the first npairs coordinate pairs of in by the angles whose (cos, sin)
+ * are cs[2m], cs[2m+1]; coordinates beyond 2*npairs are copied unchanged.
+ * in / out of length len may alias. */
+static void rotate_pairs(int npairs, const double* cs, const double* in, double* out, int len)
 {
     for (int m = 0; m < npairs; ++m) {
-        double a = orc_pair_angle(c, m, pos);
-        double ca = cos(a), sa = sin(a);
+        double ca = cs[2 * m], sa = cs[2 * m + 1];
         double x = in[2 * m], y = in[2 * m + 1];
         out[2 * m] = x * ca - y * sa;
         out[2 * m + 1] = x * sa + y * ca;
     }
     for (int i = 2 * npairs; i < len; ++i) out[i] = in[i];
+}
+
+/* (cos, sin) of every pair angle at position pos: cs[2m], cs[2m+1], m < dh/2. */
+static void pair_cs(const orc_cfg* c, const double pos[3], double* cs)
+{
+    for (int m = 0; m < c->dh / 2; ++m) {
+        double a = orc_pair_angle(c, m, pos);
+        cs[2 * m] = cos(a);
+        cs[2 * m + 1] = sin(a);
+    }
+}
+
+/* out = R(pos) restricted to the first 2*npairs coordinates, applied to in. */
+void orc_rotate(const orc_cfg* c, int npairs, const double pos[3], const double* in,
+                double* out, int len)
+{
+    double* cs = (double*)malloc(sizeof(double) * (size_t)c->dh);
+    pair_cs(c, pos, cs);
+    rotate_pairs(npairs, cs, in, out, len);
+    free(cs);
+}
+
+/* The same (cos, sin) for every token position, computed once per call:
+ * tcs[n*dh + 2m + {0,1}]. */
+static double* token_cs(const orc_cfg* c)
+{
+    double* tcs = (double*)malloc(sizeof(double) * (size_t)c->N * c->dh);
+#pragma omp parallel for schedule(static)
+    for (int n = 0; n < c->N; ++n) {
+        double pos[3];
+        orc_position(c, n, pos);
+        pair_cs(c, pos, tcs + (size_t)n * c->dh);
+    }
+    return tcs;
 }
 
 static double silu(double x) { return x / (1.0 + exp(-x)); }
@@ -122,12 +154,11 @@ static double silu(double x) { return x / (1.0 + exp(-x)); }
 /* low-rank features, Eq. (qklr) and its two ablations                */
 /* ------------------------------------------------------------------ */
 
-/* feat[r] for one token: x [dh] (float input), P [r][dh] (one head). */
-static void lowrank_feature(const orc_cfg* c, int n, const float* x, const float* P, double* feat)
+/* feat[r] for one token: cs its pair (cos, sin), x [dh] (float input), P [r][dh] (one head). */
+static void lowrank_feature(const orc_cfg* c, const double* cs, const float* x, const float* P,
+                            double* feat)
 {
     int r = c->r, dh = c->dh;
-    double pos[3];
-    orc_position(c, n, pos);
     double* u = (double*)malloc(sizeof(double) * (size_t)r);
     for (int a = 0; a < r; ++a) {
         double s = 0.0;
@@ -136,9 +167,9 @@ static void lowrank_feature(const orc_cfg* c, int n, const float* x, const float
     }
     if (c->rope_mode == 0) {            /* R_r(p) SiLU(P x) */
         for (int a = 0; a < r; ++a) u[a] = silu(u[a]);
-        orc_rotate(c, r / 2, pos, u, feat, r);
+        rotate_pairs(r / 2, cs, u, feat, r);
     } else if (c->rope_mode == 1) {     /* SiLU(R_r(p) P x) */
-        orc_rotate(c, r / 2, pos, u, feat, r);
+        rotate_pairs(r / 2, cs, u, feat, r);
         for (int a = 0; a < r; ++a) feat[a] = silu(feat[a]);
     } else {                            /* SiLU(P x) */
         for (int a = 0; a < r; ++a) feat[a] = silu(u[a]);
@@ -150,13 +181,15 @@ static void lowrank_feature(const orc_cfg* c, int n, const float* x, const float
 void orc_lowrank_features(const orc_cfg* c, const float* x, const float* P, double* out)
 {
     int BH = c->B * c->H;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         int h = bh % c->H;
         for (int n = 0; n < c->N; ++n)
-            lowrank_feature(c, n, x + ((size_t)bh * c->N + n) * c->dh,
+            lowrank_feature(c, tcs + (size_t)n * c->dh, x + ((size_t)bh * c->N + n) * c->dh,
                             P + (size_t)h * c->r * c->dh, out + ((size_t)bh * c->N + n) * c->r);
     }
+    free(tcs);
 }
 
 /* ------------------------------------------------------------------ */
@@ -167,6 +200,7 @@ void orc_lowrank_summary(const orc_cfg* c, const float* k, const float* v, const
                          double* C, double* z)
 {
     int BH = c->B * c->H, r = c->r, dh = c->dh;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         int h = bh % c->H;
@@ -176,7 +210,8 @@ void orc_lowrank_summary(const orc_cfg* c, const float* k, const float* v, const
         memset(Cb, 0, sizeof(double) * (size_t)r * dh);
         if (zb) memset(zb, 0, sizeof(double) * (size_t)r);
         for (int n = 0; n < c->N; ++n) {
-            lowrank_feature(c, n, k + ((size_t)bh * c->N + n) * dh, Pk + (size_t)h * r * dh, kt);
+            lowrank_feature(c, tcs + (size_t)n * dh, k + ((size_t)bh * c->N + n) * dh,
+                            Pk + (size_t)h * r * dh, kt);
             const float* vn = v + ((size_t)bh * c->N + n) * dh;
             for (int a = 0; a < r; ++a) {
                 for (int d = 0; d < dh; ++d) Cb[(size_t)a * dh + d] += kt[a] * (double)vn[d];
@@ -185,6 +220,7 @@ void orc_lowrank_summary(const orc_cfg* c, const float* k, const float* v, const
         }
         free(kt);
     }
+    free(tcs);
 }
 
 /* ------------------------------------------------------------------ */
@@ -198,13 +234,13 @@ static double gate_value(const orc_cfg* c, const float* gate, int b, int n)
 }
 
 /* O^lr for token n of head bh into olr[dh]; y (pre-RMSNorm) into y if non-NULL. */
-static void lowrank_readout(const orc_cfg* c, int bh, int n, const float* q, const float* Pq,
-                            const double* C, double* olr, double* y)
+static void lowrank_readout(const orc_cfg* c, const double* tcs, int bh, int n, const float* q,
+                            const float* Pq, const double* C, double* olr, double* y)
 {
     int r = c->r, dh = c->dh, h = bh % c->H;
     double* qt = (double*)malloc(sizeof(double) * (size_t)r);
     double* yy = (double*)malloc(sizeof(double) * (size_t)dh);
-    lowrank_feature(c, n, q + ((size_t)bh * c->N + n) * dh, Pq + (size_t)h * r * dh, qt);
+    lowrank_feature(c, tcs + (size_t)n * dh, q + ((size_t)bh * c->N + n) * dh, Pq + (size_t)h * r * dh, qt);
     const double* Cb = C + (size_t)bh * r * dh;
     double ss = 0.0;
     for (int d = 0; d < dh; ++d) {
@@ -244,6 +280,7 @@ void orc_lowrank_apply(const orc_cfg* c, const float* q, const float* Pq, const 
                        const float* gate, const float* o_s, const uint8_t* qb_sel, double* o)
 {
     int BH = c->B * c->H, dh = c->dh;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         int b = bh / c->H;
@@ -252,23 +289,26 @@ void orc_lowrank_apply(const orc_cfg* c, const float* q, const float* Pq, const 
         for (int n = 0; n < c->N; ++n) {
             if (!token_in_selection(c, n, qb_sel)) continue;
             size_t off = ((size_t)bh * c->N + n) * dh;
-            lowrank_readout(c, bh, n, q, Pq, C, olr, NULL);
+            lowrank_readout(c, tcs, bh, n, q, Pq, C, olr, NULL);
             for (int d = 0; d < dh; ++d) os[d] = (double)o_s[off + d];
             fuse(c, os, olr, gate_value(c, gate, b, n), o + off);
         }
         free(olr);
         free(os);
     }
+    free(tcs);
 }
 
 /* Pre-RMSNorm readout y_p = q~_p^T C for every token: y [B][H][N][dh]. */
 void orc_lowrank_readout(const orc_cfg* c, const float* q, const float* Pq, const double* C, double* y)
 {
     int BH = c->B * c->H;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh)
         for (int n = 0; n < c->N; ++n)
-            lowrank_readout(c, bh, n, q, Pq, C, NULL, y + ((size_t)bh * c->N + n) * c->dh);
+            lowrank_readout(c, tcs, bh, n, q, Pq, C, NULL, y + ((size_t)bh * c->N + n) * c->dh);
+    free(tcs);
 }
 
 /* Explicit O(N^2) form of the pre-RMSNorm low-rank output,
@@ -277,16 +317,18 @@ void orc_lowrank_explicit(const orc_cfg* c, const float* q, const float* k, cons
                           const float* Pq, const float* Pk, double* y)
 {
     int BH = c->B * c->H, r = c->r, dh = c->dh, N = c->N;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         int h = bh % c->H;
         double* kt = (double*)malloc(sizeof(double) * (size_t)N * r);
         double* qt = (double*)malloc(sizeof(double) * (size_t)r);
         for (int n = 0; n < N; ++n)
-            lowrank_feature(c, n, k + ((size_t)bh * N + n) * dh, Pk + (size_t)h * r * dh,
-                            kt + (size_t)n * r);
+            lowrank_feature(c, tcs + (size_t)n * dh, k + ((size_t)bh * N + n) * dh,
+                            Pk + (size_t)h * r * dh, kt + (size_t)n * r);
         for (int p = 0; p < N; ++p) {
-            lowrank_feature(c, p, q + ((size_t)bh * N + p) * dh, Pq + (size_t)h * r * dh, qt);
+            lowrank_feature(c, tcs + (size_t)p * dh, q + ((size_t)bh * N + p) * dh,
+                            Pq + (size_t)h * r * dh, qt);
             double* yp = y + ((size_t)bh * N + p) * dh;
             for (int d = 0; d < dh; ++d) yp[d] = 0.0;
             for (int n = 0; n < N; ++n) {
@@ -299,6 +341,7 @@ void orc_lowrank_explicit(const orc_cfg* c, const float* q, const float* k, cons
         free(kt);
         free(qt);
     }
+    free(tcs);
 }
 
 /* ------------------------------------------------------------------ */
@@ -309,18 +352,18 @@ void orc_lowrank_explicit(const orc_cfg* c, const float* q, const float* k, cons
 void orc_rope_full(const orc_cfg* c, const float* x, double* xr)
 {
     int BH = c->B * c->H, dh = c->dh;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         double* tmp = (double*)malloc(sizeof(double) * (size_t)dh);
         for (int n = 0; n < c->N; ++n) {
-            double pos[3];
-            orc_position(c, n, pos);
             size_t off = ((size_t)bh * c->N + n) * dh;
             for (int d = 0; d < dh; ++d) tmp[d] = (double)x[off + d];
-            orc_rotate(c, dh / 2, pos, tmp, xr + off, dh);
+            rotate_pairs(dh / 2, tcs + (size_t)n * dh, tmp, xr + off, dh);
         }
         free(tmp);
     }
+    free(tcs);
 }
 
 /* ------------------------------------------------------------------ */
@@ -365,6 +408,7 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
     int nB = orc_num_blocks(c), nk = orc_num_keep(c);
     double isd = 1.0 / sqrt((double)dh);
     const double u = ldexp(1.0, -24);
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         size_t nbd = (size_t)nB * dh;
@@ -380,11 +424,9 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
             double* mean = which == 0 ? qb : kb;
             double* mag = which == 0 ? qa : ka;
             for (int n = 0; n < N; ++n) {
-                double pos[3];
-                orc_position(c, n, pos);
                 size_t off = ((size_t)bh * N + n) * dh;
                 for (int d = 0; d < dh; ++d) xi[d] = (double)x[off + d];
-                orc_rotate(c, dh / 2, pos, xi, xr, dh);
+                rotate_pairs(dh / 2, tcs + (size_t)n * dh, xi, xr, dh);
                 int blk = n / bs;
                 for (int d = 0; d < dh; ++d) {
                     mean[(size_t)blk * dh + d] += xr[d];
@@ -429,6 +471,7 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
         }
         free(qb); free(kb); free(qa); free(ka); free(xr); free(xi); free(row);
     }
+    free(tcs);
 }
 
 /* ------------------------------------------------------------------ */
@@ -523,6 +566,7 @@ void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* 
     orc_lowrank_summary(c, k, v, Pk, C, z);
 
     int BH = c->B * c->H, dh = c->dh;
+    double* tcs = token_cs(c);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         int b = bh / c->H;
@@ -530,11 +574,12 @@ void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* 
         for (int n = 0; n < c->N; ++n) {
             if (!token_in_selection(c, n, qb_sel)) continue;
             size_t off = ((size_t)bh * c->N + n) * dh;
-            lowrank_readout(c, bh, n, q, Pq, C, olr, NULL);
+            lowrank_readout(c, tcs, bh, n, q, Pq, C, olr, NULL);
             fuse(c, os + off, olr, gate_value(c, gate, b, n), o + off);
         }
         free(olr);
     }
+    free(tcs);
     if (o_s_out) memcpy(o_s_out, os, sizeof(double) * nel);
     if (C_out) memcpy(C_out, C, sizeof(double) * nC);
     if (z_out) memcpy(z_out, z, sizeof(double) * (size_t)c->B * c->H * c->r);

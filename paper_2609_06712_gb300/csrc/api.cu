@@ -1,0 +1,308 @@
+// C ABI entry points of include/rola.h: validation, workspace layout, launches.
+#include <math.h>
+#include <string.h>
+
+#include "common.cuh"
+
+using namespace rola;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int num_blocks_of(const rola_config_t& c) { return (c.N + c.block - 1) / c.block; }
+
+int num_keep_of(const rola_config_t& c)
+{
+    int nkb = num_blocks_of(c);
+    double x = floor((double)c.keep_ratio * (double)nkb + 0.5);
+    int n = (int)x;
+    if (n < 1) n = 1;
+    if (n > nkb) n = nkb;
+    return n;
+}
+
+// Returns ROLA_OK if the configuration is one the kernels handle.
+rola_status_t validate(const rola_config_t* c)
+{
+    if (!c) return ROLA_ERR_INVALID_ARG;
+    if (c->B < 1 || c->H < 1 || c->N < 1 || c->T < 1 || c->Hh < 1 || c->Ww < 1) return ROLA_ERR_INVALID_ARG;
+    if ((int64_t)c->T * c->Hh * c->Ww != c->N) return ROLA_ERR_INVALID_ARG;
+    if (c->dtype != ROLA_BF16 && c->dtype != ROLA_FP32) return ROLA_ERR_INVALID_ARG;
+    if (c->d_h != kDh) return c->d_h > 0 ? ROLA_ERR_UNSUPPORTED : ROLA_ERR_INVALID_ARG;
+    if (c->block != kBlock) return c->block > 0 ? ROLA_ERR_UNSUPPORTED : ROLA_ERR_INVALID_ARG;
+    for (int a = 0; a < 3; ++a)
+        if (c->rope_split[a] < 0 || (c->rope_split[a] & 1)) return ROLA_ERR_INVALID_ARG;
+    if (c->rope_split[0] + c->rope_split[1] + c->rope_split[2] != c->d_h) return ROLA_ERR_INVALID_ARG;
+    if (!(c->rope_theta > 0.0) || !isfinite(c->rope_theta)) return ROLA_ERR_INVALID_ARG;
+    if (!(c->keep_ratio >= 0.0f && c->keep_ratio <= 1.0f)) return ROLA_ERR_INVALID_ARG;
+    if (c->r < 2 || (c->r & 1) || c->r > c->d_h) return ROLA_ERR_INVALID_ARG;
+    if (c->r % 16 != 0) return ROLA_ERR_UNSUPPORTED;
+    if (!(c->eps_lr >= 0.0f) || !(c->eps_fuse >= 0.0f) || !isfinite(c->eps_lr) || !isfinite(c->eps_fuse))
+        return ROLA_ERR_INVALID_ARG;
+    if (!isfinite(c->gate_bias)) return ROLA_ERR_INVALID_ARG;
+    for (int a = 0; a < 3; ++a)
+        if (c->pos_offset[a] < -(1 << 20) || c->pos_offset[a] > (1 << 20)) return ROLA_ERR_INVALID_ARG;
+    // grid / index limits of the kernels
+    if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
+    if ((int64_t)c->B * c->H * c->N * c->d_h > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
+    return ROLA_OK;
+}
+
+Shape make_shape(const rola_config_t& c)
+{
+    Shape s;
+    s.B = c.B; s.H = c.H; s.N = c.N; s.r = c.r;
+    s.nB = num_blocks_of(c);
+    s.n_keep = num_keep_of(c);
+    s.T = c.T; s.Hh = c.Hh; s.Ww = c.Ww;
+    s.pt = c.rope_split[0] / 2;
+    s.px = c.rope_split[1] / 2;
+    s.eps_lr = c.eps_lr;
+    s.eps_fuse = c.eps_fuse;
+    s.default_gate = (float)(1.0 / (1.0 + exp(-(double)c.gate_bias)));
+    s.sm_scale_log2 = (float)(1.4426950408889634 / sqrt((double)kDh));
+    return s;
+}
+
+Workspace layout(const rola_config_t& c)
+{
+    Shape s = make_shape(c);
+    size_t esz = c.dtype == ROLA_BF16 ? 2 : 4;
+    size_t bh = (size_t)c.B * c.H;
+    Workspace w;
+    w.nsplit = summary_splits(s);
+    size_t off = 0;
+    w.status = off; off = align_up(off + sizeof(DeviceStatus));
+    w.table = off; off = align_up(off + sizeof(float2) * (size_t)(c.T + c.Hh + c.Ww) * kPairs);
+    w.qr = off; off = align_up(off + esz * bh * c.N * kDh);
+    w.kr = off; off = align_up(off + esz * bh * c.N * kDh);
+    w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
+    w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
+    w.scores = off; off = align_up(off + 4 * bh * s.nB * s.nB);
+    w.kv_idx = off; off = align_up(off + 4 * bh * s.nB * s.n_keep);
+    w.C = off; off = align_up(off + 4 * bh * c.r * kDh);
+    w.z = off; off = align_up(off + 4 * bh * c.r);
+    w.Cbf = off; off = align_up(off + 2 * bh * c.r * kDh);
+    w.partials = off; off = align_up(off + 4 * bh * w.nsplit * ((size_t)c.r * kDh + c.r));
+    w.total = off;
+    return w;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) { return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off); }
+
+rola_status_t check_ws(const rola_config_t& c, const void* ws, size_t ws_bytes)
+{
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1))) return ROLA_ERR_WORKSPACE;
+    if (ws_bytes < layout(c).total) return ROLA_ERR_WORKSPACE;
+    return ROLA_OK;
+}
+
+#define ROLA_TRY(expr)                                  \
+    do {                                                \
+        cudaError_t e_ = (expr);                        \
+        if (e_ != cudaSuccess) return ROLA_ERR_CUDA;    \
+    } while (0)
+
+#define ROLA_CHECK(expr)                                \
+    do {                                                \
+        rola_status_t st_ = (expr);                     \
+        if (st_ != ROLA_OK) return st_;                 \
+    } while (0)
+
+// Start of every entry point: clear the status word, build the RoPE table.
+rola_status_t prologue(const rola_config_t& c, void* ws, const Workspace& w, cudaStream_t st)
+{
+    ROLA_TRY(cudaMemsetAsync(at<uint8_t>(ws, w.status), 0, sizeof(DeviceStatus), st));
+    ROLA_TRY(launch_rope_table(c, at<float2>(ws, w.table), st));
+    return ROLA_OK;
+}
+
+rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& w, const void* q, const void* k,
+                       int32_t* kv_idx, void* ws, cudaStream_t st)
+{
+    ROLA_TRY(launch_rope_pool(c, s, q, k, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
+                              at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
+    ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv_idx,
+                               st));
+    return ROLA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+rola_status_t rola_config_init(rola_config_t* cfg)
+{
+    if (!cfg) return ROLA_ERR_INVALID_ARG;
+    memset(cfg, 0, sizeof(*cfg));
+    cfg->d_h = kDh;
+    cfg->rope_split[0] = 44;
+    cfg->rope_split[1] = 42;
+    cfg->rope_split[2] = 42;
+    cfg->rope_theta = 10000.0;
+    cfg->block = kBlock;
+    cfg->keep_ratio = 0.1f;
+    cfg->r = 32;
+    cfg->eps_lr = 1e-6f;
+    cfg->eps_fuse = 1e-6f;
+    cfg->gate_bias = -1.946f;
+    cfg->dtype = ROLA_BF16;
+    return ROLA_OK;
+}
+
+int32_t rola_num_blocks(const rola_config_t* cfg)
+{
+    if (validate(cfg) != ROLA_OK) return 0;
+    return num_blocks_of(*cfg);
+}
+
+int32_t rola_num_keep(const rola_config_t* cfg)
+{
+    if (validate(cfg) != ROLA_OK) return 0;
+    return num_keep_of(*cfg);
+}
+
+size_t rola_workspace_bytes(const rola_config_t* cfg)
+{
+    if (validate(cfg) != ROLA_OK) return 0;
+    return layout(*cfg).total;
+}
+
+rola_status_t rola_block_mask(const rola_config_t* cfg, const void* q, const void* k, int32_t* kv_idx, void* ws,
+                              size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!q || !k || !kv_idx || !aligned16(q) || !aligned16(k) || !aligned16(kv_idx)) return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    return run_mask(*cfg, s, w, q, k, kv_idx, ws, st);
+}
+
+rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                               const int32_t* kv_idx, void* o_s, void* ws, size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!q || !k || !v || !kv_idx || !o_s) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(kv_idx) || !aligned16(o_s))
+        return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    // rotated copies (the pooled means are a by-product here)
+    ROLA_TRY(launch_rope_pool(*cfg, s, q, k, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
+                              at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv_idx, o_s, st));
+    return ROLA_OK;
+}
+
+rola_status_t rola_lowrank_summary(const rola_config_t* cfg, const void* k, const void* v, const void* P_k, float* C,
+                                   float* z, void* ws, size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!k || !v || !P_k || !C) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(k) || !aligned16(v) || !aligned16(P_k) || !aligned16(C) || (z && !aligned16(z)))
+        return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    ROLA_TRY(launch_lowrank_summary(cfg->dtype, s, w.nsplit, k, v, P_k, at<float2>(ws, w.table),
+                                    at<float>(ws, w.partials), C, z, nullptr, st));
+    return ROLA_OK;
+}
+
+rola_status_t rola_lowrank_apply(const rola_config_t* cfg, const void* q, const void* P_q, const float* C,
+                                 const float* gate, const void* o_s, void* o, void* ws, size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!q || !P_q || !C || !o_s || !o) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(P_q) || !aligned16(C) || !aligned16(o_s) || !aligned16(o) ||
+        (gate && (reinterpret_cast<uintptr_t>(gate) & 3u)))
+        return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    __nv_bfloat16* Cbf = at<__nv_bfloat16>(ws, w.Cbf);
+    if (cfg->dtype == ROLA_BF16) ROLA_TRY(launch_c_to_bf16(s, C, Cbf, st));
+    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, C, Cbf, gate, o_s, o, at<float2>(ws, w.table), st));
+    return ROLA_OK;
+}
+
+rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                                 const void* P_q, const void* P_k, const float* gate, void* o, int32_t* kv_idx_out,
+                                 void* ws, size_t ws_bytes, void* stream, void* const* stage_events)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!q || !k || !v || !P_q || !P_k || !o) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(P_q) || !aligned16(P_k) || !aligned16(o) ||
+        (kv_idx_out && !aligned16(kv_idx_out)) || (gate && (reinterpret_cast<uintptr_t>(gate) & 3u)))
+        return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    auto mark = [&](int i) -> cudaError_t {
+        return stage_events ? cudaEventRecord(static_cast<cudaEvent_t>(stage_events[i]), st) : cudaSuccess;
+    };
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    int32_t* kv = kv_idx_out ? kv_idx_out : at<int32_t>(ws, w.kv_idx);
+    ROLA_TRY(mark(0));
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    ROLA_CHECK(run_mask(*cfg, s, w, q, k, kv, ws, st));
+    ROLA_TRY(mark(1));
+    ROLA_TRY(launch_lowrank_summary(cfg->dtype, s, w.nsplit, k, v, P_k, at<float2>(ws, w.table),
+                                    at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
+                                    at<__nv_bfloat16>(ws, w.Cbf), st));
+    ROLA_TRY(mark(2));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv, o, st));
+    ROLA_TRY(mark(3));
+    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, o,
+                                  o, at<float2>(ws, w.table), st));
+    ROLA_TRY(mark(4));
+    return ROLA_OK;
+}
+
+rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* k, const void* v, const void* P_q,
+                           const void* P_k, const float* gate, void* o, int32_t* kv_idx_out, void* ws,
+                           size_t ws_bytes, void* stream)
+{
+    return rola_forward_timed(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, ws_bytes, stream, nullptr);
+}
+
+rola_status_t rola_get_device_status(const void* ws, void* stream)
+{
+    if (!ws) return ROLA_ERR_WORKSPACE;
+    DeviceStatus h;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(st) != cudaSuccess) return ROLA_ERR_CUDA;
+    if (cudaMemcpy(&h, ws, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess) return ROLA_ERR_CUDA;
+    return h.code == 0 ? ROLA_OK : static_cast<rola_status_t>(h.code);
+}
+
+const char* rola_status_string(rola_status_t status)
+{
+    switch (status) {
+        case ROLA_OK: return "ROLA_OK";
+        case ROLA_ERR_INVALID_ARG: return "ROLA_ERR_INVALID_ARG: bad pointer, shape, alignment or value";
+        case ROLA_ERR_UNSUPPORTED: return "ROLA_ERR_UNSUPPORTED: configuration not built (d_h, block, r)";
+        case ROLA_ERR_WORKSPACE: return "ROLA_ERR_WORKSPACE: workspace NULL, misaligned or too small";
+        case ROLA_ERR_CUDA: return "ROLA_ERR_CUDA: a CUDA launch or runtime call failed";
+        case ROLA_ERR_TIMEOUT: return "ROLA_ERR_TIMEOUT: a device-side bounded wait expired";
+        default: return "unknown rola_status_t";
+    }
+}
+
+}  // extern "C"

@@ -1,0 +1,143 @@
+// Internal declarations shared by the RoLA CUDA translation units.
+//
+// Layout conventions (all tensors dense):
+//   q, k, v, o          [B][H][N][128]      bf16 (ROLA_BF16) or fp32 (ROLA_FP32)
+//   P_q, P_k            [H][r][128]
+//   rotated q^r, k^r    [B][H][N][128]      workspace, storage dtype
+//   pooled q_bar, k_bar [B][H][nB][128]     workspace, fp32
+//   RoPE table          [T + Hh + Ww][64]   float2 (cos, sin) per grid row and pair;
+//                                           row t for temporal pairs, T + x for height
+//                                           pairs, T + Hh + y for width pairs
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/rola.h"
+
+namespace rola {
+
+constexpr int kDh = 128;      // head dimension supported by the kernels
+constexpr int kBlock = 64;    // token block of the mask and of the sparse branch
+constexpr int kPairs = kDh / 2;
+
+// Status words at the start of the workspace (one 256-byte line).
+struct DeviceStatus {
+    int32_t code;             // rola_status_t of the last failing device-side check
+    int32_t where;            // kernel-specific site id
+    int32_t pad[62];
+};
+
+// Kernel-side view of a validated configuration.
+struct Shape {
+    int B, H, N, nB, n_keep, r;
+    int T, Hh, Ww;
+    int pt, px;               // pairs on the temporal / height axis (rest: width)
+    float eps_lr, eps_fuse;
+    float default_gate;       // sigmoid(gate_bias)
+    float sm_scale_log2;      // log2(e) / sqrt(128)
+};
+
+// Rotation (cos, sin) of pair m for the token at flat index n.
+__device__ __forceinline__ float2 rope_cs(const float2* __restrict__ tab, const Shape& s, int n, int m)
+{
+    int hw = s.Hh * s.Ww;
+    int row;
+    if (m < s.pt) row = n / hw;
+    else if (m < s.pt + s.px) row = s.T + (n / s.Ww) % s.Hh;
+    else row = s.T + s.Hh + n % s.Ww;
+    return tab[row * kPairs + m];
+}
+
+// ---------------------------------------------------------------- host side
+
+// Workspace carve-up for one configuration.
+struct Workspace {
+    size_t status, table, qr, kr, qbar, kbar, scores, kv_idx, C, z, Cbf, partials, total;
+    int nsplit;
+};
+
+// Host launchers, one per kernel family.  All return cudaGetLastError().
+cudaError_t launch_rope_table(const rola_config_t& cfg, float2* tab, cudaStream_t st);
+cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k,
+                             const float2* tab, void* qr, void* kr, float* qbar, float* kbar,
+                             cudaStream_t st);
+cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
+                              int32_t* kv_idx, cudaStream_t st);
+cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr,
+                               const void* v, const int32_t* kv_idx, void* o_s, cudaStream_t st);
+cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, const void* k,
+                                   const void* v, const void* P_k, const float2* tab, float* partials,
+                                   float* C, float* z, __nv_bfloat16* Cbf, cudaStream_t st);
+cudaError_t launch_c_to_bf16(const Shape& s, const float* C, __nv_bfloat16* Cbf, cudaStream_t st);
+cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q, const void* P_q,
+                                 const float* C, const __nv_bfloat16* Cbf, const float* gate,
+                                 const void* o_s, void* o, const float2* tab, cudaStream_t st);
+
+// Number of N-splits of the summary reduction for this shape.
+int summary_splits(const Shape& s);
+
+// ---------------------------------------------------------------- device PTX helpers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// 16-byte async copy global -> shared; src_bytes < 16 zero-fills the rest.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "r"(addr));
+}
+
+// D += A(16x16 bf16, row) * B(16x8 bf16, col), fp32 accumulate.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1)
+{
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+                 "{%8,%9}, {%0,%1,%2,%3};\n"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 unpack_bf16(uint32_t u)
+{
+    __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+    return __bfloat1622float2(v);
+}
+
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x)); }
+
+// Byte offset of 16-byte chunk c of row r in a [rows][128 bf16] tile with the
+// chunk index XOR-swizzled by the row (conflict-free ldmatrix on 8-row groups).
+__device__ __forceinline__ uint32_t sw128(int r, int c) { return r * 256 + ((c ^ (r & 7)) << 4); }
+
+}  // namespace rola

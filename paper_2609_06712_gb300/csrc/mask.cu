@@ -1,0 +1,174 @@
+// Block mask: pooled block scores and per-query-block top-n_keep (kernel 1).
+//
+// The paper's sparse engine selects key blocks by a "topk ratio" (Alg. 1)
+// without stating the score.  This library scores block pairs by the mean-
+// pooled ROTATED vectors, s_ij = q_bar_i . k_bar_j / sqrt(d_h), keeps the
+// n_keep largest per row (ties to the lower block id) and lists them
+// ascending.  All score arithmetic is fp32.
+#include "common.cuh"
+
+namespace rola {
+
+// ---------------------------------------------------------------------------
+// scores[bh][i][j] = (q_bar_i . k_bar_j) / sqrt(128): one 64 x 64 tile per CTA,
+// 256 threads with 4 x 4 register tiles, d staged through shared memory in
+// chunks of 32.
+
+constexpr int kSTile = 64, kSChunk = 32;
+
+__global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float* __restrict__ qbar,
+                                                           const float* __restrict__ kbar,
+                                                           float* __restrict__ scores)
+{
+    __shared__ float qs[kSChunk][kSTile + 4];
+    __shared__ float ks[kSChunk][kSTile + 4];
+    const int bh = blockIdx.z, i0 = blockIdx.y * kSTile, j0 = blockIdx.x * kSTile;
+    const float* Q = qbar + (size_t)bh * s.nB * kDh;
+    const float* K = kbar + (size_t)bh * s.nB * kDh;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float acc[4][4] = {};
+    for (int d0 = 0; d0 < kDh; d0 += kSChunk) {
+        // 64 rows x 32 d of each operand: 2048 floats, 8 per thread, stored transposed
+        for (int e = threadIdx.x; e < kSTile * kSChunk; e += 256) {
+            int row = e / kSChunk, d = e % kSChunk;
+            int gi = i0 + row, gj = j0 + row;
+            qs[d][row] = gi < s.nB ? Q[(size_t)gi * kDh + d0 + d] : 0.0f;
+            ks[d][row] = gj < s.nB ? K[(size_t)gj * kDh + d0 + d] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int d = 0; d < kSChunk; ++d) {
+            float4 a = *reinterpret_cast<const float4*>(&qs[d][ty * 4]);
+            float4 b = *reinterpret_cast<const float4*>(&ks[d][tx * 4]);
+            float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int w = 0; w < 4; ++w) acc[u][w] = fmaf(av[u], bv[w], acc[u][w]);
+        }
+        __syncthreads();
+    }
+    const float scale = 0.08838834764831845f;   // 1 / sqrt(128)
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        int gi = i0 + ty * 4 + u;
+        if (gi >= s.nB) continue;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            int gj = j0 + tx * 4 + w;
+            if (gj < s.nB) scores[((size_t)bh * s.nB + gi) * s.nB + gj] = acc[u][w] * scale;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// top-n_keep of each score row: one warp per row, 8 rows per CTA.  The row is
+// mapped to order-preserving unsigned keys (+0 and -0 identified) and the
+// n_keep-th largest key is found by a 4-pass 8-bit radix select over a
+// per-warp histogram; the row is then scanned in ascending block order,
+// taking every key above the threshold and the lowest-index keys equal to it.
+
+__device__ __forceinline__ uint32_t order_key(float f)
+{
+    uint32_t u = __float_as_uint(f == 0.0f ? 0.0f : f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+constexpr int kTopkWarps = 8;
+
+__global__ void __launch_bounds__(kTopkWarps * 32) block_topk_kernel(Shape s, const float* __restrict__ scores,
+                                                                     int32_t* __restrict__ kv_idx)
+{
+    extern __shared__ uint32_t tk_smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t* hist = tk_smem + warp * 256;
+    uint32_t* keys = tk_smem + kTopkWarps * 256 + (size_t)warp * s.nB;
+    const int row = blockIdx.x * kTopkWarps + warp;
+    const int bh = blockIdx.y;
+    if (row >= s.nB) return;
+    const float* srow = scores + ((size_t)bh * s.nB + row) * s.nB;
+    for (int j = lane; j < s.nB; j += 32) keys[j] = order_key(srow[j]);
+    __syncwarp();
+
+    uint32_t prefix = 0, pmask = 0;
+    int need = s.n_keep;             // how many keys >= threshold are still to be placed
+#pragma unroll 1
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int b = lane; b < 256; b += 32) hist[b] = 0;
+        __syncwarp();
+        for (int j = lane; j < s.nB; j += 32) {
+            uint32_t key = keys[j];
+            if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+        }
+        __syncwarp();
+        // lane owns bins 8*(31-lane) .. 8*(31-lane)+7 so that lane 0 holds the top bins
+        int base = 8 * (31 - lane);
+        uint32_t c[8];
+        uint32_t tot = 0;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) { c[t] = hist[base + t]; tot += c[t]; }
+        // inclusive prefix over lanes (from the top bins down)
+        uint32_t incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        uint32_t excl = incl - tot;
+        // the lane whose range holds the need-th key from the top
+        bool mine = excl < (uint32_t)need && incl >= (uint32_t)need;
+        uint32_t ballot = __ballot_sync(0xffffffffu, mine);
+        int src = ballot ? __ffs(ballot) - 1 : 0;
+        int bin = 0, above = 0;
+        if (lane == src) {
+            uint32_t run = excl;
+            for (int t = 7; t >= 0; --t) {
+                if (run + c[t] >= (uint32_t)need) { bin = base + t; above = (int)run; break; }
+                run += c[t];
+            }
+        }
+        bin = __shfl_sync(0xffffffffu, bin, src);
+        above = __shfl_sync(0xffffffffu, above, src);
+        need -= above;
+        prefix |= (uint32_t)bin << shift;
+        pmask |= 255u << shift;
+        __syncwarp();
+    }
+    // prefix is now the threshold key; `need` keys equal to it are kept (lowest j first)
+    const uint32_t thr = prefix;
+    int32_t* out = kv_idx + ((size_t)bh * s.nB + row) * s.n_keep;
+    int written = 0, eq_taken = 0;
+    for (int j0 = 0; j0 < s.nB; j0 += 32) {
+        int j = j0 + lane;
+        uint32_t key = j < s.nB ? keys[j] : 0u;
+        bool gt = j < s.nB && key > thr;
+        bool eq = j < s.nB && key == thr;
+        uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+        int eq_rank = eq_taken + __popc(eqb & ((1u << lane) - 1u));
+        bool sel = gt || (eq && eq_rank < need);
+        uint32_t selb = __ballot_sync(0xffffffffu, sel);
+        int pos = written + __popc(selb & ((1u << lane) - 1u));
+        if (sel && pos < s.n_keep) out[pos] = j;
+        written += __popc(selb);
+        eq_taken += __popc(eqb);
+    }
+}
+
+cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
+                              int32_t* kv_idx, cudaStream_t st)
+{
+    int t = (s.nB + kSTile - 1) / kSTile;
+    block_scores_kernel<<<dim3(t, t, s.B * s.H), 256, 0, st>>>(s, qbar, kbar, scores);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    size_t smem = (size_t)kTopkWarps * 256 * 4 + (size_t)kTopkWarps * s.nB * 4;
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(block_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    dim3 grid((s.nB + kTopkWarps - 1) / kTopkWarps, s.B * s.H);
+    block_topk_kernel<<<grid, kTopkWarps * 32, smem, st>>>(s, scores, kv_idx);
+    return cudaGetLastError();
+}
+
+}  // namespace rola

@@ -1,0 +1,147 @@
+// 3D RoPE tables and the rotate + block-pool pass of the block mask.
+//
+// RoPE (Sec. 3, Eq. shiftinv; truncation Sec. 4.2): pair m acts on coordinates
+// (2m, 2m+1); the first d_t/2 pairs turn with the temporal position, the next
+// d_x/2 with the row, the rest with the column; within an axis the i-th pair
+// turns by pos * theta^(-2i/d_axis).  The table holds (cos, sin) in fp32,
+// evaluated in fp64 once per call.
+#include "common.cuh"
+
+namespace rola {
+
+__global__ void rope_table_kernel(float2* __restrict__ tab, int T, int Hh, int Ww, int d_t, int d_x, int d_y,
+                                  int off_t, int off_x, int off_y, double theta)
+{
+    int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    int rows = T + Hh + Ww;
+    if (idx >= rows * kPairs) return;
+    int row = idx / kPairs, m = idx % kPairs;
+    int pt = d_t / 2, px = d_x / 2;
+    int axis = m < pt ? 0 : (m < pt + px ? 1 : 2);
+    int row_axis = row < T ? 0 : (row < T + Hh ? 1 : 2);
+    float2 out = make_float2(1.0f, 0.0f);
+    if (axis == row_axis) {
+        int i = axis == 0 ? m : (axis == 1 ? m - pt : m - pt - px);
+        int d_axis = axis == 0 ? d_t : (axis == 1 ? d_x : d_y);
+        int pos = axis == 0 ? row + off_t : (axis == 1 ? row - T + off_x : row - T - Hh + off_y);
+        double freq = pow(theta, -2.0 * (double)i / (double)d_axis);
+        double s, c;
+        sincos((double)pos * freq, &s, &c);
+        out = make_float2((float)c, (float)s);
+    }
+    tab[idx] = out;
+}
+
+cudaError_t launch_rope_table(const rola_config_t& cfg, float2* tab, cudaStream_t st)
+{
+    int n = (cfg.T + cfg.Hh + cfg.Ww) * kPairs;
+    rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(tab, cfg.T, cfg.Hh, cfg.Ww, cfg.rope_split[0],
+                                                       cfg.rope_split[1], cfg.rope_split[2], cfg.pos_offset[0],
+                                                       cfg.pos_offset[1], cfg.pos_offset[2], cfg.rope_theta);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// rotate + pool: one CTA per (64-token block, head, q|k).  256 threads: 16 per
+// token row (8 coordinates = 4 pairs each), 16 rows per pass, 4 passes.  Writes
+// the rotated rows in the storage dtype and the fp32 block mean of the
+// fp32-rotated (unrounded) values.
+
+template <typename T>
+struct Vec8;
+template <>
+struct Vec8<__nv_bfloat16> {
+    __device__ static void load(const __nv_bfloat16* p, float (&x)[8])
+    {
+        uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+        uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float2 f = unpack_bf16(w[i]);
+            x[2 * i] = f.x;
+            x[2 * i + 1] = f.y;
+        }
+    }
+    __device__ static void store(__nv_bfloat16* p, const float (&x)[8])
+    {
+        uint4 u = make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]),
+                             pack_bf16(x[6], x[7]));
+        *reinterpret_cast<uint4*>(p) = u;
+    }
+};
+template <>
+struct Vec8<float> {
+    __device__ static void load(const float* p, float (&x)[8])
+    {
+        float4 a = __ldg(reinterpret_cast<const float4*>(p));
+        float4 b = __ldg(reinterpret_cast<const float4*>(p) + 1);
+        x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+        x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    }
+    __device__ static void store(float* p, const float (&x)[8])
+    {
+        reinterpret_cast<float4*>(p)[0] = make_float4(x[0], x[1], x[2], x[3]);
+        reinterpret_cast<float4*>(p)[1] = make_float4(x[4], x[5], x[6], x[7]);
+    }
+};
+
+template <typename T>
+__global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __restrict__ q, const T* __restrict__ k,
+                                                        const float2* __restrict__ tab, T* __restrict__ qr,
+                                                        T* __restrict__ kr, float* __restrict__ qbar,
+                                                        float* __restrict__ kbar)
+{
+    __shared__ float part[16][kDh];
+    const int blk = blockIdx.x, bh = blockIdx.y;
+    const T* x = blockIdx.z == 0 ? q : k;
+    T* xr = blockIdx.z == 0 ? qr : kr;
+    float* xbar = blockIdx.z == 0 ? qbar : kbar;
+    const int c8 = threadIdx.x & 15;        // coordinates 8*c8 .. 8*c8+7 (pairs 4*c8 .. 4*c8+3)
+    const int rsub = threadIdx.x >> 4;      // row within a pass
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    const int n0 = blk * kBlock;
+#pragma unroll
+    for (int pass = 0; pass < kBlock / 16; ++pass) {
+        int n = n0 + pass * 16 + rsub;
+        if (n < s.N) {
+            size_t off = ((size_t)bh * s.N + n) * kDh + c8 * 8;
+            float v[8], o[8];
+            Vec8<T>::load(x + off, v);
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+                float2 cs = rope_cs(tab, s, n, c8 * 4 + p);
+                o[2 * p] = v[2 * p] * cs.x - v[2 * p + 1] * cs.y;
+                o[2 * p + 1] = v[2 * p] * cs.y + v[2 * p + 1] * cs.x;
+            }
+            Vec8<T>::store(xr + off, o);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] += o[i];
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) part[rsub][c8 * 8 + i] = acc[i];
+    __syncthreads();
+    if (threadIdx.x < kDh) {
+        float sum = 0.0f;
+#pragma unroll
+        for (int r = 0; r < 16; ++r) sum += part[r][threadIdx.x];
+        int cnt = min(kBlock, s.N - n0);
+        xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = sum / (float)cnt;
+    }
+}
+
+cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k,
+                             const float2* tab, void* qr, void* kr, float* qbar, float* kbar, cudaStream_t st)
+{
+    dim3 grid(s.nB, s.B * s.H, 2);
+    if (cfg.dtype == ROLA_BF16)
+        rope_pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
+            s, (const __nv_bfloat16*)q, (const __nv_bfloat16*)k, tab, (__nv_bfloat16*)qr, (__nv_bfloat16*)kr,
+            qbar, kbar);
+    else
+        rope_pool_kernel<float><<<grid, 256, 0, st>>>(s, (const float*)q, (const float*)k, tab, (float*)qr,
+                                                      (float*)kr, qbar, kbar);
+    return cudaGetLastError();
+}
+
+}  // namespace rola

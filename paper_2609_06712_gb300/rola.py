@@ -1,0 +1,196 @@
+"""Thin Python binding of the C ABI in include/rola.h.
+
+Argument marshalling only: every step of the module runs in the CUDA kernels
+of librola.so.  Torch tensors supply device memory and the current stream.
+Importing this module loads librola.so and raises if it is missing -- there is
+no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "librola.so")
+
+ROLA_OK, ROLA_ERR_INVALID_ARG, ROLA_ERR_UNSUPPORTED, ROLA_ERR_WORKSPACE, ROLA_ERR_CUDA, ROLA_ERR_TIMEOUT = range(6)
+ROLA_BF16, ROLA_FP32 = 0, 1
+
+
+class RolaConfig(ctypes.Structure):
+    """Mirror of rola_config_t."""
+    _fields_ = [
+        ("B", ctypes.c_int32), ("H", ctypes.c_int32), ("N", ctypes.c_int32), ("d_h", ctypes.c_int32),
+        ("T", ctypes.c_int32), ("Hh", ctypes.c_int32), ("Ww", ctypes.c_int32),
+        ("pos_offset", ctypes.c_int32 * 3),
+        ("rope_split", ctypes.c_int32 * 3),
+        ("rope_theta", ctypes.c_double),
+        ("block", ctypes.c_int32),
+        ("keep_ratio", ctypes.c_float),
+        ("r", ctypes.c_int32),
+        ("eps_lr", ctypes.c_float),
+        ("eps_fuse", ctypes.c_float),
+        ("gate_bias", ctypes.c_float),
+        ("dtype", ctypes.c_int32),
+    ]
+
+
+class RolaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {_lib.rola_status_string(status).decode()}")
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with paper_2609_06712_gb300.build.build() "
+                          "(the RoLA module has no CPU fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, S = ctypes.c_void_p, ctypes.c_size_t
+    cfgp = ctypes.POINTER(RolaConfig)
+    st = ctypes.c_int
+    sig = {
+        "rola_config_init": (st, [cfgp]),
+        "rola_num_blocks": (ctypes.c_int32, [cfgp]),
+        "rola_num_keep": (ctypes.c_int32, [cfgp]),
+        "rola_workspace_bytes": (S, [cfgp]),
+        "rola_block_mask": (st, [cfgp, P, P, P, P, S, P]),
+        "rola_sparse_attn": (st, [cfgp, P, P, P, P, P, P, S, P]),
+        "rola_lowrank_summary": (st, [cfgp, P, P, P, P, P, P, S, P]),
+        "rola_lowrank_apply": (st, [cfgp, P, P, P, P, P, P, P, S, P]),
+        "rola_forward": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P]),
+        "rola_forward_timed": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P, P]),
+        "rola_get_device_status": (st, [P, P]),
+        "rola_status_string": (ctypes.c_char_p, [st]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+
+
+def library():
+    """The loaded ctypes library (for tests that call the ABI directly)."""
+    return _lib
+
+
+def make_config(cfg: dict, dtype: int = ROLA_BF16) -> RolaConfig:
+    """rola_config_t from a plain dict of layer sizes (see configs.py)."""
+    c = RolaConfig()
+    _lib.rola_config_init(ctypes.byref(c))
+    c.B, c.H, c.N = cfg["B"], cfg["H"], cfg["N"]
+    c.d_h = cfg.get("d_h", 128)
+    c.T, c.Hh, c.Ww = cfg["T"], cfg["Hh"], cfg["Ww"]
+    c.pos_offset[:] = list(cfg.get("pos_offset", (0, 0, 0)))
+    c.rope_split[:] = list(cfg.get("rope_split", (44, 42, 42)))
+    c.rope_theta = float(cfg.get("rope_theta", 10000.0))
+    c.block = cfg.get("block", 64)
+    c.keep_ratio = float(cfg["keep"])
+    c.r = cfg["r"]
+    c.eps_lr = float(cfg.get("eps_lr", 1e-6))
+    c.eps_fuse = float(cfg.get("eps_fuse", 1e-6))
+    c.gate_bias = float(cfg.get("gate_bias", -1.946))
+    c.dtype = dtype
+    return c
+
+
+def _p(t):
+    if t is None:
+        return None
+    if not (t.is_cuda and t.is_contiguous()):
+        raise ValueError("RoLA tensors must be contiguous CUDA tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(status: int, where: str):
+    if status != ROLA_OK:
+        raise RolaError(status, where)
+
+
+def num_blocks(c: RolaConfig) -> int:
+    return _lib.rola_num_blocks(ctypes.byref(c))
+
+
+def num_keep(c: RolaConfig) -> int:
+    return _lib.rola_num_keep(ctypes.byref(c))
+
+
+def workspace_bytes(c: RolaConfig) -> int:
+    return _lib.rola_workspace_bytes(ctypes.byref(c))
+
+
+def workspace(c: RolaConfig, device="cuda") -> torch.Tensor:
+    """A workspace tensor of rola_workspace_bytes(c) bytes (torch allocations are 256-byte aligned)."""
+    n = workspace_bytes(c)
+    if n == 0:
+        raise RolaError(ROLA_ERR_INVALID_ARG, "rola_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def block_mask(c, q, k, kv_idx, ws, stream=None):
+    _check(_lib.rola_block_mask(ctypes.byref(c), _p(q), _p(k), _p(kv_idx), _p(ws), ws.numel(), _stream(stream)),
+           "rola_block_mask")
+
+
+def sparse_attn(c, q, k, v, kv_idx, o_s, ws, stream=None):
+    _check(_lib.rola_sparse_attn(ctypes.byref(c), _p(q), _p(k), _p(v), _p(kv_idx), _p(o_s), _p(ws), ws.numel(),
+                                 _stream(stream)), "rola_sparse_attn")
+
+
+def lowrank_summary(c, k, v, P_k, C, z, ws, stream=None):
+    _check(_lib.rola_lowrank_summary(ctypes.byref(c), _p(k), _p(v), _p(P_k), _p(C), _p(z), _p(ws), ws.numel(),
+                                     _stream(stream)), "rola_lowrank_summary")
+
+
+def lowrank_apply(c, q, P_q, C, gate, o_s, o, ws, stream=None):
+    _check(_lib.rola_lowrank_apply(ctypes.byref(c), _p(q), _p(P_q), _p(C), _p(gate), _p(o_s), _p(o), _p(ws),
+                                   ws.numel(), _stream(stream)), "rola_lowrank_apply")
+
+
+def forward(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, stream=None):
+    _check(_lib.rola_forward(ctypes.byref(c), _p(q), _p(k), _p(v), _p(P_q), _p(P_k), _p(gate), _p(o),
+                             _p(kv_idx_out), _p(ws), ws.numel(), _stream(stream)), "rola_forward")
+
+
+def forward_timed(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, events, stream=None):
+    """rola_forward recording 5 stage events (torch.cuda.Event, already created)."""
+    arr = (ctypes.c_void_p * 5)(*[ctypes.c_void_p(e.cuda_event) for e in events])
+    _check(_lib.rola_forward_timed(ctypes.byref(c), _p(q), _p(k), _p(v), _p(P_q), _p(P_k), _p(gate), _p(o),
+                                   _p(kv_idx_out), _p(ws), ws.numel(), _stream(stream), arr),
+           "rola_forward_timed")
+
+
+def get_device_status(ws, stream=None) -> int:
+    return _lib.rola_get_device_status(_p(ws), _stream(stream))
+
+
+class RoLAAttention:
+    """Convenience wrapper: owns the workspace for one layer shape and runs rola_forward.
+
+    ``__call__(q, k, v, P_q, P_k, gate=None)`` returns (o, kv_idx) as new tensors."""
+
+    def __init__(self, cfg: dict, dtype: int = ROLA_BF16, device="cuda"):
+        self.cfg = make_config(cfg, dtype)
+        self.ws = workspace(self.cfg, device)
+        self.nB = num_blocks(self.cfg)
+        self.n_keep = num_keep(self.cfg)
+
+    def __call__(self, q, k, v, P_q, P_k, gate=None, out=None, kv_idx=None, stream=None):
+        c = self.cfg
+        if out is None:
+            out = torch.empty_like(q)
+        if kv_idx is None:
+            kv_idx = torch.empty((c.B, c.H, self.nB, self.n_keep), dtype=torch.int32, device=q.device)
+        forward(c, q, k, v, P_q, P_k, gate, out, kv_idx, self.ws, stream)
+        return out, kv_idx

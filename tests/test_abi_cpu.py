@@ -1,0 +1,124 @@
+"""The C ABI library on a machine without a GPU: it builds, loads, exports every
+entry point include/rola.h declares, and its host-side validation returns the
+documented status codes before touching the device."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "rola.h")
+
+
+@pytest.fixture(scope="module")
+def rl():
+    from paper_2609_06712_gb300 import build
+    build.build()
+    from paper_2609_06712_gb300 import rola
+    return rola
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(rola_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_entry_point(rl):
+    names = declared_functions()
+    assert {"rola_block_mask", "rola_sparse_attn", "rola_lowrank_summary", "rola_lowrank_apply",
+            "rola_forward"} <= set(names)
+    out = subprocess.run(["nm", "-D", "--defined-only", rl.LIB_PATH], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(line.split()[-1] for line in out.splitlines() if line.strip())
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        getattr(rl.library(), n)
+
+
+def cfg_tiny(rl, **kw):
+    from paper_2609_06712_gb300 import configs
+    c = rl.make_config(configs.get("tiny"))
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+def test_defaults_and_sizes(rl):
+    c = rl.RolaConfig()
+    assert rl.library().rola_config_init(ctypes.byref(c)) == rl.ROLA_OK
+    assert (c.d_h, c.block, list(c.rope_split), c.rope_theta) == (128, 64, [44, 42, 42], 10000.0)
+    assert c.gate_bias == pytest.approx(-1.946) and c.eps_lr == pytest.approx(1e-6)
+    from paper_2609_06712_gb300 import configs
+    for name, nb, nk in [("tiny", 16, 2), ("wan13b_480p", 512, 51), ("wan14b_720p", 1182, 118),
+                         ("wan14b_720p_long", 2307, 231)]:
+        cc = rl.make_config(configs.get(name))
+        assert rl.num_blocks(cc) == nb and rl.num_keep(cc) == nk
+        assert rl.workspace_bytes(cc) > 0
+
+
+def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
+    """Every compute entry point with dummy (never dereferenced) pointers."""
+    L = rl.library()
+    P = ctypes.c_void_p
+    p, w = P(ptr), P(ws)
+    b = ctypes.byref(c)
+    return [
+        L.rola_block_mask(b, p, p, p, w, ws_bytes, None),
+        L.rola_sparse_attn(b, p, p, p, p, p, w, ws_bytes, None),
+        L.rola_lowrank_summary(b, p, p, p, p, None, w, ws_bytes, None),
+        L.rola_lowrank_apply(b, p, p, p, None, p, p, w, ws_bytes, None),
+        L.rola_forward(b, p, p, p, p, p, None, p, None, w, ws_bytes, None),
+    ]
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("N", 1000, 1),            # N != T*Hh*Ww
+    ("B", 0, 1),
+    ("d_h", 64, 2),            # valid shape, not built
+    ("block", 128, 2),
+    ("r", 24, 2),              # even but not a multiple of 16
+    ("r", 15, 1),
+    ("r", 256, 1),             # r > d_h
+    ("keep_ratio", 1.5, 1),
+    ("keep_ratio", float("nan"), 1),
+    ("rope_theta", 0.0, 1),
+    ("eps_lr", -1.0, 1),
+    ("dtype", 7, 1),
+])
+def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
+    c = cfg_tiny(rl, **{field: value})
+    assert all(s == code for s in call_all(rl, c)), call_all(rl, c)
+    assert rl.workspace_bytes(c) == 0 and rl.num_keep(c) == 0
+
+
+def test_rope_split_must_sum_to_head_dim(rl):
+    c = cfg_tiny(rl)
+    c.rope_split[:] = [44, 42, 40]
+    assert all(s == rl.ROLA_ERR_INVALID_ARG for s in call_all(rl, c))
+    c.rope_split[:] = [43, 43, 42]
+    assert all(s == rl.ROLA_ERR_INVALID_ARG for s in call_all(rl, c))
+
+
+def test_null_and_misaligned_pointers(rl):
+    c = cfg_tiny(rl)
+    assert all(s == rl.ROLA_ERR_INVALID_ARG for s in call_all(rl, c, ptr=0))
+    assert all(s == rl.ROLA_ERR_INVALID_ARG for s in call_all(rl, c, ptr=0x10008))
+
+
+def test_workspace_checks(rl):
+    c = cfg_tiny(rl)
+    need = rl.workspace_bytes(c)
+    assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws_bytes=need - 1))
+    assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws=0x100080))   # not 256-aligned
+    assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws=0))
+
+
+def test_status_strings(rl):
+    L = rl.library()
+    for code in range(6):
+        assert L.rola_status_string(code).decode().startswith("ROLA_")
+    assert b"unknown" in L.rola_status_string(42)

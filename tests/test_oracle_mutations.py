@@ -22,8 +22,8 @@ MUTATIONS = {
     "axis_boundary": ("if (m < pt) { axis = 0;", "if (m <= pt) { axis = 0;"),
     "position_row_index": ("int x = (n / c->Ww) % c->Hh;", "int x = (n / c->Hh) % c->Ww;"),
     "silu_sign": ("return x / (1.0 + exp(-x));", "return x / (1.0 + exp(x));"),
-    "truncation_pairs": ("orc_rotate(c, r / 2, pos, u, feat, r);\n    } else if",
-                         "orc_rotate(c, r / 2 - 1, pos, u, feat, r);\n    } else if"),
+    "truncation_pairs": ("rotate_pairs(r / 2, cs, u, feat, r);\n    } else if",
+                         "rotate_pairs(r / 2 - 1, cs, u, feat, r);\n    } else if"),
     "summary_transposed": ("Cb[(size_t)a * dh + d] += kt[a] * (double)vn[d];",
                            "Cb[(size_t)a * dh + d] += kt[a] * (double)vn[(d + 1) % dh];"),
     "mask_tie_order": ("return (x->j < y->j) ? -1 : (x->j > y->j);",

@@ -1,0 +1,248 @@
+"""CUDA path vs the fp64 oracle, element by element, through the C ABI.
+
+Per kernel (mask, sparse branch, summary, apply) and for the whole module, in
+bf16 and in the fp32 validation mode, on small layers that still span many
+blocks and a ragged tail, and on the Wan2.1 layer shapes with sampled query
+blocks.  Inputs come from the shared seeded generator; expected values come
+from the oracle only.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2609_06712_gb300 import configs, inputs
+from parity_util import assert_close, check_mask, dev, rows_of_blocks, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rl():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2609_06712_gb300 import build
+    build.build()
+    from paper_2609_06712_gb300 import rola
+    O.build()
+    return rola
+
+
+def layer(name=None, **kw):
+    c = configs.get(name or "tiny")
+    c.update(kw)
+    c["N"] = c["T"] * c["Hh"] * c["Ww"]
+    return c
+
+
+SMALL = {
+    "tiny": layer(),
+    "ragged_105": layer(T=3, Hh=5, Ww=7, H=3, r=16, keep=0.5, seed=21),
+    "ragged_585_r64": layer(T=5, Hh=9, Ww=13, H=2, r=64, keep=0.3, seed=22),
+    "r128_keep1": layer(T=2, Hh=12, Ww=16, H=2, r=128, keep=1.0, seed=23),
+    "r48_gate": layer(T=3, Hh=10, Ww=20, H=2, r=48, keep=0.2, seed=24, dist="normal_gate"),
+    "rmsnorm_gain_b2": layer(T=4, Hh=8, Ww=9, B=2, H=2, r=32, keep=0.25, seed=25, dist="rmsnorm_gain"),
+    "offset": layer(T=3, Hh=8, Ww=8, H=2, r=32, keep=0.25, seed=26, pos_offset=(5, -3, 7)),
+}
+
+
+def draw(cfg, dtype):
+    x = inputs.make_inputs(cfg, dtype=dtype)
+    host = {k: (None if v is None else v.float().numpy()) for k, v in x.items()}
+    return x, host
+
+
+def dtype_cases():
+    return [("bf16", torch.bfloat16), ("fp32", torch.float32)]
+
+
+def rola_dtype(rl, name):
+    return rl.ROLA_BF16 if name == "bf16" else rl.ROLA_FP32
+
+
+# ------------------------------------------------------------------ per kernel
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_block_mask(rl, case, dname, tdt):
+    cfg = SMALL[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    nB, nk = rl.num_blocks(c), rl.num_keep(c)
+    kv = torch.empty((cfg["B"], cfg["H"], nB, nk), dtype=torch.int32, device="cuda")
+    rl.block_mask(c, dev(x["q"]), dev(x["k"]), kv, ws)
+    torch.cuda.synchronize()
+    idx, scores, gap, tau = O.block_mask(cfg, h["q"], h["k"])
+    check_mask(kv.cpu().numpy(), idx, scores, gap, tau, nB)
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_sparse_attn(rl, case, dname, tdt):
+    cfg = SMALL[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    idx, _, _, _ = O.block_mask(cfg, h["q"], h["k"])
+    o_s = torch.empty_like(dev(x["q"]))
+    rl.sparse_attn(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), torch.from_numpy(idx).cuda(), o_s, ws)
+    torch.cuda.synchronize()
+    want = O.sparse_attn(cfg, O.rope_full(cfg, h["q"]), O.rope_full(cfg, h["k"]), h["v"], idx)
+    assert_close(to_np(o_s), want, dname == "bf16", f"O^s[{case},{dname}]")
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_lowrank_summary(rl, case, dname, tdt):
+    cfg = SMALL[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    B, H, r = cfg["B"], cfg["H"], cfg["r"]
+    C = torch.empty((B, H, r, 128), dtype=torch.float32, device="cuda")
+    z = torch.empty((B, H, r), dtype=torch.float32, device="cuda")
+    rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, z, ws)
+    torch.cuda.synchronize()
+    Cw, zw = O.lowrank_summary(cfg, h["k"], h["v"], h["P_k"])
+    assert_close(to_np(C), Cw, dname == "bf16", f"C[{case},{dname}]", unit_rms=True)
+    assert_close(to_np(z), zw, dname == "bf16", f"z[{case},{dname}]", unit_rms=True)
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_lowrank_apply(rl, case, dname, tdt):
+    cfg = SMALL[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    Cw, _ = O.lowrank_summary(cfg, h["k"], h["v"], h["P_k"])
+    # O^s stand-in: attention-sized values, stored in the layer dtype
+    g = torch.Generator().manual_seed(cfg["seed"] + 1000)
+    o_s = (0.02 * torch.randn(x["q"].shape, generator=g)).to(tdt)
+    C32 = torch.from_numpy(Cw.astype(np.float32))
+    o = torch.empty_like(dev(o_s))
+    rl.lowrank_apply(c, dev(x["q"]), dev(x["P_q"]), dev(C32), dev(x["gate"]), dev(o_s), o, ws)
+    torch.cuda.synchronize()
+    want = O.lowrank_apply(cfg, h["q"], h["P_q"], C32.double().numpy(), h["gate"], o_s.float().numpy())
+    assert_close(to_np(o), want, dname == "bf16", f"O[{case},{dname}]")
+    # in place: o aliases o_s
+    o_s_dev = dev(o_s)
+    rl.lowrank_apply(c, dev(x["q"]), dev(x["P_q"]), dev(C32), dev(x["gate"]), o_s_dev, o_s_dev, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(o_s_dev, o)
+
+
+# ------------------------------------------------------------------ module
+
+
+def run_forward(rl, cfg, x, dname, o=None):
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    nB, nk = rl.num_blocks(c), rl.num_keep(c)
+    q = dev(x["q"])
+    out = torch.empty_like(q) if o is None else o
+    kv = torch.empty((cfg["B"], cfg["H"], nB, nk), dtype=torch.int32, device="cuda")
+    rl.forward(c, q, dev(x["k"]), dev(x["v"]), dev(x["P_q"]), dev(x["P_k"]), dev(x["gate"]), out, kv, ws)
+    assert rl.get_device_status(ws) == rl.ROLA_OK
+    return out, kv
+
+
+def compare_forward(cfg, x, h, out, kv, dname, qblocks=None):
+    res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], qblocks=qblocks)
+    idx, scores, gap, tau = O.block_mask(cfg, h["q"], h["k"])
+    assert (idx == res["kv_idx"]).all()
+    nB = idx.shape[2]
+    equal = check_mask(kv.cpu().numpy(), idx, scores, gap, tau, nB)
+    blocks = range(nB) if qblocks is None else qblocks
+    got = to_np(out)
+    for b in range(cfg["B"]):
+        for hh in range(cfg["H"]):
+            sel = [i for i in blocks if equal[b, hh, i]]
+            rows = rows_of_blocks(sel, cfg["block"], cfg["N"])
+            assert rows.sum() > 0
+            assert_close(got[b, hh, rows], res["o"][b, hh, rows], dname == "bf16",
+                         f"O[{cfg['name']},{dname},b{b},h{hh}]")
+    return res
+
+
+@pytest.mark.parametrize("case", sorted(SMALL))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_forward_small(rl, case, dname, tdt):
+    cfg = SMALL[case]
+    x, h = draw(cfg, tdt)
+    out, kv = run_forward(rl, cfg, x, dname)
+    torch.cuda.synchronize()
+    compare_forward(cfg, x, h, out, kv, dname)
+
+
+def test_forward_is_deterministic_and_stays_in_bounds(rl):
+    """Two runs are bitwise equal; bytes around the output are never written."""
+    cfg = SMALL["ragged_585_r64"]
+    x, _ = draw(cfg, torch.bfloat16)
+    n = x["q"].numel()
+    pad = 4096
+    canvas = torch.full((n + 2 * pad,), 7.25, dtype=torch.bfloat16, device="cuda")
+    o1 = canvas[pad:pad + n].view(x["q"].shape)
+    _, kv1 = run_forward(rl, cfg, x, "bf16", o=o1)
+    o2, kv2 = run_forward(rl, cfg, x, "bf16")
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(kv1, kv2)
+    assert (canvas[:pad] == 7.25).all() and (canvas[pad + n:] == 7.25).all()
+
+
+def test_shift_invariance_on_gpu(rl):
+    """Eq. (shiftinv): a uniform shift of all positions leaves the GPU output unchanged
+    up to fp32 table rounding (outputs match the unshifted oracle)."""
+    cfg = SMALL["offset"]
+    x, h = draw(cfg, torch.bfloat16)
+    out, kv = run_forward(rl, cfg, x, "bf16")
+    base = dict(cfg, pos_offset=(0, 0, 0))
+    out0, kv0 = run_forward(rl, base, x, "bf16")
+    torch.cuda.synchronize()
+    assert torch.equal(kv, kv0)
+    assert_close(to_np(out), to_np(out0), True, "shifted vs unshifted")
+
+
+def test_gate_zero_returns_sparse_branch(rl):
+    """Eq. (gate) with g = 0 gives O = O^s."""
+    cfg = SMALL["tiny"]
+    x, h = draw(cfg, torch.float32)
+    x["gate"] = torch.zeros((cfg["B"], cfg["N"]))
+    out, kv = run_forward(rl, cfg, x, "fp32")
+    c = rl.make_config(cfg, rl.ROLA_FP32)
+    ws = rl.workspace(c)
+    o_s = torch.empty_like(out)
+    rl.sparse_attn(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), kv, o_s, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out, o_s)
+
+
+# ------------------------------------------------------------------ layer shapes
+
+
+def sample_blocks(nB, n=32, seed=0):
+    rng = np.random.default_rng(seed)
+    mid = rng.choice(np.arange(1, nB - 1), size=min(n - 2, nB - 2), replace=False)
+    return sorted({0, nB - 1, *mid.tolist()})
+
+
+@pytest.mark.parametrize("name", ["wan13b_480p", "wan14b_480p", "wan14b_720p"])
+def test_forward_layer_shapes_sampled(rl, name):
+    """The Wan2.1 layer shapes at full size, in the launch configuration the bench
+    times: the mask and C in full, O on 32 sampled query blocks of every head
+    (including the first and the ragged last block)."""
+    cfg = configs.get(name)
+    x, h = draw(cfg, torch.bfloat16)
+    out, kv = run_forward(rl, cfg, x, "bf16")
+    torch.cuda.synchronize()
+    nB = configs.get(name)["N"] // 64 + (1 if configs.get(name)["N"] % 64 else 0)
+    blocks = sample_blocks(nB, 32, seed=cfg["seed"])
+    res = compare_forward(cfg, x, h, out, kv, "bf16", qblocks=blocks)
+    # the summary in full
+    c = rl.make_config(cfg)
+    ws = rl.workspace(c)
+    C = torch.empty((cfg["B"], cfg["H"], cfg["r"], 128), dtype=torch.float32, device="cuda")
+    rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, None, ws)
+    torch.cuda.synchronize()
+    assert_close(to_np(C), res["C"], True, f"C[{name}]", unit_rms=True)
