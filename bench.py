@@ -137,7 +137,7 @@ def oracle_sample_time(cfg, heads, qblocks):
     return time.perf_counter() - t0
 
 
-def cpu_oracle_estimate(cfg, heads=None, q_lo=2, q_hi=6):
+def cpu_oracle_estimate(cfg, heads=None, q_lo=8, q_hi=96):
     """Layer time of the oracle extrapolated from a bounded sample: `heads` heads in
     parallel with q_lo and q_hi query blocks each; the difference gives the
     per-query-block cost, the rest the per-head fixed cost (mask, summary)."""
