@@ -182,6 +182,31 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                  void* const* stage_events);
 
 /*
+ * rola_lowrank_summary_static: the low-rank summary (C and optionally z, as
+ * rola_lowrank_summary computes them) for callers that cannot give the
+ * library any device scratch -- e.g. a plugin whose host framework owns the
+ * allocator and hands the op only its inputs and outputs, or a runtime that
+ * forbids device allocation once it is serving.  The paper has no
+ * counterpart; this is a deployment variant of the entry point above.
+ *
+ * It takes no workspace and allocates nothing: its scratch (RoPE table and
+ * split-N partial sums) is one file-scope __device__ array of 16 MiB that
+ * every GPU loading the library holds until the process exits.  The first
+ * call on a device looks up that array's device address and caches it; make
+ * that first call before any stream capture.  Every call reuses the same
+ * array, so calls whose executions overlap on the GPU (other streams, other
+ * host threads) race and must be serialised by the caller.
+ *   k, v, P_k, C, z : as rola_lowrank_summary (device pointers, caller-owned)
+ * Returns ROLA_ERR_UNSUPPORTED when the layer's scratch (table plus one
+ * partial per head, 4*(r*d_h + r) bytes per head) exceeds the 16 MiB array,
+ * and the usual validation codes otherwise.  When the array cannot hold the
+ * regular number of splits it uses fewer, so C may differ from
+ * rola_lowrank_summary's in the last bits (same fixed-order sum, coarser split).
+ */
+rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, const void* k, const void* v,
+                                          const void* P_k, float* C, float* z, void* stream);
+
+/*
  * Synchronises `stream`, then reads the device status word at the start of
  * ws: ROLA_OK, or ROLA_ERR_TIMEOUT if a bounded device wait expired since the
  * workspace was last cleared by an entry point.  ROLA_ERR_CUDA if the

@@ -6,13 +6,7 @@
 
 using namespace rola;
 
-namespace {
-
-constexpr size_t kAlign = 256;
-
-size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
-
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+namespace rola {
 
 int num_blocks_of(const rola_config_t& c) { return (c.N + c.block - 1) / c.block; }
 
@@ -26,7 +20,6 @@ int num_keep_of(const rola_config_t& c)
     return n;
 }
 
-// Returns ROLA_OK if the configuration is one the kernels handle.
 rola_status_t validate(const rola_config_t* c)
 {
     if (!c) return ROLA_ERR_INVALID_ARG;
@@ -68,6 +61,16 @@ Shape make_shape(const rola_config_t& c)
     s.sm_scale_log2 = (float)(1.4426950408889634 / sqrt((double)kDh));
     return s;
 }
+
+}  // namespace rola
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 Workspace layout(const rola_config_t& c)
 {

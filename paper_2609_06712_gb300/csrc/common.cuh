@@ -78,6 +78,12 @@ cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q,
 // Number of N-splits of the summary reduction for this shape.
 int summary_splits(const Shape& s);
 
+// Host-side configuration checks shared by the entry points (api.cu).
+rola_status_t validate(const rola_config_t* cfg);   // ROLA_OK if the kernels handle cfg
+Shape make_shape(const rola_config_t& cfg);          // cfg must be valid
+int num_blocks_of(const rola_config_t& cfg);
+int num_keep_of(const rola_config_t& cfg);
+
 // ---------------------------------------------------------------- device PTX helpers
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p)

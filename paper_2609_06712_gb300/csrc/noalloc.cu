@@ -1,0 +1,88 @@
+// rola_lowrank_summary_static: the low-rank summary with no caller workspace.
+//
+// Some callers cannot hand this library any device scratch: a plugin whose
+// host framework owns the allocator and passes the op only its input and
+// output tensors, or a runtime that forbids device allocation once it has
+// started (fixed memory budget, no cudaMalloc on the serving path).  For
+// them this entry point keeps its scratch -- the RoPE table and the split-N
+// partial sums of the summary -- in one file-scope __device__ array of
+// kStaticScratchBytes, which every GPU that loads the library holds until
+// the process exits.  It allocates nothing itself.
+//
+// The array's name is usable only in device code; host code needs its
+// device address, which cudaGetSymbolAddress returns.  That lookup is done
+// once per device, on the first call made while that device is current, and
+// cached.  Make that first call before any stream capture.
+//
+// Every call shares the one array and it keeps the last call's contents.
+// Everything a call reads from it, the call has written first (the table and
+// every partial are overwritten in full), so nothing needs clearing.  Calls
+// whose executions overlap on the GPU -- on different streams, or from
+// different host threads -- race on the array and must be serialised by the
+// caller.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace rola {
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;   // 16 MiB per device
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_lock;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device (looked up once).
+cudaError_t scratch_address(void** out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> guard(g_lock);
+    if (!g_scratch_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return cudaSuccess;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+}  // namespace
+}  // namespace rola
+
+using namespace rola;
+
+extern "C" rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, const void* k, const void* v,
+                                                     const void* P_k, float* C, float* z, void* stream)
+{
+    rola_status_t st = validate(cfg);
+    if (st != ROLA_OK) return st;
+    auto a16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+    if (!k || !v || !P_k || !C || !a16(k) || !a16(v) || !a16(P_k) || !a16(C) || (z && !a16(z)))
+        return ROLA_ERR_INVALID_ARG;
+    const Shape s = make_shape(*cfg);
+    // scratch = RoPE table | partials [B*H][nsplit][r*128 + r]; fewer splits if needed to fit
+    const size_t table = align256(sizeof(float2) * (size_t)(cfg->T + cfg->Hh + cfg->Ww) * kPairs);
+    const size_t per_split = sizeof(float) * (size_t)s.B * s.H * ((size_t)s.r * kDh + s.r);
+    if (table + per_split > kStaticScratchBytes) return ROLA_ERR_UNSUPPORTED;   // layer too large for the array
+    int nsplit = summary_splits(s);
+    const int fit = (int)((kStaticScratchBytes - table) / per_split);
+    if (nsplit > fit) nsplit = fit;
+    void* base = nullptr;
+    if (scratch_address(&base) != cudaSuccess) return ROLA_ERR_CUDA;
+    float2* tab = reinterpret_cast<float2*>(base);
+    float* partials = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + table);
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    if (launch_rope_table(*cfg, tab, cs) != cudaSuccess) return ROLA_ERR_CUDA;
+    if (launch_lowrank_summary(cfg->dtype, s, nsplit, k, v, P_k, tab, partials, C, z, nullptr, cs) != cudaSuccess)
+        return ROLA_ERR_CUDA;
+    return ROLA_OK;
+}

@@ -59,6 +59,7 @@ def _load():
         "rola_block_mask": (st, [cfgp, P, P, P, P, S, P]),
         "rola_sparse_attn": (st, [cfgp, P, P, P, P, P, P, S, P]),
         "rola_lowrank_summary": (st, [cfgp, P, P, P, P, P, P, S, P]),
+        "rola_lowrank_summary_static": (st, [cfgp, P, P, P, P, P, P]),
         "rola_lowrank_apply": (st, [cfgp, P, P, P, P, P, P, P, S, P]),
         "rola_forward": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P]),
         "rola_forward_timed": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P, P]),
@@ -151,6 +152,12 @@ def sparse_attn(c, q, k, v, kv_idx, o_s, ws, stream=None):
 def lowrank_summary(c, k, v, P_k, C, z, ws, stream=None):
     _check(_lib.rola_lowrank_summary(ctypes.byref(c), _p(k), _p(v), _p(P_k), _p(C), _p(z), _p(ws), ws.numel(),
                                      _stream(stream)), "rola_lowrank_summary")
+
+
+def lowrank_summary_static(c, k, v, P_k, C, z, stream=None):
+    """The summary with no workspace: scratch lives in the library's static device array."""
+    _check(_lib.rola_lowrank_summary_static(ctypes.byref(c), _p(k), _p(v), _p(P_k), _p(C), _p(z),
+                                            _stream(stream)), "rola_lowrank_summary_static")
 
 
 def lowrank_apply(c, q, P_q, C, gate, o_s, o, ws, stream=None):
