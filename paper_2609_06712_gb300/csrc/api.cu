@@ -205,7 +205,8 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
     // rotated copies (the pooled means are a by-product here)
     ROLA_TRY(launch_rope_pool(*cfg, s, q, k, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
                               at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
-    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv_idx, o_s, st));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv_idx, o_s,
+                                at<DeviceStatus>(ws, w.status), st));
     return ROLA_OK;
 }
 
@@ -270,7 +271,8 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                     at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
                                     at<__nv_bfloat16>(ws, w.Cbf), st));
     ROLA_TRY(mark(2));
-    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv, o, st));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv, o,
+                                at<DeviceStatus>(ws, w.status), st));
     ROLA_TRY(mark(3));
     ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, o,
                                   o, at<float2>(ws, w.table), st));

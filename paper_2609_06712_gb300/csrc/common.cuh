@@ -66,7 +66,10 @@ cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const voi
 cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
                               int32_t* kv_idx, cudaStream_t st);
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr,
-                               const void* v, const int32_t* kv_idx, void* o_s, cudaStream_t st);
+                               const void* v, const int32_t* kv_idx, void* o_s, DeviceStatus* status,
+                               cudaStream_t st);
+cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
+                                  const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st);
 cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, const void* k,
                                    const void* v, const void* P_k, const float2* tab, float* partials,
                                    float* C, float* z, __nv_bfloat16* Cbf, cudaStream_t st);
