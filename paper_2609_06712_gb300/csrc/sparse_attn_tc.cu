@@ -9,6 +9,8 @@
 // kept 64-key blocks as the 128-row operand.
 //   S^T[key][q]  = K_pair (128 x 128, smem, K-major)  x  Q^T (N = 64, smem, K-major)
 //   O^T[d][q]   += V_pair^T (128 x 128 keys, smem, MN-major) x P^T (128 keys x 64 q, smem, MN-major)
+// Shared-memory tiles: Q [chunk][64 rows], K pair [chunk][block][64 rows],
+// V pair [block][chunk][64 rows], rows of 128 B in 128-byte swizzle atoms.
 // S^T and O^T live in TMEM (fp32); TMEM lane = key (for S^T) or d (for O^T).
 //
 // Softmax.  A softmax thread owns one key (one TMEM lane) and sees that
@@ -17,21 +19,28 @@
 // current m_q; only when some score exceeds m_q by more than 2^8 (in base 2)
 // does the warpgroup compute the tile's exact column maxima, raise m_q and
 // rescale O^T (in TMEM) and its row sums.  The first tile of a query block
-// always takes that path.  Row sums are accumulated per thread and reduced
-// across the 128 threads once per query block.  Weights are rounded to bf16
-// for the P V product and the row sums add the same rounded values.
+// always takes that path.  Row sums are accumulated per thread in fp32 and
+// reduced across the 128 threads once per query block; the weights enter the
+// P V product rounded to bf16.
 //
-// Warp roles (192 threads, one persistent CTA per SM):
-//   warps 0-3  softmax + epilogue (TMEM lanes 32w .. 32w+31)
-//   warp  4    TMA producer: Q (per query block), K and V pairs (per tile)
-//   warp  5    MMA issuer and TMEM owner
-// Double buffers: Q, K, V, S^T, P^T and O^T, so the next tile's Q K^T runs
-// while the current tile's softmax does, and the next query block's first
-// tiles run while the current one's epilogue does.  Every wait on an
+// Warp roles (384 threads, one persistent CTA per SM):
+//   warps 0-7  softmax + epilogue: two warpgroups, each owning 32 of the 64
+//              query columns of every tile (warp w reads TMEM lanes
+//              32 (w mod 4) .. +31, so both warpgroups see all 128 keys)
+//   warp  8    TMA producer: Q (per query block) and the K pairs
+//   warp  9    TMA producer: the V blocks
+//   warp 10    Q K^T issuer and TMEM owner
+//   warp 11    P V issuer
+// Buffers: K pairs in a 3-deep ring and V blocks in a 5-deep ring of single
+// blocks (the L2 -> shared-memory latency under load is ~2 us, so the bytes in
+// flight set the pace; 224 KB of the 227 KB go to tiles); S^T, P^T and O^T double-buffered, so the next tile's Q K^T
+// runs while the current tile's softmax does and the next query block's
+// first tiles run while the current one's epilogue does; Q single-buffered.  Every wait on an
 // mbarrier is bounded (2 s); a wait that gives up records ROLA_ERR_TIMEOUT
 // in the workspace status word, and the CTA stops issuing, drains what it
 // issued and releases its TMEM.
 #include <cudaTypedefs.h>
+#include <stddef.h>
 
 #include "common.cuh"
 #include "tcgen05.cuh"
@@ -41,34 +50,51 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 192;
-constexpr int kSoftmaxThreads = 128;
+constexpr int kSoftmaxWG = 2;                        // softmax warpgroups, each owns 64/kSoftmaxWG query columns
+constexpr int kCols = 64 / kSoftmaxWG;               // query columns per softmax warpgroup
+constexpr int kSoftmaxWarps = 4 * kSoftmaxWG;
+constexpr int kProducerKWarp = kSoftmaxWarps;      // Q and the K pairs
+constexpr int kProducerVWarp = kSoftmaxWarps + 1;  // V blocks
+constexpr int kMmaWarp = kSoftmaxWarps + 2;        // Q K^T issuer, TMEM owner
+constexpr int kPvWarp = kSoftmaxWarps + 3;         // P V issuer
+constexpr int kThreads = 32 * (kSoftmaxWarps + 4);
+constexpr int kWGThreads = 128;
 constexpr uint32_t kQBytes = 64 * 128 * 2;          // one query block
 constexpr uint32_t kKVBytes = 128 * 128 * 2;        // a pair of key blocks
 constexpr uint32_t kPBytes = 128 * 64 * 2;          // P^T tile
 constexpr uint32_t kOBytes = 64 * 128 * 2;          // output staging
+constexpr int KS = 3;                               // K ring: pairs of key blocks ([chunk][block][row])
+constexpr int VB = 5;                               // V ring: single key blocks (16 KB, [chunk][row])
+constexpr uint32_t kVBlockBytes = 64 * 128 * 2;
 constexpr uint32_t kSmemQ = 0;
-constexpr uint32_t kSmemK = kSmemQ + 2 * kQBytes;
-constexpr uint32_t kSmemV = kSmemK + 2 * kKVBytes;
-constexpr uint32_t kSmemP = kSmemV + 2 * kKVBytes;
-constexpr uint32_t kSmemO = kSmemP + 2 * kPBytes;
-constexpr uint32_t kSmemTiles = kSmemO + kOBytes;   // 208 KB, 1024-aligned pieces
+constexpr uint32_t kSmemK = kSmemQ + kQBytes;
+constexpr uint32_t kSmemV = kSmemK + KS * kKVBytes;
+constexpr uint32_t kSmemP = kSmemV + VB * kVBlockBytes;
+constexpr uint32_t kSmemO = kSmemP;                 // output staging reuses P buffer 0 (free at the epilogue)
+constexpr uint32_t kSmemTiles = kSmemP + 2 * kPBytes;   // 224 KB, 1024-aligned pieces
+static_assert(kOBytes <= kPBytes, "output staging fits a P buffer");
 constexpr uint32_t kTmemCols = 256;                 // S^T x2 (64 cols each), O^T x2
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr float kRescaleThreshold = 8.0f;           // log2 units
 
-enum Bar { Q_FULL = 0, Q_EMPTY = 2, K_FULL = 4, K_EMPTY = 6, V_FULL = 8, V_EMPTY = 10, S_FULL = 12,
-           S_EMPTY = 14, P_FULL = 16, PV_DONE = 18, O_FULL = 20, O_EMPTY = 22, DRAIN = 24, NUM_BARS = 25 };
+enum Bar { Q_FULL = 0, Q_EMPTY = 1, K_FULL = 2, K_EMPTY = K_FULL + KS, V_FULL = K_EMPTY + KS,
+           V_EMPTY = V_FULL + VB, S_FULL = V_EMPTY + VB, S_EMPTY = S_FULL + 2, P_FULL = S_EMPTY + 2,
+           PV_DONE = P_FULL + 2, O_FULL = PV_DONE + 2, O_EMPTY = O_FULL + 2, DRAIN = O_EMPTY + 2, NUM_BARS = DRAIN + 2 };
 
+// Per-CTA control block after the tiles.  The float arrays are read with
+// 16-byte vector loads, so they come first and are 16-byte aligned.
 struct Smem {
+    alignas(16) float m[64];          // minus the running maximum per query (log2 units)
+    alignas(16) float alpha[64];      // rescale factors of the current tile
+    alignas(16) float red[kSoftmaxWG][4][kCols];   // cross-warp reduction scratch, per warpgroup
+    alignas(16) float inv_l[64];
     uint64_t bar[NUM_BARS];
     uint32_t tmem_base;
     int abort;
-    float m[64];          // running maximum per query (log2 units)
-    float alpha[64];      // rescale factors of the current tile
-    float red[4][64];     // cross-warp reduction scratch
-    float inv_l[64];
 };
+static_assert(offsetof(Smem, m) % 16 == 0 && offsetof(Smem, alpha) % 16 == 0 && offsetof(Smem, inv_l) % 16 == 0,
+              "vector-loaded arrays are 16-byte aligned");
+static_assert(kSmemTiles % 1024 == 0, "the control block starts 16-byte aligned");
 
 struct Params {
     Shape s;
@@ -84,19 +110,20 @@ __device__ __forceinline__ void record_timeout(const Params& p, int where)
     if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = where;
 }
 
-// Column reduction of v[64] over the 128 softmax threads; result for
-// column q in out[q] (q < 64).  MAX selects max, else sum.  Uses named barrier 1.
+// Column reduction of v[kCols] over the 128 threads of softmax warpgroup wg;
+// result for column c in out[c] (c < kCols).  MAX selects max, else sum.
+// Uses named barrier 1 + wg.
 template <bool MAX>
-__device__ __forceinline__ void column_reduce(float (&v)[64], Smem& sm, int tid, float* out)
+__device__ __forceinline__ void column_reduce(float (&v)[kCols], Smem& sm, int wg, int wtid, float* out)
 {
-    const int lane = tid & 31, warp = tid >> 5;
+    const int lane = wtid & 31, warp = wtid >> 5;
 #pragma unroll
     for (int step = 0; step < 5; ++step) {
         const int off = 16 >> step;
-        const int half = 32 >> step;              // values kept after this step
+        const int half = (kCols / 2) >> step;     // values kept after this step
         const bool upper = (lane & off) != 0;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
+        for (int i = 0; i < kCols / 2; ++i) {
             if (i < half) {
                 float keep = upper ? v[i + half] : v[i];
                 float send = upper ? v[i] : v[i + half];
@@ -105,15 +132,25 @@ __device__ __forceinline__ void column_reduce(float (&v)[64], Smem& sm, int tid,
             }
         }
     }
-    // lane holds columns 2*lane, 2*lane+1
-    sm.red[warp][2 * lane] = v[0];
-    sm.red[warp][2 * lane + 1] = v[1];
-    bar_sync(1, kSoftmaxThreads);
-    if (tid < 64) {
-        float a = sm.red[0][tid], b = sm.red[1][tid], c = sm.red[2][tid], d = sm.red[3][tid];
-        out[tid] = MAX ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
+    // lane holds column lane (kCols == 32)
+    static_assert(kCols == 32, "the reduction leaves one column per lane");
+    sm.red[wg][warp][lane] = v[0];
+    bar_sync(1 + wg, kWGThreads);
+    if (wtid < kCols) {
+        float a = sm.red[wg][0][wtid], b = sm.red[wg][1][wtid], c = sm.red[wg][2][wtid], d = sm.red[wg][3][wtid];
+        out[wtid] = MAX ? fmaxf(fmaxf(a, b), fmaxf(c, d)) : (a + b) + (c + d);
     }
-    bar_sync(1, kSoftmaxThreads);
+    bar_sync(1 + wg, kWGThreads);
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
+{
+    float (&a)[16] = *reinterpret_cast<float(*)[16]>(&v[0]);
+    float (&b)[16] = *reinterpret_cast<float(*)[16]>(&v[16]);
+    tmem_ld16(taddr, a);
+    tmem_ld16(taddr + 16, b);
+    tmem_ld_wait(a);
+    reg_fence(b);
 }
 
 __device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64])
@@ -138,7 +175,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                                                                      const Params p)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* tiles = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    // the 128-byte-swizzle atoms need a 1024-byte aligned base; the kernel has
+    // no static shared memory, so the dynamic block starts on the window base
+    if (smem_u32(smem_raw) & 1023u) {
+        if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
+        return;
+    }
+    uint8_t* tiles = smem_raw;
     Smem& sm = *reinterpret_cast<Smem*>(tiles + kSmemTiles);
     const uint32_t sbase = smem_u32(tiles);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -150,28 +193,33 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
 
     if (tid == 0) {
         sm.abort = 0;
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(bar(Q_FULL + i), 1);
-            mbar_init(bar(Q_EMPTY + i), 1);
+        mbar_init(bar(Q_FULL), 1);
+        mbar_init(bar(Q_EMPTY), 1);
+        for (int i = 0; i < KS; ++i) {
             mbar_init(bar(K_FULL + i), 1);
             mbar_init(bar(K_EMPTY + i), 1);
+        }
+        for (int i = 0; i < VB; ++i) {
             mbar_init(bar(V_FULL + i), 1);
             mbar_init(bar(V_EMPTY + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(bar(S_FULL + i), 1);
-            mbar_init(bar(S_EMPTY + i), 4);
-            mbar_init(bar(P_FULL + i), 4);
+            mbar_init(bar(S_EMPTY + i), kSoftmaxWarps);
+            mbar_init(bar(P_FULL + i), kSoftmaxWarps);
             mbar_init(bar(PV_DONE + i), 1);
             mbar_init(bar(O_FULL + i), 1);
-            mbar_init(bar(O_EMPTY + i), 4);
+            mbar_init(bar(O_EMPTY + i), kSoftmaxWarps);
         }
         mbar_init(bar(DRAIN), 1);
+        mbar_init(bar(DRAIN + 1), 1);
         fence_mbar_init();
     }
-    if (warp == 5) {
+    if (warp == kMmaWarp) {
         tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
         tmem_relinquish();
     }
-    if (warp == 4 && lane == 0) {
+    if ((warp == kProducerKWarp || warp == kProducerVWarp) && lane == 0) {
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_k);
         tma_prefetch_desc(&map_v);
@@ -182,224 +230,286 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
     const uint32_t tmem = sm.tmem_base;
     volatile int* abort = &sm.abort;
 
-    if (warp == 4) {
-        // ------------------------------------------------------------ TMA producer
-        if (lane == 0) {
-            int k = 0, issued_q = 0, issued_k = 0, issued_v = 0;
-            bool ok = true;
-            for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
-                const int bh = item / nB, qb = item - bh * nB;
-                const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
-                const int qs = k & 1;
-                if (k >= 2 && !(ok = mbar_wait(bar(Q_EMPTY + qs), ((k >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
-                mbar_expect_tx(bar(Q_FULL + qs), kQBytes);
-                for (int c = 0; c < 2; ++c)
-                    tma_load_3d(sbase + kSmemQ + qs * kQBytes + c * 8192, &map_q, bar(Q_FULL + qs), c * 64, qb * 64, bh);
+    if (warp == kProducerKWarp || warp == kProducerVWarp) {
+        // ------------------------------------------------------------ TMA producers
+        // The loads of a tile are issued from several lanes: the K warp's lanes
+        // 2h + c load d-chunk c of block h of the K pair (8 KB boxes; K keeps
+        // the [chunk][block][row] layout its M = 128 operand needs); the V
+        // warp's lane h loads block h (one 16 KB box, [chunk][row], into a ring
+        // of single-block slots so that V needs no pair alignment).  The K warp
+        // also loads Q (16 KB).
+        const bool is_v = warp == kProducerVWarp;
+        const int h = is_v ? lane : (lane >> 1);        // block of the pair
+        const int kc = lane & 1;                        // K d-chunk (K warp)
+        int k = 0, issued_q = 0, issued_k = 0, issued_vb = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
+            const int bh = item / nB, qb = item - bh * nB;
+            const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
+            if (warp == kProducerKWarp) {
+                if (k >= 1) ok = mbar_wait(bar(Q_EMPTY), (k - 1) & 1, abort, kWaitLimitNs);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                if (lane == 0) {
+                    mbar_expect_tx(bar(Q_FULL), kQBytes);
+                    tma_load_4d(sbase + kSmemQ, &map_q, bar(Q_FULL), 0, qb * 64, 0, bh);
+                }
                 ++issued_q;
-                for (int t = 0; t < T; ++t) {
-                    const int g = k * T + t, st = g & 1;
-                    const int ja = __ldg(kept + 2 * t);
-                    const int jb = 2 * t + 1 < s.n_keep ? __ldg(kept + 2 * t + 1) : -1;
-                    const uint32_t bytes = (jb >= 0 ? 2u : 1u) * 16384u;
-                    if (g >= 2 && !(ok = mbar_wait(bar(K_EMPTY + st), ((g >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
-                    mbar_expect_tx(bar(K_FULL + st), bytes);
-                    for (int c = 0; c < 2; ++c) {
-                        tma_load_3d(sbase + kSmemK + st * kKVBytes + c * 16384, &map_k, bar(K_FULL + st), c * 64,
-                                    ja * 64, bh);
-                        if (jb >= 0)
-                            tma_load_3d(sbase + kSmemK + st * kKVBytes + c * 16384 + 8192, &map_k, bar(K_FULL + st),
-                                        c * 64, jb * 64, bh);
-                    }
-                    ++issued_k;
-                    if (g >= 2 && !(ok = mbar_wait(bar(V_EMPTY + st), ((g >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
-                    mbar_expect_tx(bar(V_FULL + st), bytes);
-                    for (int c = 0; c < 2; ++c) {
-                        tma_load_3d(sbase + kSmemV + st * kKVBytes + c * 16384, &map_v, bar(V_FULL + st), c * 64,
-                                    ja * 64, bh);
-                        if (jb >= 0)
-                            tma_load_3d(sbase + kSmemV + st * kKVBytes + c * 16384 + 8192, &map_v, bar(V_FULL + st),
-                                        c * 64, jb * 64, bh);
-                    }
-                    ++issued_v;
-                }
             }
-            if (!ok) record_timeout(p, 1);
-            // every TMA this thread issued must land before the CTA exits: wait
-            // for the latest issued phase of each buffer, bounded by time only
-            int never = 0;
-            for (int b = 0; b < 2; ++b) {
-                if (issued_q > b) {
-                    const int last = issued_q - 1 - ((issued_q - 1 - b) & 1);
-                    mbar_wait(bar(Q_FULL + b), (last >> 1) & 1, &never, kWaitLimitNs);
-                }
-                if (issued_k > b) {
-                    const int last = issued_k - 1 - ((issued_k - 1 - b) & 1);
-                    mbar_wait(bar(K_FULL + b), (last >> 1) & 1, &never, kWaitLimitNs);
-                }
-                if (issued_v > b) {
-                    const int last = issued_v - 1 - ((issued_v - 1 - b) & 1);
-                    mbar_wait(bar(V_FULL + b), (last >> 1) & 1, &never, kWaitLimitNs);
+            for (int t = 0; t < T; ++t) {
+                const int g = k * T + t;
+                const int ja = __ldg(kept + 2 * t);
+                const int jb = 2 * t + 1 < s.n_keep ? __ldg(kept + 2 * t + 1) : -1;
+                const int nblk = jb >= 0 ? 2 : 1;
+                if (is_v) {
+                    // cumulative block index of block h of this tile; both lanes
+                    // wait for their slots, then issue together (or neither does)
+                    const int c = k * s.n_keep + 2 * t + h;
+                    const int slot = c % VB;
+                    bool okl = true;
+                    if (lane < 2 && h < nblk && c >= VB)
+                        okl = mbar_wait(bar(V_EMPTY + slot), ((c / VB) - 1) & 1, abort, kWaitLimitNs);
+                    ok = __shfl_sync(0xffffffffu, okl, 0) && __shfl_sync(0xffffffffu, okl, 1);
+                    if (!ok) break;
+                    if (lane < 2 && h < nblk) {
+                        mbar_expect_tx(bar(V_FULL + slot), kVBlockBytes);
+                        tma_load_4d(sbase + kSmemV + slot * kVBlockBytes, &map_v, bar(V_FULL + slot), 0,
+                                    (h ? jb : ja) * 64, 0, bh);
+                    }
+                    issued_vb += nblk;
+                } else {
+                    const int st = g % KS;
+                    if (g >= KS) ok = mbar_wait(bar(K_EMPTY + st), ((g / KS) - 1) & 1, abort, kWaitLimitNs);
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) break;
+                    if (lane == 0) mbar_expect_tx(bar(K_FULL + st), nblk * 16384u);
+                    __syncwarp();
+                    if (lane < 4 && h < nblk)
+                        tma_load_3d(sbase + kSmemK + st * kKVBytes + kc * 16384 + h * 8192, &map_k, bar(K_FULL + st),
+                                    kc * 64, (h ? jb : ja) * 64, bh);
+                    ++issued_k;
                 }
             }
         }
-    } else if (warp == 5) {
-        // ------------------------------------------------------------ MMA issuer
+        if (!ok && lane == 0) record_timeout(p, is_v ? 4 : 1);
+        // every copy this warp issued must land before the CTA exits: wait for
+        // the latest issued phase of each buffer, bounded by time only
         if (lane == 0) {
+            int never = 0;
+            if (issued_q > 0) mbar_wait(bar(Q_FULL), (issued_q - 1) & 1, &never, kWaitLimitNs);
+            const int NS = is_v ? VB : KS, issued = is_v ? issued_vb : issued_k;
+            const int full0 = is_v ? V_FULL : K_FULL;
+            for (int b = 0; b < NS; ++b) {
+                if (issued > b) {
+                    const int last = issued - 1 - ((issued - 1 - b) % NS);   // latest use of slot b
+                    mbar_wait(bar(full0 + b), (last / NS) & 1, &never, kWaitLimitNs);
+                }
+            }
+        }
+    } else if (warp == kMmaWarp || warp == kPvWarp) {
+        // ------------------------------------------------------------ MMA issuers
+        // Two issuing warps, so that a P V waiting for the softmax never holds
+        // back the next Q K^T (and vice versa); each commits only its own MMAs.
+        // Descriptors are built once; a K step adds its offset (in 16-byte
+        // units) to the low word.
+        if (lane == 0) {
+            const bool pv = warp == kPvWarp;
             const uint32_t id_qk = idesc_bf16(128, 64, false, false);
             const uint32_t id_pv = idesc_bf16(128, 64, true, true);
+            const uint64_t dq = smem_desc(sbase + kSmemQ, 16, 1024);            // Q: B of Q K^T (K-major)
+            const uint64_t dk = smem_desc(sbase + kSmemK, 16, 1024);            // K pair ring: A of Q K^T
+            const uint64_t dv = smem_desc(sbase + kSmemV, 8192, 1024);          // V block ring: A of P V (MN-major)
+            const uint64_t dp = smem_desc(sbase + kSmemP, 8192, 1024);          // P^T: B of P V (MN-major)
+            const uint32_t q_lo = (uint32_t)dq, q_hi = (uint32_t)(dq >> 32);
+            const uint32_t k_lo = (uint32_t)dk, k_hi = (uint32_t)(dk >> 32);
+            const uint32_t v_lo = (uint32_t)dv, v_hi = (uint32_t)(dv >> 32);
+            const uint32_t p_lo = (uint32_t)dp, p_hi = (uint32_t)(dp >> 32);
             bool ok = true;
             int k = 0;
-            // PV of global tile gp (item-local tile tp) into O buffer ob
-            auto issue_pv = [&](int gp, int tp, int ob, int kitem) -> bool {
-                const int pb = gp & 1;
-                if (!mbar_wait(bar(P_FULL + pb), (gp >> 1) & 1, abort, kWaitLimitNs)) return false;
-                if (!mbar_wait(bar(V_FULL + pb), (gp >> 1) & 1, abort, kWaitLimitNs)) return false;
-                if (tp == 0 && kitem >= 2 &&
-                    !mbar_wait(bar(O_EMPTY + ob), ((kitem >> 1) - 1) & 1, abort, kWaitLimitNs))
-                    return false;
-                fence_after_sync();
-                const bool half = 2 * tp + 1 >= s.n_keep;
-                const uint32_t vaddr = sbase + kSmemV + pb * kKVBytes;
-                const uint32_t paddr = sbase + kSmemP + pb * kPBytes;
-                const uint32_t d = tmem + 128 + ob * 64;
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    if (half && kk >= 4) break;
-                    mma_ss(d, smem_desc(vaddr + kk * 2048, 16384, 1024), smem_desc(paddr + kk * 2048, 8192, 1024),
-                           id_pv, (tp > 0 || kk > 0) ? 1u : 0u);
-                }
-                mma_commit(bar(PV_DONE + pb));
-                mma_commit(bar(V_EMPTY + pb));
-                return true;
-            };
             for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
-                const int qs = k & 1, ob = k & 1;
-                if (!(ok = mbar_wait(bar(Q_FULL + qs), (k >> 1) & 1, abort, kWaitLimitNs))) break;
-                const uint32_t qaddr = sbase + kSmemQ + qs * kQBytes;
-                for (int t = 0; t < T; ++t) {
-                    const int g = k * T + t, st = g & 1;
-                    if (!(ok = mbar_wait(bar(K_FULL + st), (g >> 1) & 1, abort, kWaitLimitNs))) break;
-                    if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + st), ((g >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
-                    fence_after_sync();
-                    const uint32_t kaddr = sbase + kSmemK + st * kKVBytes;
-                    const uint32_t d = tmem + st * 64;
+                const int ob = k & 1;
+                if (!pv) {
+                    if (!(ok = mbar_wait(bar(Q_FULL), k & 1, abort, kWaitLimitNs))) break;
+                    for (int t = 0; t < T; ++t) {
+                        const int g = k * T + t, sb = g & 1, ks = g % KS;
+                        if (!(ok = mbar_wait(bar(K_FULL + ks), (g / KS) & 1, abort, kWaitLimitNs))) break;
+                        if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + sb), ((g >> 1) - 1) & 1, abort, kWaitLimitNs)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t a = k_lo + ks * (kKVBytes >> 4);
+                        const uint32_t d = tmem + sb * 64;
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk)
-                        mma_ss(d, smem_desc(kaddr + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                               smem_desc(qaddr + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
-                    mma_commit(bar(S_FULL + st));
-                    mma_commit(bar(K_EMPTY + st));
-                    if (t == T - 1) mma_commit(bar(Q_EMPTY + qs));
-                    if (t >= 1 && !(ok = issue_pv(g - 1, t - 1, ob, k))) break;
+                        for (int kk = 0; kk < 8; ++kk)
+                            mma_ss_split(d, a + (kk >> 2) * 1024 + (kk & 3) * 2, k_hi,
+                                         q_lo + (kk >> 2) * 512 + (kk & 3) * 2, q_hi, id_qk, kk > 0 ? 1u : 0u);
+                        mma_commit(bar(S_FULL + sb));
+                        mma_commit(bar(K_EMPTY + ks));
+                        if (t == T - 1) mma_commit(bar(Q_EMPTY));
+                    }
+                } else {
+                    for (int t = 0; t < T; ++t) {
+                        const int g = k * T + t, pb = g & 1;
+                        const bool half = 2 * t + 1 >= s.n_keep;
+                        const int c0 = k * s.n_keep + 2 * t;             // cumulative index of block a
+                        const int va = c0 % VB, vb = (c0 + 1) % VB;
+                        if (!(ok = mbar_wait(bar(P_FULL + pb), (g >> 1) & 1, abort, kWaitLimitNs))) break;
+                        if (!(ok = mbar_wait(bar(V_FULL + va), (c0 / VB) & 1, abort, kWaitLimitNs))) break;
+                        if (!half && !(ok = mbar_wait(bar(V_FULL + vb), ((c0 + 1) / VB) & 1, abort, kWaitLimitNs)))
+                            break;
+                        if (t == 0 && k >= 2 &&
+                            !(ok = mbar_wait(bar(O_EMPTY + ob), ((k >> 1) - 1) & 1, abort, kWaitLimitNs)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t a0 = v_lo + va * (kVBlockBytes >> 4), a1 = v_lo + vb * (kVBlockBytes >> 4);
+                        const uint32_t b0 = p_lo + pb * (kPBytes >> 4);
+                        const uint32_t d = tmem + 128 + ob * 64;
+                        mma_ss_split(d, a0, v_hi, b0, p_hi, id_pv, t > 0 ? 1u : 0u);
+#pragma unroll
+                        for (int kk = 1; kk < 4; ++kk)
+                            mma_ss_split(d, a0 + kk * 128, v_hi, b0 + kk * 128, p_hi, id_pv, 1u);
+                        if (!half) {
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk)
+                                mma_ss_split(d, a1 + kk * 128, v_hi, b0 + (4 + kk) * 128, p_hi, id_pv, 1u);
+                        }
+                        mma_commit(bar(PV_DONE + pb));
+                        mma_commit(bar(V_EMPTY + va));
+                        if (!half) mma_commit(bar(V_EMPTY + vb));
+                    }
+                    if (!ok) break;
+                    mma_commit(bar(O_FULL + ob));
                 }
-                if (!ok) break;
-                if (!(ok = issue_pv(k * T + T - 1, T - 1, ob, k))) break;
-                mma_commit(bar(O_FULL + ob));
             }
-            if (!ok) record_timeout(p, 2);
-            // drain: every MMA issued by this thread completes before TMEM is released
+            if (!ok) record_timeout(p, pv ? 5 : 2);
+            // drain: every MMA this thread issued completes before TMEM is released
             int never = 0;
-            mma_commit(bar(DRAIN));
-            mbar_wait(bar(DRAIN), 0, &never, kWaitLimitNs);
+            const uint32_t drain = bar(pv ? DRAIN + 1 : DRAIN);
+            mma_commit(drain);
+            mbar_wait(drain, 0, &never, kWaitLimitNs);
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue
+        // Softmax warpgroup wg owns query columns [32 wg, 32 wg + 32) of every
+        // tile; thread wtid owns key wtid of the tile (TMEM lane wtid).  Per key
+        // and query: t = s * log2(e)/sqrt(d) - m_q (one FFMA against the stored
+        // -m_q), p = 2^t.  A tile whose t exceeds the threshold anywhere in the
+        // warpgroup's columns takes the rescale path: exact column maxima of t,
+        // m_q += max(tmax_q, 0), O^T columns and row sums scaled by 2^-delta.
+        // The first tile of a query block starts from m_q = 0 and always takes
+        // that path with delta = tmax (m_q becomes the tile's exact maximum).
+        const int wg = warp >> 2, wtid = tid & 127;
+        const int col0 = wg * kCols;
         const float c_log2 = s.sm_scale_log2;
-        const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+        const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
         bool ok = true;
         int k = 0;
         for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
             const int bh = item / nB, qb = item - bh * nB;
             const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
             const int ob = k & 1;
-            if (tid < 64) sm.m[tid] = -INFINITY;
-            float l[64];
+            if (wtid < kCols) sm.m[col0 + wtid] = 0.0f;       // holds -m_q
+            float l[kCols];
 #pragma unroll
-            for (int q = 0; q < 64; ++q) l[q] = 0.0f;
-            bar_sync(1, kSoftmaxThreads);
+            for (int q = 0; q < kCols; ++q) l[q] = 0.0f;
+            int ja_n = __ldg(kept);
+            int jb_n = s.n_keep > 1 ? __ldg(kept + 1) : -1;
+            bar_sync(1 + wg, kWGThreads);
             for (int t = 0; t < T; ++t) {
                 const int g = k * T + t, sb = g & 1;
-                const int ja = __ldg(kept + 2 * t);
-                const int jb = 2 * t + 1 < s.n_keep ? __ldg(kept + 2 * t + 1) : -1;
-                const int blk = tid < 64 ? ja : jb;
-                const int key = blk * 64 + (tid & 63);
+                const int ja = ja_n, jb = jb_n;
+                if (t + 1 < T) {                               // kept ids of the next tile, one tile ahead
+                    ja_n = __ldg(kept + 2 * t + 2);
+                    jb_n = 2 * t + 3 < s.n_keep ? __ldg(kept + 2 * t + 3) : -1;
+                }
+                const int blk = wtid < 64 ? ja : jb;
+                const int key = blk * 64 + (wtid & 63);
                 const bool valid = blk >= 0 && key < s.N;
                 if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, kWaitLimitNs))) break;
                 fence_after_sync();
-                const uint32_t saddr = tmem + lane_off + sb * 64;
-                float x[64];
-                tmem_ld64(saddr, x);
-                bool need = false;
+                const uint32_t saddr = tmem + lane_off + sb * 64 + col0;
+                float x[kCols];
+                tmem_ld32(saddr, x);
+                bool need = t == 0;
+                if (valid) {
 #pragma unroll
-                for (int q = 0; q < 64; q += 4) {
-                    float4 m4 = *reinterpret_cast<const float4*>(&sm.m[q]);
-                    float mm[4] = {m4.x, m4.y, m4.z, m4.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        float xv = valid ? x[q + e] * c_log2 : -INFINITY;
-                        x[q + e] = xv;
-                        need |= xv > mm[e] + kRescaleThreshold;
+                    for (int q = 0; q < kCols; q += 4) {
+                        const float4 nm = *reinterpret_cast<const float4*>(&sm.m[col0 + q]);
+                        x[q] = fmaf(x[q], c_log2, nm.x);
+                        x[q + 1] = fmaf(x[q + 1], c_log2, nm.y);
+                        x[q + 2] = fmaf(x[q + 2], c_log2, nm.z);
+                        x[q + 3] = fmaf(x[q + 3], c_log2, nm.w);
+                        need |= (x[q] > kRescaleThreshold) | (x[q + 1] > kRescaleThreshold) |
+                                (x[q + 2] > kRescaleThreshold) | (x[q + 3] > kRescaleThreshold);
                     }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < kCols; ++q) x[q] = -INFINITY;
                 }
-                if (bar_red_or(1, kSoftmaxThreads, need)) {
-                    column_reduce<true>(x, sm, tid, sm.alpha);        // alpha <- tile maxima (x consumed)
-                    if (tid < 64) {
-                        const float mo = sm.m[tid];
-                        const float mn = fmaxf(mo, sm.alpha[tid]);
-                        sm.alpha[tid] = fast_exp2(mo - mn);            // 0 when mo = -inf
-                        sm.m[tid] = mn;
+                if (bar_red_or(1 + wg, kWGThreads, need)) {
+                    column_reduce<true>(x, sm, wg, wtid, sm.alpha + col0);   // alpha <- column maxima of t
+                    if (wtid < kCols) {
+                        const float tmax = sm.alpha[col0 + wtid];
+                        const float delta = t == 0 ? tmax : fmaxf(tmax, 0.0f);
+                        sm.m[col0 + wtid] -= delta;
+                        sm.alpha[col0 + wtid] = fast_exp2(-delta);
                     }
-                    bar_sync(1, kSoftmaxThreads);
-                    tmem_ld64(saddr, x);                               // S^T is still ours: reload
+                    bar_sync(1 + wg, kWGThreads);
+                    tmem_ld32(saddr, x);                                     // S^T is still ours: recompute t
+                    if (valid) {
 #pragma unroll
-                    for (int q = 0; q < 64; ++q) x[q] = valid ? x[q] * c_log2 : -INFINITY;
+                        for (int q = 0; q < kCols; q += 4) {
+                            const float4 nm = *reinterpret_cast<const float4*>(&sm.m[col0 + q]);
+                            x[q] = fmaf(x[q], c_log2, nm.x);
+                            x[q + 1] = fmaf(x[q + 1], c_log2, nm.y);
+                            x[q + 2] = fmaf(x[q + 2], c_log2, nm.z);
+                            x[q + 3] = fmaf(x[q + 3], c_log2, nm.w);
+                        }
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < kCols; ++q) x[q] = -INFINITY;
+                    }
                     if (t > 0) {
                         // O^T must hold PV(t-1) before it is rescaled
                         if (!(ok = mbar_wait(bar(PV_DONE + ((g - 1) & 1)), ((g - 1) >> 1) & 1, abort, kWaitLimitNs)))
                             break;
                         fence_after_sync();
-                        const uint32_t oaddr = tmem + lane_off + 128 + ob * 64;
+                        const uint32_t oaddr = tmem + lane_off + 128 + ob * 64 + col0;
 #pragma unroll
-                        for (int c = 0; c < 4; ++c) {
+                        for (int c = 0; c < kCols / 16; ++c) {
                             float ov[16];
                             tmem_ld16(oaddr + c * 16, ov);
                             tmem_ld_wait(ov);
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) ov[e] *= sm.alpha[c * 16 + e];
+                            for (int e = 0; e < 16; ++e) ov[e] *= sm.alpha[col0 + c * 16 + e];
                             tmem_st16(oaddr + c * 16, ov);
                         }
                         tmem_st_wait();
 #pragma unroll
-                        for (int q = 0; q < 64; ++q) l[q] *= sm.alpha[q];
+                        for (int q = 0; q < kCols; ++q) l[q] *= sm.alpha[col0 + q];
                     }
                 }
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));
-                // P^T row of this key, bf16, 128-byte-swizzled
-                uint32_t pk[32];
+                // p = 2^t; this warpgroup's half of the key's P^T row, bf16, 128-byte-swizzled
+                uint32_t pk[kCols / 2];
 #pragma unroll
-                for (int q = 0; q < 64; q += 4) {
-                    float4 m4 = *reinterpret_cast<const float4*>(&sm.m[q]);
-                    float mm[4] = {m4.x, m4.y, m4.z, m4.w};
-#pragma unroll
-                    for (int e = 0; e < 4; e += 2) {
-                        float p0 = fast_exp2(x[q + e] - mm[e]);
-                        float p1 = fast_exp2(x[q + e + 1] - mm[e + 1]);
-                        uint32_t u = pack_bf16(p0, p1);
-                        float2 r = unpack_bf16(u);
-                        l[q + e] += r.x;
-                        l[q + e + 1] += r.y;
-                        pk[(q + e) >> 1] = u;
-                    }
+                for (int q = 0; q < kCols; q += 2) {
+                    const float p0 = fast_exp2(x[q]);
+                    const float p1 = fast_exp2(x[q + 1]);
+                    l[q] += p0;
+                    l[q + 1] += p1;
+                    pk[q >> 1] = pack_bf16(p0, p1);
                 }
                 if (g >= 2 && !(ok = mbar_wait(bar(PV_DONE + sb), ((g >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
-                const uint32_t prow = sbase + kSmemP + sb * kPBytes + (tid >> 3) * 1024 + (tid & 7) * 128;
+                const uint32_t prow = sbase + kSmemP + sb * kPBytes + (wtid >> 3) * 1024 + (wtid & 7) * 128;
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + ((c ^ (tid & 7)) << 4)),
+                for (int c = 0; c < kCols / 8; ++c) {
+                    const int chunk = wg * (kCols / 8) + c;
+                    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + ((chunk ^ (wtid & 7)) << 4)),
                                  "r"(pk[4 * c]), "r"(pk[4 * c + 1]), "r"(pk[4 * c + 2]), "r"(pk[4 * c + 3])
                                  : "memory");
+                }
                 fence_proxy_async_smem();
                 fence_before_sync();
                 __syncwarp();
@@ -409,39 +519,40 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             // ---- epilogue: O^s = O^T / l, transposed through shared memory
             if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, kWaitLimitNs))) break;
             fence_after_sync();
-            column_reduce<false>(l, sm, tid, sm.inv_l);
-            if (tid < 64) sm.inv_l[tid] = 1.0f / sm.inv_l[tid];
-            bar_sync(1, kSoftmaxThreads);
+            column_reduce<false>(l, sm, wg, wtid, sm.inv_l + col0);
+            if (wtid < kCols) sm.inv_l[col0 + wtid] = 1.0f / sm.inv_l[col0 + wtid];
+            bar_sync(1 + wg, kWGThreads);
             {
-                float ov[64];
-                tmem_ld64(tmem + lane_off + 128 + ob * 64, ov);
+                float ov[kCols];
+                tmem_ld32(tmem + lane_off + 128 + ob * 64 + col0, ov);
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
                 __nv_bfloat16* ostage = reinterpret_cast<__nv_bfloat16*>(tiles + kSmemO);
 #pragma unroll
-                for (int q = 0; q < 64; ++q) ostage[q * 128 + tid] = __float2bfloat16_rn(ov[q] * sm.inv_l[q]);
+                for (int q = 0; q < kCols; ++q)
+                    ostage[(col0 + q) * 128 + wtid] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
             }
-            bar_sync(1, kSoftmaxThreads);
+            bar_sync(1 + kSoftmaxWG, kSoftmaxWarps * 32);                  // both halves staged
             {
                 const uint4* src = reinterpret_cast<const uint4*>(tiles + kSmemO);
                 __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64) * kDh;
 #pragma unroll
-                for (int it = 0; it < 8; ++it) {
-                    const int e = it * kSoftmaxThreads + tid;
+                for (int it = 0; it < 1024 / (kSoftmaxWarps * 32); ++it) {
+                    const int e = it * kSoftmaxWarps * 32 + tid;
                     const int row = e >> 4, c = e & 15;
                     if (qb * 64 + row < s.N)
                         *reinterpret_cast<uint4*>(dst + (size_t)row * kDh + c * 8) = src[e];
                 }
             }
-            bar_sync(1, kSoftmaxThreads);
+            bar_sync(1 + kSoftmaxWG, kSoftmaxWarps * 32);
         }
         if (!ok) record_timeout(p, 3);
     }
     fence_before_sync();
     __syncthreads();
     fence_after_sync();
-    if (warp == 5) tmem_dealloc(tmem, kTmemCols);
+    if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
@@ -458,9 +569,9 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// [BH][N][128] bf16 viewed as a 3-D tensor (d, token, head); 64 x 64 boxes,
-// 128-byte swizzle; rows past N read as zero.
-bool make_map(CUtensorMap* m, const void* ptr, const Shape& s)
+// [BH][N][128] bf16 viewed as a 3-D tensor (d, token, head); 64 x 64 boxes
+// (one d-chunk of a key block), 128-byte swizzle; rows past N read as zero.
+bool make_map3(CUtensorMap* m, const void* ptr, const Shape& s)
 {
     auto enc = encode_fn();
     if (!enc) return false;
@@ -473,13 +584,29 @@ bool make_map(CUtensorMap* m, const void* ptr, const Shape& s)
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same tensor viewed as 4-D (d within chunk, token, d-chunk, head) so that
+// one 64 x 64 x 2 box brings a whole key block in as [chunk][row][64]: 16 KB,
+// 128-byte swizzle, rows past N read as zero.
+bool make_map4(CUtensorMap* m, const void* ptr, const Shape& s)
+{
+    auto enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[4] = {64, (cuuint64_t)s.N, 2, (cuuint64_t)s.B * s.H};
+    cuuint64_t strides[3] = {(cuuint64_t)kDh * 2, 128, (cuuint64_t)s.N * kDh * 2};
+    cuuint32_t box[4] = {64, 64, 2, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
                                   const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st)
 {
     CUtensorMap mq, mk, mv;
-    if (!make_map(&mq, qr, s) || !make_map(&mk, kr, s) || !make_map(&mv, v, s)) return cudaErrorInvalidValue;
+    if (!make_map4(&mq, qr, s) || !make_map3(&mk, kr, s) || !make_map4(&mv, v, s)) return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -492,7 +619,7 @@ cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr
     p.status = status;
     p.total_items = s.B * s.H * s.nB;
     p.tiles = (s.n_keep + 1) / 2;
-    const size_t smem = 1024 + kSmemTiles + sizeof(Smem);
+    const size_t smem = kSmemTiles + sizeof(Smem);
     e = cudaFuncSetAttribute(sparse_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = p.total_items < nsm ? p.total_items : nsm;
