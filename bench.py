@@ -34,6 +34,12 @@ sys.path.insert(0, ROOT)
 METRIC = "RoLA attn layer ms & tokens/s (Wan2.1-14B 720p shape); % of TC/HBM roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the current sparse
+# kernel from one ncu capture of the 480p layer (12 heads x 32760 tokens), scaled
+# to a launch by heads x tokens (the traffic is the streaming q^r, k^r, v reads and
+# the O^s write, which grow in proportion).  Set to None whenever the kernel changes.
+SPARSE_TRAFFIC_PER_HEAD_TOKEN = (303.255296e6 + 87.174656e6) / (12 * 32760)
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -295,8 +301,11 @@ def main():
     sp_ms = stage_ms["sparse_attn"]
     achieved = fl / (sp_ms * 1e-3) / 1e12
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    traffic = None
+    if SPARSE_TRAFFIC_PER_HEAD_TOKEN is not None:
+        traffic = SPARSE_TRAFFIC_PER_HEAD_TOKEN * cfg["B"] * cfg["H"] * cfg["N"]
     roofline = {"bound": "tensor", "kernel": "sparse_attn", "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16_tflops_sustained",
                 "algorithmic_flops_per_launch": fl, "ms_per_launch": sp_ms}
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))

@@ -26,7 +26,8 @@
 // Warp roles (384 threads, one persistent CTA per SM):
 //   warps 0-7  softmax + epilogue: two warpgroups, each owning 32 of the 64
 //              query columns of every tile (warp w reads TMEM lanes
-//              32 (w mod 4) .. +31, so both warpgroups see all 128 keys)
+//              32 (w mod 4) .. +31, so every warpgroup sees all 128 keys;
+//              the warpgroup count is a compile-time parameter)
 //   warp  8    TMA producer: Q (per query block) and the K pairs
 //   warp  9    TMA producer: the V blocks
 //   warp 10    Q K^T issuer and TMEM owner
@@ -112,13 +113,16 @@ __device__ __forceinline__ void record_timeout(const Params& p, int where)
 
 // Column reduction of v[kCols] over the 128 threads of softmax warpgroup wg;
 // result for column c in out[c] (c < kCols).  MAX selects max, else sum.
-// Uses named barrier 1 + wg.
+// A butterfly halves the columns a lane holds at each step; with kCols = 16
+// a last exchange leaves column lane / 2 on lanes 2c and 2c + 1.  Uses named
+// barrier 1 + wg.
 template <bool MAX>
 __device__ __forceinline__ void column_reduce(float (&v)[kCols], Smem& sm, int wg, int wtid, float* out)
 {
     const int lane = wtid & 31, warp = wtid >> 5;
+    constexpr int kSteps = kCols == 32 ? 5 : 4;
 #pragma unroll
-    for (int step = 0; step < 5; ++step) {
+    for (int step = 0; step < kSteps; ++step) {
         const int off = 16 >> step;
         const int half = (kCols / 2) >> step;     // values kept after this step
         const bool upper = (lane & off) != 0;
@@ -132,9 +136,13 @@ __device__ __forceinline__ void column_reduce(float (&v)[kCols], Smem& sm, int w
             }
         }
     }
-    // lane holds column lane (kCols == 32)
-    static_assert(kCols == 32, "the reduction leaves one column per lane");
-    sm.red[wg][warp][lane] = v[0];
+    int col = lane;
+    if (kCols == 16) {
+        const float recv = __shfl_xor_sync(0xffffffffu, v[0], 1);
+        v[0] = MAX ? fmaxf(v[0], recv) : v[0] + recv;
+        col = lane >> 1;
+    }
+    if (kCols == 32 || (lane & 1) == 0) sm.red[wg][warp][col] = v[0];
     bar_sync(1 + wg, kWGThreads);
     if (wtid < kCols) {
         float a = sm.red[wg][0][wtid], b = sm.red[wg][1][wtid], c = sm.red[wg][2][wtid], d = sm.red[wg][3][wtid];
@@ -143,30 +151,15 @@ __device__ __forceinline__ void column_reduce(float (&v)[kCols], Smem& sm, int w
     bar_sync(1 + wg, kWGThreads);
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
+template <int NC>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[NC])
 {
-    float (&a)[16] = *reinterpret_cast<float(*)[16]>(&v[0]);
-    float (&b)[16] = *reinterpret_cast<float(*)[16]>(&v[16]);
-    tmem_ld16(taddr, a);
-    tmem_ld16(taddr + 16, b);
-    tmem_ld_wait(a);
-    reg_fence(b);
-}
-
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64])
-{
-    float (&a)[16] = *reinterpret_cast<float(*)[16]>(&v[0]);
-    float (&b)[16] = *reinterpret_cast<float(*)[16]>(&v[16]);
-    float (&c)[16] = *reinterpret_cast<float(*)[16]>(&v[32]);
-    float (&d)[16] = *reinterpret_cast<float(*)[16]>(&v[48]);
-    tmem_ld16(taddr, a);
-    tmem_ld16(taddr + 16, b);
-    tmem_ld16(taddr + 32, c);
-    tmem_ld16(taddr + 48, d);
-    tmem_ld_wait(a);
-    reg_fence(b);
-    reg_fence(c);
-    reg_fence(d);
+    static_assert(NC % 16 == 0, "loads of 16 columns");
+#pragma unroll
+    for (int c = 0; c < NC / 16; ++c) tmem_ld16(taddr + c * 16, *reinterpret_cast<float(*)[16]>(&v[c * 16]));
+    tmem_ld_wait(*reinterpret_cast<float(*)[16]>(&v[0]));
+#pragma unroll
+    for (int c = 1; c < NC / 16; ++c) reg_fence(*reinterpret_cast<float(*)[16]>(&v[c * 16]));
 }
 
 __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
@@ -428,7 +421,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 fence_after_sync();
                 const uint32_t saddr = tmem + lane_off + sb * 64 + col0;
                 float x[kCols];
-                tmem_ld32(saddr, x);
+                tmem_ld_cols<kCols>(saddr, x);
+                float s_raw[kCols];                            // kept for the rare rescale path
+#pragma unroll
+                for (int q = 0; q < kCols; ++q) s_raw[q] = x[q];
+                fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));  // S^T buffer free for Q K^T(g + 2)
                 bool need = t == 0;
                 if (valid) {
 #pragma unroll
@@ -454,15 +453,14 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                         sm.alpha[col0 + wtid] = fast_exp2(-delta);
                     }
                     bar_sync(1 + wg, kWGThreads);
-                    tmem_ld32(saddr, x);                                     // S^T is still ours: recompute t
-                    if (valid) {
+                    if (valid) {                                                     // recompute t against the new m
 #pragma unroll
                         for (int q = 0; q < kCols; q += 4) {
                             const float4 nm = *reinterpret_cast<const float4*>(&sm.m[col0 + q]);
-                            x[q] = fmaf(x[q], c_log2, nm.x);
-                            x[q + 1] = fmaf(x[q + 1], c_log2, nm.y);
-                            x[q + 2] = fmaf(x[q + 2], c_log2, nm.z);
-                            x[q + 3] = fmaf(x[q + 3], c_log2, nm.w);
+                            x[q] = fmaf(s_raw[q], c_log2, nm.x);
+                            x[q + 1] = fmaf(s_raw[q + 1], c_log2, nm.y);
+                            x[q + 2] = fmaf(s_raw[q + 2], c_log2, nm.z);
+                            x[q + 3] = fmaf(s_raw[q + 3], c_log2, nm.w);
                         }
                     } else {
 #pragma unroll
@@ -488,10 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                         for (int q = 0; q < kCols; ++q) l[q] *= sm.alpha[col0 + q];
                     }
                 }
-                fence_before_sync();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));
-                // p = 2^t; this warpgroup's half of the key's P^T row, bf16, 128-byte-swizzled
+                // p = 2^t; this warpgroup's columns of the key's P^T row, bf16, 128-byte-swizzled
                 uint32_t pk[kCols / 2];
 #pragma unroll
                 for (int q = 0; q < kCols; q += 2) {
@@ -524,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             bar_sync(1 + wg, kWGThreads);
             {
                 float ov[kCols];
-                tmem_ld32(tmem + lane_off + 128 + ob * 64 + col0, ov);
+                tmem_ld_cols<kCols>(tmem + lane_off + 128 + ob * 64 + col0, ov);
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
