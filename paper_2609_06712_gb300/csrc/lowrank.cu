@@ -331,7 +331,9 @@ cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, 
 // apply, bf16: CTA = (64-token block, head), 4 warps x 16 tokens.
 //   U = Q P_q^T -> q~ = R_r SiLU(U) (registers, never stored) -> y = q~ C (MMA,
 //   C in bf16) -> O^lr = y / sqrt(mean y^2 + eps_lr) -> fuse with O^s.
-// Shared memory: P_q r x 256 B | C r x 256 B | Q 16 KB, all 256-byte rows, swizzled.
+// Shared memory: P_q r x 256 B | C r x 256 B | Q 16 KB | O^s 16 KB, all 256-byte
+// rows, swizzled.  O^s comes in and O goes out through the shared tile with
+// 16-byte accesses.
 
 template <int R>
 __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
@@ -348,10 +350,13 @@ __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfl
     const uint32_t sP = smem_u32(smem);
     const uint32_t sC = sP + R * 256;
     const uint32_t sQ = sC + R * 256;
+    const uint32_t sO = sQ + kBlock * 256;
+    uint8_t* o_gen = smem + 2 * R * 256 + kBlock * 256;
     const size_t head = (size_t)bh * s.N * kDh;
     load_rows_async(sP, Pq + (size_t)h * R * kDh, 0, R, R, tid, 128);
     load_rows_async(sC, Cbf + (size_t)bh * R * kDh, 0, R, R, tid, 128);
     load_rows_async(sQ, q + head, blk * kBlock, kBlock, s.N, tid, 128);
+    load_rows_async(sO, o_s + head, blk * kBlock, kBlock, s.N, tid, 128);
     cp_async_commit();
     cp_async_wait<0>();
     __syncthreads();
@@ -397,13 +402,14 @@ __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfl
         }
     }
     // per-row RMS of y and of O^s (the 4 lanes of a quad share a row)
+    const int r_lo = warp * 16 + g, r_hi = r_lo + 8;                 // rows within the tile
     float os[16][4];
     float ssy[2] = {0.0f, 0.0f}, sso[2] = {0.0f, 0.0f};
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) {
-        int col = dt * 8 + t4 * 2;
-        float2 lo = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_s + head + (size_t)n_lo_c * kDh + col));
-        float2 hi = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_s + head + (size_t)n_hi_c * kDh + col));
+        const uint32_t lo_off = sw128(r_lo, dt) + t4 * 4, hi_off = sw128(r_hi, dt) + t4 * 4;
+        float2 lo = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + lo_off));
+        float2 hi = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + hi_off));
         os[dt][0] = lo.x; os[dt][1] = lo.y; os[dt][2] = hi.x; os[dt][3] = hi.y;
         ssy[0] += y[dt][0] * y[dt][0] + y[dt][1] * y[dt][1];
         ssy[1] += y[dt][2] * y[dt][2] + y[dt][3] * y[dt][3];
@@ -422,15 +428,23 @@ __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfl
         float rp = sqrtf(sso[hr] * (1.0f / kDh) + s.eps_fuse);
         coef[hr] = gp * rp * rsqrtf(ssy[hr] * (1.0f / kDh) + s.eps_lr);
     }
+    // fused rows back into the shared tile (each thread rewrites what it read), then 16-byte stores
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) {
-        int col = dt * 8 + t4 * 2;
-        if (n_lo < s.N)
-            *reinterpret_cast<uint32_t*>(o + head + (size_t)n_lo * kDh + col) =
-                pack_bf16(os[dt][0] + coef[0] * y[dt][0], os[dt][1] + coef[0] * y[dt][1]);
-        if (n_hi < s.N)
-            *reinterpret_cast<uint32_t*>(o + head + (size_t)n_hi * kDh + col) =
-                pack_bf16(os[dt][2] + coef[1] * y[dt][2], os[dt][3] + coef[1] * y[dt][3]);
+        *reinterpret_cast<uint32_t*>(o_gen + sw128(r_lo, dt) + t4 * 4) =
+            pack_bf16(os[dt][0] + coef[0] * y[dt][0], os[dt][1] + coef[0] * y[dt][1]);
+        *reinterpret_cast<uint32_t*>(o_gen + sw128(r_hi, dt) + t4 * 4) =
+            pack_bf16(os[dt][2] + coef[1] * y[dt][2], os[dt][3] + coef[1] * y[dt][3]);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+        const int e = it * 128 + tid;
+        const int row = e >> 4, c = e & 15;
+        const int n = blk * kBlock + row;
+        if (n < s.N)
+            *reinterpret_cast<uint4*>(o + head + (size_t)n * kDh + c * 8) =
+                *reinterpret_cast<const uint4*>(o_gen + sw128(row, c));
     }
 }
 
@@ -503,7 +517,7 @@ template <int R>
 static cudaError_t launch_apply_bf16_r(const Shape& s, const void* q, const void* P_q, const __nv_bfloat16* Cbf,
                                        const float* gate, const void* o_s, void* o, const float2* tab, cudaStream_t st)
 {
-    size_t smem = (size_t)R * 512 + kBlock * 256;
+    size_t smem = (size_t)R * 512 + 2 * kBlock * 256;
     cudaError_t e = cudaFuncSetAttribute(apply_bf16_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     apply_bf16_kernel<R><<<dim3(s.nB, s.B * s.H), 128, smem, st>>>(

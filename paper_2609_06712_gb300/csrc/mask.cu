@@ -10,53 +10,63 @@
 namespace rola {
 
 // ---------------------------------------------------------------------------
-// scores[bh][i][j] = (q_bar_i . k_bar_j) / sqrt(128): one 64 x 64 tile per CTA,
-// 256 threads with 4 x 4 register tiles, d staged through shared memory in
-// chunks of 32.
+// scores[bh][i][j] = (q_bar_i . k_bar_j) / sqrt(128): fp32 SIMT GEMM, one 128 x 128
+// tile per CTA, 256 threads with 8 x 8 register tiles (rows ty + 16 u, columns
+// tx + 16 w), d staged through shared memory in chunks of 16, transposed.
 
-constexpr int kSTile = 64, kSChunk = 32;
+constexpr int kSTile = 128, kSChunk = 16;
 
 __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float* __restrict__ qbar,
                                                            const float* __restrict__ kbar,
                                                            float* __restrict__ scores)
 {
-    __shared__ float qs[kSChunk][kSTile + 4];
-    __shared__ float ks[kSChunk][kSTile + 4];
+    __shared__ __align__(16) float qs[kSChunk][kSTile + 4];
+    __shared__ __align__(16) float ks[kSChunk][kSTile + 4];
     const int bh = blockIdx.z, i0 = blockIdx.y * kSTile, j0 = blockIdx.x * kSTile;
     const float* Q = qbar + (size_t)bh * s.nB * kDh;
     const float* K = kbar + (size_t)bh * s.nB * kDh;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float acc[4][4] = {};
+    // loader: 128 rows x 16 d per operand = 512 float4, two per thread
+    const int lrow = threadIdx.x >> 2, lq = threadIdx.x & 3;     // rows lrow, lrow + 64; d 4*lq .. 4*lq+3
+    float acc[8][8] = {};
     for (int d0 = 0; d0 < kDh; d0 += kSChunk) {
-        // 64 rows x 32 d of each operand: 2048 floats, 8 per thread, stored transposed
-        for (int e = threadIdx.x; e < kSTile * kSChunk; e += 256) {
-            int row = e / kSChunk, d = e % kSChunk;
-            int gi = i0 + row, gj = j0 + row;
-            qs[d][row] = gi < s.nB ? Q[(size_t)gi * kDh + d0 + d] : 0.0f;
-            ks[d][row] = gj < s.nB ? K[(size_t)gj * kDh + d0 + d] : 0.0f;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int row = lrow + 64 * h;
+            const int gi = i0 + row, gj = j0 + row;
+            const float4 a = gi < s.nB ? __ldg(reinterpret_cast<const float4*>(Q + (size_t)gi * kDh + d0) + lq)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 b = gj < s.nB ? __ldg(reinterpret_cast<const float4*>(K + (size_t)gj * kDh + d0) + lq)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            qs[4 * lq][row] = a.x; qs[4 * lq + 1][row] = a.y; qs[4 * lq + 2][row] = a.z; qs[4 * lq + 3][row] = a.w;
+            ks[4 * lq][row] = b.x; ks[4 * lq + 1][row] = b.y; ks[4 * lq + 2][row] = b.z; ks[4 * lq + 3][row] = b.w;
         }
         __syncthreads();
-#pragma unroll 8
+#pragma unroll
         for (int d = 0; d < kSChunk; ++d) {
-            float4 a = *reinterpret_cast<const float4*>(&qs[d][ty * 4]);
-            float4 b = *reinterpret_cast<const float4*>(&ks[d][tx * 4]);
-            float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+            const float4 a0 = *reinterpret_cast<const float4*>(&qs[d][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&qs[d][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4*>(&ks[d][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4*>(&ks[d][64 + tx * 4]);
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+            for (int u = 0; u < 8; ++u)
 #pragma unroll
-                for (int w = 0; w < 4; ++w) acc[u][w] = fmaf(av[u], bv[w], acc[u][w]);
+                for (int w = 0; w < 8; ++w) acc[u][w] = fmaf(av[u], bv[w], acc[u][w]);
         }
         __syncthreads();
     }
     const float scale = 0.08838834764831845f;   // 1 / sqrt(128)
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-        int gi = i0 + ty * 4 + u;
+    for (int u = 0; u < 8; ++u) {
+        const int gi = i0 + (u < 4 ? ty * 4 + u : 64 + ty * 4 + u - 4);
         if (gi >= s.nB) continue;
+        float* out = scores + ((size_t)bh * s.nB + gi) * s.nB;
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
-            int gj = j0 + tx * 4 + w;
-            if (gj < s.nB) scores[((size_t)bh * s.nB + gi) * s.nB + gj] = acc[u][w] * scale;
+        for (int w = 0; w < 8; ++w) {
+            const int gj = j0 + (w < 4 ? tx * 4 + w : 64 + tx * 4 + w - 4);
+            if (gj < s.nB) out[gj] = acc[u][w] * scale;
         }
     }
 }

@@ -97,25 +97,51 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
     T* xr = blockIdx.z == 0 ? qr : kr;
     float* xbar = blockIdx.z == 0 ? qbar : kbar;
     const int c8 = threadIdx.x & 15;        // coordinates 8*c8 .. 8*c8+7 (pairs 4*c8 .. 4*c8+3)
-    const int rsub = threadIdx.x >> 4;      // row within a pass
-    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    const int n0 = blk * kBlock;
+    const int rsub = threadIdx.x >> 4;      // row within a pass; rows rsub + 16 * pass
+    const int n0 = blk * kBlock + rsub;
+    constexpr int kPasses = kBlock / 16;
+    // all loads first: four 16- or 32-byte vectors in flight per thread
+    float v[kPasses][8];
 #pragma unroll
-    for (int pass = 0; pass < kBlock / 16; ++pass) {
-        int n = n0 + pass * 16 + rsub;
+    for (int pass = 0; pass < kPasses; ++pass) {
+        const int n = n0 + 16 * pass;
+        if (n < s.N) Vec8<T>::load(x + ((size_t)bh * s.N + n) * kDh + c8 * 8, v[pass]);
+    }
+    // grid position of the first row, then advanced by 16 tokens per pass
+    const int hw = s.Hh * s.Ww;
+    int t = n0 / hw, rem = n0 - t * hw;
+    int xx = rem / s.Ww, yy = rem - xx * s.Ww;
+    // table row base of each of this thread's 4 pairs: the pair's axis is fixed
+    int axis[4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+        const int m = c8 * 4 + p;
+        axis[p] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
+    }
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+    for (int pass = 0; pass < kPasses; ++pass) {
+        const int n = n0 + 16 * pass;
         if (n < s.N) {
-            size_t off = ((size_t)bh * s.N + n) * kDh + c8 * 8;
-            float v[8], o[8];
-            Vec8<T>::load(x + off, v);
+            float o[8];
 #pragma unroll
             for (int p = 0; p < 4; ++p) {
-                float2 cs = rope_cs(tab, s, n, c8 * 4 + p);
-                o[2 * p] = v[2 * p] * cs.x - v[2 * p + 1] * cs.y;
-                o[2 * p + 1] = v[2 * p] * cs.y + v[2 * p + 1] * cs.x;
+                const int row = axis[p] == 0 ? t : (axis[p] == 1 ? s.T + xx : s.T + s.Hh + yy);
+                const float2 cs = __ldg(tab + row * kPairs + c8 * 4 + p);
+                o[2 * p] = v[pass][2 * p] * cs.x - v[pass][2 * p + 1] * cs.y;
+                o[2 * p + 1] = v[pass][2 * p] * cs.y + v[pass][2 * p + 1] * cs.x;
             }
-            Vec8<T>::store(xr + off, o);
+            Vec8<T>::store(xr + ((size_t)bh * s.N + n) * kDh + c8 * 8, o);
 #pragma unroll
             for (int i = 0; i < 8; ++i) acc[i] += o[i];
+        }
+        yy += 16;                           // advance to the token 16 further on
+        while (yy >= s.Ww) {
+            yy -= s.Ww;
+            if (++xx == s.Hh) {
+                xx = 0;
+                ++t;
+            }
         }
     }
 #pragma unroll
@@ -125,7 +151,7 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
         float sum = 0.0f;
 #pragma unroll
         for (int r = 0; r < 16; ++r) sum += part[r][threadIdx.x];
-        int cnt = min(kBlock, s.N - n0);
+        const int cnt = min(kBlock, s.N - blk * kBlock);
         xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = sum / (float)cnt;
     }
 }
