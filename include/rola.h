@@ -87,7 +87,13 @@ typedef struct {
     float eps_fuse;            /* epsilon of the sparse-output RMS r_p, Eq. (gate); default 1e-6 */
     float gate_bias;           /* g = sigmoid(gate_bias) when gate == NULL; default -1.946 */
     rola_dtype_t dtype;        /* ROLA_BF16 (default) or ROLA_FP32 */
+    int32_t wait_limit_ms;     /* bound of every device-side wait (0 = 2000 ms); at most 60000 */
+    int32_t debug_flags;       /* 0 normally.  ROLA_DEBUG_SKIP_FIRST_K_COPY makes each CTA of the
+                                  bf16 sparse kernel skip its first K copy, so a bounded wait runs
+                                  out and the call reports ROLA_ERR_TIMEOUT (tests the timeout path) */
 } rola_config_t;
+
+#define ROLA_DEBUG_SKIP_FIRST_K_COPY 1
 
 /* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
 rola_status_t rola_config_init(rola_config_t* cfg);

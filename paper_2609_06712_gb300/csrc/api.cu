@@ -40,6 +40,8 @@ rola_status_t validate(const rola_config_t* c)
     if (!isfinite(c->gate_bias)) return ROLA_ERR_INVALID_ARG;
     for (int a = 0; a < 3; ++a)
         if (c->pos_offset[a] < -(1 << 20) || c->pos_offset[a] > (1 << 20)) return ROLA_ERR_INVALID_ARG;
+    if (c->wait_limit_ms < 0 || c->wait_limit_ms > 60000) return ROLA_ERR_INVALID_ARG;
+    if (c->debug_flags & ~ROLA_DEBUG_SKIP_FIRST_K_COPY) return ROLA_ERR_INVALID_ARG;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
     if ((int64_t)c->B * c->H * c->N * c->d_h > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
@@ -59,6 +61,8 @@ Shape make_shape(const rola_config_t& c)
     s.eps_fuse = c.eps_fuse;
     s.default_gate = (float)(1.0 / (1.0 + exp(-(double)c.gate_bias)));
     s.sm_scale_log2 = (float)(1.4426950408889634 / sqrt((double)kDh));
+    s.wait_limit_ns = (uint64_t)(c.wait_limit_ms > 0 ? c.wait_limit_ms : 2000) * 1000000ull;
+    s.debug_flags = c.debug_flags;
     return s;
 }
 

@@ -37,6 +37,8 @@ struct Shape {
     float eps_lr, eps_fuse;
     float default_gate;       // sigmoid(gate_bias)
     float sm_scale_log2;      // log2(e) / sqrt(128)
+    uint64_t wait_limit_ns;   // bound of every device-side wait
+    int debug_flags;          // ROLA_DEBUG_* test hooks
 };
 
 // Rotation (cos, sin) of pair m for the token at flat index n.

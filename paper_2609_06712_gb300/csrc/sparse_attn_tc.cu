@@ -75,7 +75,6 @@ constexpr uint32_t kSmemO = kSmemP;                 // output staging reuses P b
 constexpr uint32_t kSmemTiles = kSmemP + 2 * kPBytes;   // 224 KB, 1024-aligned pieces
 static_assert(kOBytes <= kPBytes, "output staging fits a P buffer");
 constexpr uint32_t kTmemCols = 256;                 // S^T x2 (64 cols each), O^T x2
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr float kRescaleThreshold = 8.0f;           // log2 units
 
 enum Bar { Q_FULL = 0, Q_EMPTY = 1, K_FULL = 2, K_EMPTY = K_FULL + KS, V_FULL = K_EMPTY + KS,
@@ -240,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             const int bh = item / nB, qb = item - bh * nB;
             const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
             if (warp == kProducerKWarp) {
-                if (k >= 1) ok = mbar_wait(bar(Q_EMPTY), (k - 1) & 1, abort, kWaitLimitNs);
+                if (k >= 1) ok = mbar_wait(bar(Q_EMPTY), (k - 1) & 1, abort, s.wait_limit_ns);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
                 if (lane == 0) {
@@ -261,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     const int slot = c % VB;
                     bool okl = true;
                     if (lane < 2 && h < nblk && c >= VB)
-                        okl = mbar_wait(bar(V_EMPTY + slot), ((c / VB) - 1) & 1, abort, kWaitLimitNs);
+                        okl = mbar_wait(bar(V_EMPTY + slot), ((c / VB) - 1) & 1, abort, s.wait_limit_ns);
                     ok = __shfl_sync(0xffffffffu, okl, 0) && __shfl_sync(0xffffffffu, okl, 1);
                     if (!ok) break;
                     if (lane < 2 && h < nblk) {
@@ -272,12 +271,14 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     issued_vb += nblk;
                 } else {
                     const int st = g % KS;
-                    if (g >= KS) ok = mbar_wait(bar(K_EMPTY + st), ((g / KS) - 1) & 1, abort, kWaitLimitNs);
+                    if (g >= KS) ok = mbar_wait(bar(K_EMPTY + st), ((g / KS) - 1) & 1, abort, s.wait_limit_ns);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) break;
-                    if (lane == 0) mbar_expect_tx(bar(K_FULL + st), nblk * 16384u);
+                    // test hook: the first K copy of the CTA is never issued, so the waits on it run out
+                    const bool skip = (s.debug_flags & ROLA_DEBUG_SKIP_FIRST_K_COPY) && g == 0;
+                    if (lane == 0 && !skip) mbar_expect_tx(bar(K_FULL + st), nblk * 16384u);
                     __syncwarp();
-                    if (lane < 4 && h < nblk)
+                    if (lane < 4 && h < nblk && !skip)
                         tma_load_3d(sbase + kSmemK + st * kKVBytes + kc * 16384 + h * 8192, &map_k, bar(K_FULL + st),
                                     kc * 64, (h ? jb : ja) * 64, bh);
                     ++issued_k;
@@ -289,15 +290,12 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
         // the latest issued phase of each buffer, bounded by time only
         if (lane == 0) {
             int never = 0;
-            if (issued_q > 0) mbar_wait(bar(Q_FULL), (issued_q - 1) & 1, &never, kWaitLimitNs);
+            if (issued_q > 0) mbar_wait(bar(Q_FULL), (issued_q - 1) & 1, &never, s.wait_limit_ns);
             const int NS = is_v ? VB : KS, issued = is_v ? issued_vb : issued_k;
             const int full0 = is_v ? V_FULL : K_FULL;
-            for (int b = 0; b < NS; ++b) {
-                if (issued > b) {
-                    const int last = issued - 1 - ((issued - 1 - b) % NS);   // latest use of slot b
-                    mbar_wait(bar(full0 + b), (last / NS) & 1, &never, kWaitLimitNs);
-                }
-            }
+            // the last NS uses (tiles of K, blocks of V), one per slot
+            for (int u = issued > NS ? issued - NS : 0; u < issued; ++u)
+                mbar_wait(bar(full0 + u % NS), (u / NS) & 1, &never, s.wait_limit_ns);
         }
     } else if (warp == kMmaWarp || warp == kPvWarp) {
         // ------------------------------------------------------------ MMA issuers
@@ -322,11 +320,11 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
                 const int ob = k & 1;
                 if (!pv) {
-                    if (!(ok = mbar_wait(bar(Q_FULL), k & 1, abort, kWaitLimitNs))) break;
+                    if (!(ok = mbar_wait(bar(Q_FULL), k & 1, abort, s.wait_limit_ns))) break;
                     for (int t = 0; t < T; ++t) {
                         const int g = k * T + t, sb = g & 1, ks = g % KS;
-                        if (!(ok = mbar_wait(bar(K_FULL + ks), (g / KS) & 1, abort, kWaitLimitNs))) break;
-                        if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + sb), ((g >> 1) - 1) & 1, abort, kWaitLimitNs)))
+                        if (!(ok = mbar_wait(bar(K_FULL + ks), (g / KS) & 1, abort, s.wait_limit_ns))) break;
+                        if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns)))
                             break;
                         fence_after_sync();
                         const uint32_t a = k_lo + ks * (kKVBytes >> 4);
@@ -345,12 +343,12 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                         const bool half = 2 * t + 1 >= s.n_keep;
                         const int c0 = k * s.n_keep + 2 * t;             // cumulative index of block a
                         const int va = c0 % VB, vb = (c0 + 1) % VB;
-                        if (!(ok = mbar_wait(bar(P_FULL + pb), (g >> 1) & 1, abort, kWaitLimitNs))) break;
-                        if (!(ok = mbar_wait(bar(V_FULL + va), (c0 / VB) & 1, abort, kWaitLimitNs))) break;
-                        if (!half && !(ok = mbar_wait(bar(V_FULL + vb), ((c0 + 1) / VB) & 1, abort, kWaitLimitNs)))
+                        if (!(ok = mbar_wait(bar(P_FULL + pb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
+                        if (!(ok = mbar_wait(bar(V_FULL + va), (c0 / VB) & 1, abort, s.wait_limit_ns))) break;
+                        if (!half && !(ok = mbar_wait(bar(V_FULL + vb), ((c0 + 1) / VB) & 1, abort, s.wait_limit_ns)))
                             break;
                         if (t == 0 && k >= 2 &&
-                            !(ok = mbar_wait(bar(O_EMPTY + ob), ((k >> 1) - 1) & 1, abort, kWaitLimitNs)))
+                            !(ok = mbar_wait(bar(O_EMPTY + ob), ((k >> 1) - 1) & 1, abort, s.wait_limit_ns)))
                             break;
                         fence_after_sync();
                         const uint32_t a0 = v_lo + va * (kVBlockBytes >> 4), a1 = v_lo + vb * (kVBlockBytes >> 4);
@@ -378,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             int never = 0;
             const uint32_t drain = bar(pv ? DRAIN + 1 : DRAIN);
             mma_commit(drain);
-            mbar_wait(drain, 0, &never, kWaitLimitNs);
+            mbar_wait(drain, 0, &never, s.wait_limit_ns);
         }
     } else {
         // ------------------------------------------------------------ softmax + epilogue
@@ -417,7 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 const int blk = wtid < 64 ? ja : jb;
                 const int key = blk * 64 + (wtid & 63);
                 const bool valid = blk >= 0 && key < s.N;
-                if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, kWaitLimitNs))) break;
+                if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
                 fence_after_sync();
                 const uint32_t saddr = tmem + lane_off + sb * 64 + col0;
                 float x[kCols];
@@ -468,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     }
                     if (t > 0) {
                         // O^T must hold PV(t-1) before it is rescaled
-                        if (!(ok = mbar_wait(bar(PV_DONE + ((g - 1) & 1)), ((g - 1) >> 1) & 1, abort, kWaitLimitNs)))
+                        if (!(ok = mbar_wait(bar(PV_DONE + ((g - 1) & 1)), ((g - 1) >> 1) & 1, abort, s.wait_limit_ns)))
                             break;
                         fence_after_sync();
                         const uint32_t oaddr = tmem + lane_off + 128 + ob * 64 + col0;
@@ -496,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     l[q + 1] += p1;
                     pk[q >> 1] = pack_bf16(p0, p1);
                 }
-                if (g >= 2 && !(ok = mbar_wait(bar(PV_DONE + sb), ((g >> 1) - 1) & 1, abort, kWaitLimitNs))) break;
+                if (g >= 2 && !(ok = mbar_wait(bar(PV_DONE + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns))) break;
                 const uint32_t prow = sbase + kSmemP + sb * kPBytes + (wtid >> 3) * 1024 + (wtid & 7) * 128;
 #pragma unroll
                 for (int c = 0; c < kCols / 8; ++c) {
@@ -512,7 +510,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             }
             if (!ok) break;
             // ---- epilogue: O^s = O^T / l, transposed through shared memory
-            if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, kWaitLimitNs))) break;
+            if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
             column_reduce<false>(l, sm, wg, wtid, sm.inv_l + col0);
             if (wtid < kCols) sm.inv_l[col0 + wtid] = 1.0f / sm.inv_l[col0 + wtid];

@@ -34,7 +34,12 @@ class RolaConfig(ctypes.Structure):
         ("eps_fuse", ctypes.c_float),
         ("gate_bias", ctypes.c_float),
         ("dtype", ctypes.c_int32),
+        ("wait_limit_ms", ctypes.c_int32),
+        ("debug_flags", ctypes.c_int32),
     ]
+
+
+ROLA_DEBUG_SKIP_FIRST_K_COPY = 1
 
 
 class RolaError(RuntimeError):

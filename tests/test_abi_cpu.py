@@ -88,6 +88,9 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
     ("rope_theta", 0.0, 1),
     ("eps_lr", -1.0, 1),
     ("dtype", 7, 1),
+    ("wait_limit_ms", -1, 1),
+    ("wait_limit_ms", 60001, 1),
+    ("debug_flags", 2, 1),
 ])
 def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
     c = cfg_tiny(rl, **{field: value})
