@@ -140,8 +140,9 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
  * Kernel (3): low-rank summary, Eq. (qklr) and Eq. (ctx):
  *   k~_q = R_r(q) SiLU(P_k k^n_q),   C = sum_q k~_q v_q^T,   z = sum_q k~_q.
  * R_r keeps the first r coordinates (r/2 complete pairs) of the native RoPE
- * ordering (Sec. 4.2).  The reduction over N is split across CTAs and
- * combined in a fixed order, so results are bitwise reproducible.
+ * ordering (Sec. 4.2).  The reduction over N is split across CTAs (one
+ * contiguous token range each) and combined in a fixed order, so results are
+ * bitwise reproducible on a given GPU model (the split follows its SM count).
  *   k, v    : [B][H][N][d_h] (k pre-RoPE), dtype;  P_k : [H][r][d_h], dtype
  *   C       : out, fp32 [B][H][r][d_h];   z : out, fp32 [B][H][r], or NULL
  */
@@ -167,6 +168,9 @@ rola_status_t rola_lowrank_apply(const rola_config_t* cfg, const void* q, const 
 /*
  * The whole module (Alg. 1, the per-head steps between the QKV projection
  * and W_o): block mask, sparse branch, low-rank summary, readout and fusion.
+ * In bf16 the rotation, the block pooling and the summary share one pass
+ * over q, k and v; the mask, C and O are those of the separate entry points
+ * (same arithmetic, same bits).
  *   o          : out, [B][H][N][d_h] fused per-head output O^fused, dtype
  *   kv_idx_out : out, the mask used (int32 [B][H][nQB][n_keep]), or NULL
  */
@@ -177,8 +181,10 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
 /*
  * rola_forward with stage timing: identical computation and launches, plus
  * cudaEventRecord(stage_events[i], stream) at five stage boundaries --
- *   [0] start  [1] after the block mask  [2] after the low-rank summary
- *   [3] after the sparse branch  [4] after the readout + fusion.
+ *   [0] start  [1] after the block mask (fp32) or the fused pass over
+ *   q, k, v (bf16: rotation, pooling, summary partials)  [2] after the
+ *   low-rank summary (fp32) or the block scores, top-k and summary combine
+ *   (bf16)  [3] after the sparse branch  [4] after the readout + fusion.
  * stage_events: array of 5 cudaEvent_t created by the caller (owned by the
  * caller), or NULL (then this is rola_forward).
  */

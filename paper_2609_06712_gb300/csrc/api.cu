@@ -95,7 +95,11 @@ Workspace layout(const rola_config_t& c)
     w.C = off; off = align_up(off + 4 * bh * c.r * kDh);
     w.z = off; off = align_up(off + 4 * bh * c.r);
     w.Cbf = off; off = align_up(off + 2 * bh * c.r * kDh);
-    w.partials = off; off = align_up(off + 4 * bh * w.nsplit * ((size_t)c.r * kDh + c.r));
+    // summary partials: fp32 split-N slots, or the bf16 pre-pass's per-(CTA, head) slots
+    const size_t units = bh * s.nB;
+    w.prepass_slots = (units < (size_t)kMaxPrepassCtas ? units : (size_t)kMaxPrepassCtas) + bh - 1;
+    const size_t slots = c.dtype == ROLA_BF16 ? w.prepass_slots : bh * w.nsplit;
+    w.partials = off; off = align_up(off + 4 * slots * ((size_t)c.r * kDh + c.r));
     w.total = off;
     return w;
 }
@@ -127,6 +131,23 @@ rola_status_t prologue(const rola_config_t& c, void* ws, const Workspace& w, cud
 {
     ROLA_TRY(cudaMemsetAsync(at<uint8_t>(ws, w.status), 0, sizeof(DeviceStatus), st));
     ROLA_TRY(launch_rope_table(c, at<float2>(ws, w.table), st));
+    return ROLA_OK;
+}
+
+// The low-rank summary alone: C (fp32), z (nullable) and, when Cbf is given, C in bf16.
+rola_status_t run_summary(const rola_config_t& c, const Shape& s, const Workspace& w, const void* k, const void* v,
+                          const void* P_k, float* C, float* z, __nv_bfloat16* Cbf, void* ws, cudaStream_t st)
+{
+    if (c.dtype == ROLA_BF16) {
+        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        ROLA_TRY(launch_prepass(s, ctas, nullptr, k, v, P_k, at<float2>(ws, w.table), nullptr, nullptr, nullptr,
+                                nullptr, at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
+        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), C, z, Cbf, st));
+    } else {
+        ROLA_TRY(launch_lowrank_summary(c.dtype, s, w.nsplit, k, v, P_k, at<float2>(ws, w.table),
+                                        at<float>(ws, w.partials), C, z, Cbf, st));
+    }
     return ROLA_OK;
 }
 
@@ -226,9 +247,7 @@ rola_status_t rola_lowrank_summary(const rola_config_t* cfg, const void* k, cons
     Workspace w = layout(*cfg);
     Shape s = make_shape(*cfg);
     ROLA_CHECK(prologue(*cfg, ws, w, st));
-    ROLA_TRY(launch_lowrank_summary(cfg->dtype, s, w.nsplit, k, v, P_k, at<float2>(ws, w.table),
-                                    at<float>(ws, w.partials), C, z, nullptr, st));
-    return ROLA_OK;
+    return run_summary(*cfg, s, w, k, v, P_k, C, z, nullptr, ws, st);
 }
 
 rola_status_t rola_lowrank_apply(const rola_config_t* cfg, const void* q, const void* P_q, const float* C,
@@ -269,11 +288,26 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
     int32_t* kv = kv_idx_out ? kv_idx_out : at<int32_t>(ws, w.kv_idx);
     ROLA_TRY(mark(0));
     ROLA_CHECK(prologue(*cfg, ws, w, st));
-    ROLA_CHECK(run_mask(*cfg, s, w, q, k, kv, ws, st));
-    ROLA_TRY(mark(1));
-    ROLA_TRY(launch_lowrank_summary(cfg->dtype, s, w.nsplit, k, v, P_k, at<float2>(ws, w.table),
-                                    at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
-                                    at<__nv_bfloat16>(ws, w.Cbf), st));
+    if (cfg->dtype == ROLA_BF16) {
+        // stage 1: one pass over q, k, v -> q^r, k^r, block means, summary partials;
+        // stage 2: block scores + top-k, and the summary combine
+        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        ROLA_TRY(launch_prepass(s, ctas, q, k, v, P_k, at<float2>(ws, w.table), at<void>(ws, w.qr),
+                                at<void>(ws, w.kr), at<float>(ws, w.qbar), at<float>(ws, w.kbar),
+                                at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
+        ROLA_TRY(mark(1));
+        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
+                                   st));
+        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
+                                        at<__nv_bfloat16>(ws, w.Cbf), st));
+    } else {
+        // stage 1: the block mask; stage 2: the summary
+        ROLA_CHECK(run_mask(*cfg, s, w, q, k, kv, ws, st));
+        ROLA_TRY(mark(1));
+        ROLA_CHECK(run_summary(*cfg, s, w, k, v, P_k, at<float>(ws, w.C), at<float>(ws, w.z),
+                               at<__nv_bfloat16>(ws, w.Cbf), ws, st));
+    }
     ROLA_TRY(mark(2));
     ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv, o,
                                 at<DeviceStatus>(ws, w.status), st));

@@ -52,12 +52,21 @@ __device__ __forceinline__ float2 rope_cs(const float2* __restrict__ tab, const 
     return tab[row * kPairs + m];
 }
 
+// One RoPE pair rotation (x0, x1) -> (x0 cos - x1 sin, x0 sin + x1 cos) with
+// its roundings spelled out, so that every kernel that rotates gets the same
+// bits for the same inputs.
+__device__ __forceinline__ float2 rope_rotate(float x0, float x1, float2 cs)
+{
+    return make_float2(__fmaf_rn(x0, cs.x, -__fmul_rn(x1, cs.y)), __fmaf_rn(x0, cs.y, __fmul_rn(x1, cs.x)));
+}
+
 // ---------------------------------------------------------------- host side
 
 // Workspace carve-up for one configuration.
 struct Workspace {
     size_t status, table, qr, kr, qbar, kbar, scores, kv_idx, C, z, Cbf, partials, total;
-    int nsplit;
+    int nsplit;               // fp32 summary splits
+    size_t prepass_slots;     // bf16 pre-pass partial slots
 };
 
 // Host launchers, one per kernel family.  All return cudaGetLastError().
@@ -80,8 +89,22 @@ cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q,
                                  const float* C, const __nv_bfloat16* Cbf, const float* gate,
                                  const void* o_s, void* o, const float2* tab, cudaStream_t st);
 
-// Number of N-splits of the summary reduction for this shape.
+// Number of N-splits of the summary reduction for this shape (fp32 kernel).
 int summary_splits(const Shape& s);
+
+// The bf16 pre-pass (prepass.cu): `ctas` persistent CTAs each walk a
+// contiguous range of (head, 64-token block) units.  Given q (fused form) it
+// writes q^r, k^r and the pooled means exactly as launch_rope_pool does; it
+// always writes the summary partials, one slot per (CTA c, head bh) at index
+// c + bh, which launch_prepass_combine adds in CTA order.  With `ctas` CTAs
+// the partial buffer needs ctas + B*H - 1 slots of r*128 + r floats.
+constexpr int kMaxPrepassCtas = 256;
+int prepass_ctas(const Shape& s, int max_ctas);     // one per SM of the current device, at most max_ctas
+cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* k, const void* v,
+                           const void* P_k, const float2* tab, void* qr, void* kr, float* qbar, float* kbar,
+                           float* partials, DeviceStatus* status, cudaStream_t st);
+cudaError_t launch_prepass_combine(const Shape& s, int ctas, const float* partials, float* C, float* z,
+                                   __nv_bfloat16* Cbf, cudaStream_t st);
 
 // Host-side configuration checks shared by the entry points (api.cu).
 rola_status_t validate(const rola_config_t* cfg);   // ROLA_OK if the kernels handle cfg
@@ -110,6 +133,10 @@ __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a, uint32_t& b,
 {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
                  : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& a, uint32_t& b)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];\n" : "=r"(a), "=r"(b) : "r"(addr));
 }
 __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c, uint32_t& d)
 {
@@ -150,5 +177,14 @@ __device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x));
 // Byte offset of 16-byte chunk c of row r in a [rows][128 bf16] tile with the
 // chunk index XOR-swizzled by the row (conflict-free ldmatrix on 8-row groups).
 __device__ __forceinline__ uint32_t sw128(int r, int c) { return r * 256 + ((c ^ (r & 7)) << 4); }
+
+// Byte offset of 16-byte chunk c (0..15) of row r in a 64-row block tile as a
+// [chunk][row][64] TMA box with 128-byte swizzle writes it: the two 64-wide
+// halves of a row are 8 KB apart, and within 1024-byte atoms chunk c & 7 of
+// row r sits at (c & 7) ^ (r & 7).
+__device__ __forceinline__ uint32_t tsw(int r, int c)
+{
+    return (c >> 3) * 8192 + r * 128 + (((c & 7) ^ (r & 7)) << 4);
+}
 
 }  // namespace rola

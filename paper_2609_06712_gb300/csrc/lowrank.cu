@@ -1,4 +1,5 @@
-// Low-rank branch: summary (kernel 3) and readout + gated fusion (kernel 4).
+// Low-rank branch: the fp32 summary of the validation mode (the bf16 summary
+// is part of the pre-pass, prepass.cu) and readout + gated fusion (kernel 4).
 //
 // Eq. (qklr):  k~_q = R_r(q) SiLU(P_k k^n_q),   q~_p = R_r(p) SiLU(P_q q^n_p)
 // Eq. (ctx):   C = sum_q k~_q v_q^T,            O^lr_p = RMSNorm(q~_p^T C)   (no gain)
@@ -6,24 +7,17 @@
 //
 // R_r keeps the first r/2 rotary pairs of the native ordering (Sec. 4.2).  The
 // fusion is evaluated as O^s_p + g_p r_p O^lr_p, which is the same expression
-// with one rounding fewer.  The summary reduction over N is split across CTAs;
-// each writes an fp32 partial to the workspace and a second kernel adds the
-// partials in split order, so C is bitwise reproducible run to run.
+// with one rounding fewer.  The fp32 summary reduction over N is split across
+// CTAs; each writes an fp32 partial to the workspace and a second kernel adds
+// the partials in split order, so C is bitwise reproducible run to run.
 #include "common.cuh"
 
 namespace rola {
 
 // ===========================================================================
-// summary, bf16: CTA = (split, head), 256 threads = 8 warps, 128-token tiles
-// double-buffered through cp.async.  Per tile:
-//   U  = K_tile P_k^T      (warp w: tokens 16w..16w+15, all r columns)
-//   k~ = R_r SiLU(U)       (fp32 in registers, bf16 into shared memory)
-//   C^T[d][r] += V^T k~    (warp w: d columns 16w..16w+15, all r rows)
-// Shared memory: P_k r x 256 B | K 2 x 32 KB | V 2 x 32 KB | k~ 128 x (2r + 16) B.
+// Split-N partitioning of the fp32 summary: CTA = (split, head).
 
-constexpr int kSumThreads = 256;
 constexpr int kSumTile = 128;
-constexpr int kSumTileBytes = kSumTile * kDh * 2;
 
 int summary_splits(const Shape& s)
 {
@@ -43,142 +37,6 @@ __device__ __forceinline__ void load_rows_async(uint32_t sbase, const __nv_bfloa
         int n = row0 + r;
         const __nv_bfloat16* src = g + (size_t)min(n, limit - 1) * kDh + c * 8;
         cp_async16(sbase + sw128(r, c), src, n < limit ? 16 : 0);
-    }
-}
-
-template <int R>
-__global__ void __launch_bounds__(kSumThreads) summary_bf16_kernel(Shape s, int tokens_per_split,
-                                                                   const __nv_bfloat16* __restrict__ k,
-                                                                   const __nv_bfloat16* __restrict__ v,
-                                                                   const __nv_bfloat16* __restrict__ Pk,
-                                                                   const float2* __restrict__ tab,
-                                                                   float* __restrict__ partials)
-{
-    extern __shared__ __align__(128) uint8_t smem[];
-    constexpr int NT = R / 8;                 // n-tiles of the projection
-    constexpr int KT_STRIDE = 2 * R + 16;     // bytes per k~ row (padded)
-    __shared__ float zsm[8][R];
-    const int split = blockIdx.x, bh = blockIdx.y, h = bh % s.H;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
-    const uint32_t sP = smem_u32(smem);
-    const uint32_t sK = sP + R * 256;
-    const uint32_t sV = sK + 2 * kSumTileBytes;
-    const uint32_t sKt = sV + 2 * kSumTileBytes;
-    uint8_t* kt_gen = smem + R * 256 + 4 * kSumTileBytes;
-    const size_t head = (size_t)bh * s.N * kDh;
-    const int n_begin = split * tokens_per_split;
-    const int n_end = min(s.N, n_begin + tokens_per_split);
-    const int ntiles = (n_end - n_begin + kSumTile - 1) / kSumTile;
-
-    load_rows_async(sP, Pk + (size_t)h * R * kDh, 0, R, R, tid, kSumThreads);
-    load_rows_async(sK, k + head, n_begin, kSumTile, s.N, tid, kSumThreads);
-    load_rows_async(sV, v + head, n_begin, kSumTile, s.N, tid, kSumThreads);
-    cp_async_commit();
-
-    float cacc[R / 16][2][4];
-#pragma unroll
-    for (int a = 0; a < R / 16; ++a)
-#pragma unroll
-        for (int b = 0; b < 2; ++b) cacc[a][b][0] = cacc[a][b][1] = cacc[a][b][2] = cacc[a][b][3] = 0.0f;
-    float zacc[NT][2];
-#pragma unroll
-    for (int a = 0; a < NT; ++a) zacc[a][0] = zacc[a][1] = 0.0f;
-
-    for (int it = 0; it < ntiles; ++it) {
-        const int stage = it & 1;
-        const int n0 = n_begin + it * kSumTile;
-        if (it + 1 < ntiles) {
-            load_rows_async(sK + (stage ^ 1) * kSumTileBytes, k + head, n0 + kSumTile, kSumTile, s.N, tid,
-                            kSumThreads);
-            load_rows_async(sV + (stage ^ 1) * kSumTileBytes, v + head, n0 + kSumTile, kSumTile, s.N, tid,
-                            kSumThreads);
-        }
-        cp_async_commit();
-        cp_async_wait<1>();
-        __syncthreads();
-        const uint32_t kb = sK + stage * kSumTileBytes, vb = sV + stage * kSumTileBytes;
-        // U = K_tile P_k^T for this warp's 16 tokens
-        float u[NT][4];
-#pragma unroll
-        for (int a = 0; a < NT; ++a) u[a][0] = u[a][1] = u[a][2] = u[a][3] = 0.0f;
-#pragma unroll
-        for (int kc = 0; kc < 8; ++kc) {
-            const int mi = lane >> 3;
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4(kb + sw128(warp * 16 + (lane & 7) + (mi & 1) * 8, kc * 2 + (mi >> 1)), a0, a1, a2, a3);
-#pragma unroll
-            for (int np = 0; np < NT / 2; ++np) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(sP + sw128(np * 16 + (mi >> 1) * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1, b2, b3);
-                mma_bf16(u[2 * np], a0, a1, a2, a3, b0, b1);
-                mma_bf16(u[2 * np + 1], a0, a1, a2, a3, b2, b3);
-            }
-        }
-        // k~ = R_r SiLU(U); rows past the split end (or N) contribute nothing
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            const int tl = warp * 16 + g + hr * 8;
-            const int n = n0 + tl;
-            const bool ok = n < n_end;
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const int m = nt * 4 + t4;
-                float x0 = silu(u[nt][2 * hr]), x1 = silu(u[nt][2 * hr + 1]);
-                float2 cs = ok ? rope_cs(tab, s, n, m) : make_float2(0.0f, 0.0f);
-                float y0 = x0 * cs.x - x1 * cs.y;
-                float y1 = x0 * cs.y + x1 * cs.x;
-                zacc[nt][0] += y0;
-                zacc[nt][1] += y1;
-                *reinterpret_cast<uint32_t*>(kt_gen + tl * KT_STRIDE + (nt * 8 + t4 * 2) * 2) = pack_bf16(y0, y1);
-            }
-        }
-        __syncthreads();
-        // C^T += V^T k~ : warp w owns d columns 16w .. 16w+15
-#pragma unroll
-        for (int kc = 0; kc < kSumTile / 16; ++kc) {
-            const int mi = lane >> 3;
-            uint32_t b0, b1, b2, b3;
-            ldsm_x4_t(vb + sw128(kc * 16 + (mi & 1) * 8 + (lane & 7), warp * 2 + (mi >> 1)), b0, b1, b2, b3);
-#pragma unroll
-            for (int mt = 0; mt < R / 16; ++mt) {
-                uint32_t a0, a1, a2, a3;
-                ldsm_x4_t(sKt + (kc * 16 + (mi >> 1) * 8 + (lane & 7)) * KT_STRIDE + (mt * 2 + (mi & 1)) * 16, a0,
-                          a1, a2, a3);
-                mma_bf16(cacc[mt][0], a0, a1, a2, a3, b0, b1);
-                mma_bf16(cacc[mt][1], a0, a1, a2, a3, b2, b3);
-            }
-        }
-        __syncthreads();
-    }
-    cp_async_wait<0>();
-    // partial C [r][d] and z [r] of this split
-    float* part = partials + ((size_t)bh * gridDim.x + split) * (size_t)(R * kDh + R);
-#pragma unroll
-    for (int mt = 0; mt < R / 16; ++mt)
-#pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-            int d = warp * 16 + nt * 8 + t4 * 2;
-            int a = mt * 16 + g;
-            *reinterpret_cast<float2*>(part + (size_t)a * kDh + d) = make_float2(cacc[mt][nt][0], cacc[mt][nt][1]);
-            *reinterpret_cast<float2*>(part + (size_t)(a + 8) * kDh + d) =
-                make_float2(cacc[mt][nt][2], cacc[mt][nt][3]);
-        }
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            float x = zacc[nt][e];
-            x += __shfl_xor_sync(0xffffffffu, x, 4);
-            x += __shfl_xor_sync(0xffffffffu, x, 8);
-            x += __shfl_xor_sync(0xffffffffu, x, 16);
-            if (g == 0) zsm[warp][nt * 8 + t4 * 2 + e] = x;
-        }
-    __syncthreads();
-    if (tid < R) {
-        float x = 0.0f;
-#pragma unroll
-        for (int w = 0; w < 8; ++w) x += zsm[w][tid];
-        part[(size_t)R * kDh + tid] = x;
     }
 }
 
@@ -280,47 +138,20 @@ cudaError_t launch_c_to_bf16(const Shape& s, const float* C, __nv_bfloat16* Cbf,
     return cudaGetLastError();
 }
 
-template <int R>
-static cudaError_t launch_summary_bf16_r(const Shape& s, int nsplit, int tps, const void* k, const void* v,
-                                         const void* Pk, const float2* tab, float* partials, cudaStream_t st)
-{
-    size_t smem = (size_t)R * 256 + 4 * (size_t)kSumTileBytes + (size_t)kSumTile * (2 * R + 16);
-    cudaError_t e =
-        cudaFuncSetAttribute(summary_bf16_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    summary_bf16_kernel<R><<<dim3(nsplit, s.B * s.H), kSumThreads, smem, st>>>(
-        s, tps, (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, (const __nv_bfloat16*)Pk, tab, partials);
-    return cudaGetLastError();
-}
-
 cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, const void* k, const void* v,
                                    const void* P_k, const float2* tab, float* partials, float* C, float* z,
                                    __nv_bfloat16* Cbf, cudaStream_t st)
 {
+    if (dt != ROLA_FP32) return cudaErrorInvalidValue;      // bf16: launch_prepass
     int tiles = (s.N + kSumTile - 1) / kSumTile;
     int tps = ((tiles + nsplit - 1) / nsplit) * kSumTile;
-    cudaError_t e = cudaSuccess;
-    if (dt == ROLA_BF16) {
-        switch (s.r) {
-            case 16: e = launch_summary_bf16_r<16>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 32: e = launch_summary_bf16_r<32>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 48: e = launch_summary_bf16_r<48>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 64: e = launch_summary_bf16_r<64>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 80: e = launch_summary_bf16_r<80>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 96: e = launch_summary_bf16_r<96>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 112: e = launch_summary_bf16_r<112>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            case 128: e = launch_summary_bf16_r<128>(s, nsplit, tps, k, v, P_k, tab, partials, st); break;
-            default: return cudaErrorInvalidValue;
-        }
-    } else {
-        size_t smem = sizeof(float) * ((size_t)s.r * (kDh + 1) + kF32Tile * (kDh + 1) + kF32Tile * kDh +
-                                       kF32Tile * (s.r + 1));
-        e = cudaFuncSetAttribute(summary_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        summary_f32_kernel<<<dim3(nsplit, s.B * s.H), 256, smem, st>>>(s, tps, (const float*)k, (const float*)v,
-                                                                        (const float*)P_k, tab, partials);
-        e = cudaGetLastError();
-    }
+    size_t smem = sizeof(float) * ((size_t)s.r * (kDh + 1) + kF32Tile * (kDh + 1) + kF32Tile * kDh +
+                                   kF32Tile * (s.r + 1));
+    cudaError_t e = cudaFuncSetAttribute(summary_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    summary_f32_kernel<<<dim3(nsplit, s.B * s.H), 256, smem, st>>>(s, tps, (const float*)k, (const float*)v,
+                                                                    (const float*)P_k, tab, partials);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     int per = s.r * kDh + s.r;
     summary_combine_kernel<<<dim3((per + 255) / 256, s.B * s.H), 256, 0, st>>>(s, nsplit, partials, C, z, Cbf);
@@ -336,7 +167,7 @@ cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, 
 // 16-byte accesses.
 
 template <int R>
-__global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
+__global__ void __launch_bounds__(128, 4) apply_bf16_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
                                                          const __nv_bfloat16* __restrict__ Pq,
                                                          const __nv_bfloat16* __restrict__ Cbf,
                                                          const float* __restrict__ gate,
@@ -401,16 +232,15 @@ __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfl
             mma_bf16(y[2 * dp + 1], qf[2 * kc][0], qf[2 * kc][1], qf[2 * kc + 1][0], qf[2 * kc + 1][1], b2, b3);
         }
     }
-    // per-row RMS of y and of O^s (the 4 lanes of a quad share a row)
+    // per-row RMS of y and of O^s (the 4 lanes of a quad share a row); O^s stays
+    // in shared memory and is read again for the fusion
     const int r_lo = warp * 16 + g, r_hi = r_lo + 8;                 // rows within the tile
-    float os[16][4];
     float ssy[2] = {0.0f, 0.0f}, sso[2] = {0.0f, 0.0f};
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) {
         const uint32_t lo_off = sw128(r_lo, dt) + t4 * 4, hi_off = sw128(r_hi, dt) + t4 * 4;
         float2 lo = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + lo_off));
         float2 hi = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + hi_off));
-        os[dt][0] = lo.x; os[dt][1] = lo.y; os[dt][2] = hi.x; os[dt][3] = hi.y;
         ssy[0] += y[dt][0] * y[dt][0] + y[dt][1] * y[dt][1];
         ssy[1] += y[dt][2] * y[dt][2] + y[dt][3] * y[dt][3];
         sso[0] += lo.x * lo.x + lo.y * lo.y;
@@ -431,10 +261,11 @@ __global__ void __launch_bounds__(128) apply_bf16_kernel(Shape s, const __nv_bfl
     // fused rows back into the shared tile (each thread rewrites what it read), then 16-byte stores
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) {
-        *reinterpret_cast<uint32_t*>(o_gen + sw128(r_lo, dt) + t4 * 4) =
-            pack_bf16(os[dt][0] + coef[0] * y[dt][0], os[dt][1] + coef[0] * y[dt][1]);
-        *reinterpret_cast<uint32_t*>(o_gen + sw128(r_hi, dt) + t4 * 4) =
-            pack_bf16(os[dt][2] + coef[1] * y[dt][2], os[dt][3] + coef[1] * y[dt][3]);
+        uint32_t* lo_p = reinterpret_cast<uint32_t*>(o_gen + sw128(r_lo, dt) + t4 * 4);
+        uint32_t* hi_p = reinterpret_cast<uint32_t*>(o_gen + sw128(r_hi, dt) + t4 * 4);
+        const float2 lo = unpack_bf16(*lo_p), hi = unpack_bf16(*hi_p);
+        *lo_p = pack_bf16(lo.x + coef[0] * y[dt][0], lo.y + coef[0] * y[dt][1]);
+        *hi_p = pack_bf16(hi.x + coef[1] * y[dt][2], hi.y + coef[1] * y[dt][3]);
     }
     __syncthreads();
 #pragma unroll

@@ -12,7 +12,10 @@ namespace rola {
 // ---------------------------------------------------------------------------
 // scores[bh][i][j] = (q_bar_i . k_bar_j) / sqrt(128): fp32 SIMT GEMM, one 128 x 128
 // tile per CTA, 256 threads with 8 x 8 register tiles (rows ty + 16 u, columns
-// tx + 16 w), d staged through shared memory in chunks of 16, transposed.
+// tx + 16 w), d staged through shared memory in chunks of 16, transposed and
+// double-buffered: the next chunk's global loads are in flight while the
+// current chunk is multiplied.  Every score is the same ascending-d FMA chain
+// whatever the tiling.
 
 constexpr int kSTile = 128, kSChunk = 16;
 
@@ -20,34 +23,50 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
                                                            const float* __restrict__ kbar,
                                                            float* __restrict__ scores)
 {
-    __shared__ __align__(16) float qs[kSChunk][kSTile + 4];
-    __shared__ __align__(16) float ks[kSChunk][kSTile + 4];
+    __shared__ __align__(16) float qs[2][kSChunk][kSTile + 4];
+    __shared__ __align__(16) float ks[2][kSChunk][kSTile + 4];
     const int bh = blockIdx.z, i0 = blockIdx.y * kSTile, j0 = blockIdx.x * kSTile;
     const float* Q = qbar + (size_t)bh * s.nB * kDh;
     const float* K = kbar + (size_t)bh * s.nB * kDh;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     // loader: 128 rows x 16 d per operand = 512 float4, two per thread
     const int lrow = threadIdx.x >> 2, lq = threadIdx.x & 3;     // rows lrow, lrow + 64; d 4*lq .. 4*lq+3
-    float acc[8][8] = {};
-    for (int d0 = 0; d0 < kDh; d0 += kSChunk) {
+    float4 ra[2], rb[2];
+    auto fetch = [&](int d0) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             const int row = lrow + 64 * h;
             const int gi = i0 + row, gj = j0 + row;
-            const float4 a = gi < s.nB ? __ldg(reinterpret_cast<const float4*>(Q + (size_t)gi * kDh + d0) + lq)
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float4 b = gj < s.nB ? __ldg(reinterpret_cast<const float4*>(K + (size_t)gj * kDh + d0) + lq)
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-            qs[4 * lq][row] = a.x; qs[4 * lq + 1][row] = a.y; qs[4 * lq + 2][row] = a.z; qs[4 * lq + 3][row] = a.w;
-            ks[4 * lq][row] = b.x; ks[4 * lq + 1][row] = b.y; ks[4 * lq + 2][row] = b.z; ks[4 * lq + 3][row] = b.w;
+            ra[h] = gi < s.nB ? __ldg(reinterpret_cast<const float4*>(Q + (size_t)gi * kDh + d0) + lq)
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+            rb[h] = gj < s.nB ? __ldg(reinterpret_cast<const float4*>(K + (size_t)gj * kDh + d0) + lq)
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        __syncthreads();
+    };
+    auto stash = [&](int buf) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int row = lrow + 64 * h;
+            qs[buf][4 * lq][row] = ra[h].x; qs[buf][4 * lq + 1][row] = ra[h].y;
+            qs[buf][4 * lq + 2][row] = ra[h].z; qs[buf][4 * lq + 3][row] = ra[h].w;
+            ks[buf][4 * lq][row] = rb[h].x; ks[buf][4 * lq + 1][row] = rb[h].y;
+            ks[buf][4 * lq + 2][row] = rb[h].z; ks[buf][4 * lq + 3][row] = rb[h].w;
+        }
+    };
+    float acc[8][8] = {};
+    fetch(0);
+    stash(0);
+    __syncthreads();
+#pragma unroll 1
+    for (int c = 0; c < kDh / kSChunk; ++c) {
+        const int buf = c & 1;
+        if (c + 1 < kDh / kSChunk) fetch((c + 1) * kSChunk);
 #pragma unroll
         for (int d = 0; d < kSChunk; ++d) {
-            const float4 a0 = *reinterpret_cast<const float4*>(&qs[d][ty * 4]);
-            const float4 a1 = *reinterpret_cast<const float4*>(&qs[d][64 + ty * 4]);
-            const float4 b0 = *reinterpret_cast<const float4*>(&ks[d][tx * 4]);
-            const float4 b1 = *reinterpret_cast<const float4*>(&ks[d][64 + tx * 4]);
+            const float4 a0 = *reinterpret_cast<const float4*>(&qs[buf][d][ty * 4]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&qs[buf][d][64 + ty * 4]);
+            const float4 b0 = *reinterpret_cast<const float4*>(&ks[buf][d][tx * 4]);
+            const float4 b1 = *reinterpret_cast<const float4*>(&ks[buf][d][64 + tx * 4]);
             const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
             const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
@@ -55,6 +74,8 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
 #pragma unroll
                 for (int w = 0; w < 8; ++w) acc[u][w] = fmaf(av[u], bv[w], acc[u][w]);
         }
+        // the other buffer was last read in chunk c - 1, before the previous barrier
+        if (c + 1 < kDh / kSChunk) stash(buf ^ 1);
         __syncthreads();
     }
     const float scale = 0.08838834764831845f;   // 1 / sqrt(128)

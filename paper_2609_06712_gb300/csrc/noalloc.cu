@@ -4,8 +4,8 @@
 // host framework owns the allocator and passes the op only its input and
 // output tensors, or a runtime that forbids device allocation once it has
 // started (fixed memory budget, no cudaMalloc on the serving path).  For
-// them this entry point keeps its scratch -- the RoPE table and the split-N
-// partial sums of the summary -- in one file-scope __device__ array of
+// them this entry point keeps its scratch -- a status word, the RoPE table and
+// the partial sums of the summary -- in one file-scope __device__ array of
 // kStaticScratchBytes, which every GPU that loads the library holds until
 // the process exits.  It allocates nothing itself.
 //
@@ -15,8 +15,10 @@
 // cached.  Make that first call before any stream capture.
 //
 // Every call shares the one array and it keeps the last call's contents.
-// Everything a call reads from it, the call has written first (the table and
-// every partial are overwritten in full), so nothing needs clearing.  Calls
+// Everything a call reads from it, the call has written first (the status
+// word is cleared, the table and every partial are overwritten in full).  A
+// device-side wait that gives up (bf16 kernel, bounded waits) is recorded in
+// that status word only; no call reports it.  Calls
 // whose executions overlap on the GPU -- on different streams, or from
 // different host threads -- race on the array and must be serialised by the
 // caller.
@@ -69,20 +71,37 @@ extern "C" rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, c
     if (!k || !v || !P_k || !C || !a16(k) || !a16(v) || !a16(P_k) || !a16(C) || (z && !a16(z)))
         return ROLA_ERR_INVALID_ARG;
     const Shape s = make_shape(*cfg);
-    // scratch = RoPE table | partials [B*H][nsplit][r*128 + r]; fewer splits if needed to fit
+    // scratch = status word | RoPE table | summary partials (slots of r*128 + r floats);
+    // fewer CTAs (bf16) or splits (fp32) if needed to fit, but at least one slot per head
+    const size_t head = align256(sizeof(DeviceStatus));
     const size_t table = align256(sizeof(float2) * (size_t)(cfg->T + cfg->Hh + cfg->Ww) * kPairs);
-    const size_t per_split = sizeof(float) * (size_t)s.B * s.H * ((size_t)s.r * kDh + s.r);
-    if (table + per_split > kStaticScratchBytes) return ROLA_ERR_UNSUPPORTED;   // layer too large for the array
-    int nsplit = summary_splits(s);
-    const int fit = (int)((kStaticScratchBytes - table) / per_split);
-    if (nsplit > fit) nsplit = fit;
+    const size_t slot = sizeof(float) * ((size_t)s.r * kDh + s.r);
+    const size_t bh = (size_t)s.B * s.H;
+    if (head + table + bh * slot > kStaticScratchBytes) return ROLA_ERR_UNSUPPORTED;   // layer too large
+    const size_t fit = (kStaticScratchBytes - head - table) / slot;                   // slots available
     void* base = nullptr;
     if (scratch_address(&base) != cudaSuccess) return ROLA_ERR_CUDA;
-    float2* tab = reinterpret_cast<float2*>(base);
-    float* partials = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + table);
+    unsigned char* b = static_cast<unsigned char*>(base);
+    DeviceStatus* status = reinterpret_cast<DeviceStatus*>(b);
+    float2* tab = reinterpret_cast<float2*>(b + head);
+    float* partials = reinterpret_cast<float*>(b + head + table);
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(status, 0, sizeof(DeviceStatus), cs) != cudaSuccess) return ROLA_ERR_CUDA;
     if (launch_rope_table(*cfg, tab, cs) != cudaSuccess) return ROLA_ERR_CUDA;
-    if (launch_lowrank_summary(cfg->dtype, s, nsplit, k, v, P_k, tab, partials, C, z, nullptr, cs) != cudaSuccess)
-        return ROLA_ERR_CUDA;
+    if (cfg->dtype == ROLA_BF16) {
+        const size_t cap = fit - bh + 1;                                    // CTAs whose slots fit
+        const int ctas = prepass_ctas(s, cap < (size_t)kMaxPrepassCtas ? (int)cap : kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        if (launch_prepass(s, ctas, nullptr, k, v, P_k, tab, nullptr, nullptr, nullptr, nullptr, partials, status,
+                           cs) != cudaSuccess ||
+            launch_prepass_combine(s, ctas, partials, C, z, nullptr, cs) != cudaSuccess)
+            return ROLA_ERR_CUDA;
+    } else {
+        int nsplit = summary_splits(s);
+        if ((size_t)nsplit > fit / bh) nsplit = (int)(fit / bh);
+        if (launch_lowrank_summary(cfg->dtype, s, nsplit, k, v, P_k, tab, partials, C, z, nullptr, cs) !=
+            cudaSuccess)
+            return ROLA_ERR_CUDA;
+    }
     return ROLA_OK;
 }

@@ -128,8 +128,9 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
             for (int p = 0; p < 4; ++p) {
                 const int row = axis[p] == 0 ? t : (axis[p] == 1 ? s.T + xx : s.T + s.Hh + yy);
                 const float2 cs = __ldg(tab + row * kPairs + c8 * 4 + p);
-                o[2 * p] = v[pass][2 * p] * cs.x - v[pass][2 * p + 1] * cs.y;
-                o[2 * p + 1] = v[pass][2 * p] * cs.y + v[pass][2 * p + 1] * cs.x;
+                const float2 y = rope_rotate(v[pass][2 * p], v[pass][2 * p + 1], cs);
+                o[2 * p] = y.x;
+                o[2 * p + 1] = y.y;
             }
             Vec8<T>::store(xr + ((size_t)bh * s.N + n) * kDh + c8 * 8, o);
 #pragma unroll

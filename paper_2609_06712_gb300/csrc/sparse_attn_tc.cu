@@ -45,6 +45,7 @@
 
 #include "common.cuh"
 #include "tcgen05.cuh"
+#include "tensor_map.cuh"
 
 namespace rola {
 namespace {
@@ -548,7 +549,9 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
     if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+}  // namespace
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
@@ -564,7 +567,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 
 // [BH][N][128] bf16 viewed as a 3-D tensor (d, token, head); 64 x 64 boxes
 // (one d-chunk of a key block), 128-byte swizzle; rows past N read as zero.
-bool make_map3(CUtensorMap* m, const void* ptr, const Shape& s)
+bool make_chunk_map(CUtensorMap* m, const void* ptr, const Shape& s)
 {
     auto enc = encode_fn();
     if (!enc) return false;
@@ -580,7 +583,7 @@ bool make_map3(CUtensorMap* m, const void* ptr, const Shape& s)
 // The same tensor viewed as 4-D (d within chunk, token, d-chunk, head) so that
 // one 64 x 64 x 2 box brings a whole key block in as [chunk][row][64]: 16 KB,
 // 128-byte swizzle, rows past N read as zero.
-bool make_map4(CUtensorMap* m, const void* ptr, const Shape& s)
+bool make_block_map(CUtensorMap* m, const void* ptr, const Shape& s)
 {
     auto enc = encode_fn();
     if (!enc) return false;
@@ -593,13 +596,11 @@ bool make_map4(CUtensorMap* m, const void* ptr, const Shape& s)
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-}  // namespace
-
 cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
                                   const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st)
 {
     CUtensorMap mq, mk, mv;
-    if (!make_map4(&mq, qr, s) || !make_map3(&mk, kr, s) || !make_map4(&mv, v, s)) return cudaErrorInvalidValue;
+    if (!make_block_map(&mq, qr, s) || !make_chunk_map(&mk, kr, s) || !make_block_map(&mv, v, s)) return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;

@@ -177,6 +177,29 @@ def test_forward_small(rl, case, dname, tdt):
     compare_forward(cfg, x, h, out, kv, dname)
 
 
+@pytest.mark.parametrize("case", ["tiny", "ragged_585_r64", "rmsnorm_gain_b2"])
+def test_fused_prepass_matches_separate_entry_points(rl, case):
+    """In bf16 the forward pass rotates, pools and summarises in one pass over
+    q, k, v; its mask must be the one rola_block_mask returns, bit for bit, and
+    its output the one the separate entry points compose to."""
+    cfg = SMALL[case]
+    x, h = draw(cfg, torch.bfloat16)
+    out, kv = run_forward(rl, cfg, x, "bf16")
+    c = rl.make_config(cfg, rl.ROLA_BF16)
+    ws = rl.workspace(c)
+    kv2 = torch.empty_like(kv)
+    rl.block_mask(c, dev(x["q"]), dev(x["k"]), kv2, ws)
+    C = torch.empty((cfg["B"], cfg["H"], cfg["r"], 128), dtype=torch.float32, device="cuda")
+    rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, None, ws)
+    o_s = torch.empty_like(out)
+    rl.sparse_attn(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), kv2, o_s, ws)
+    o = torch.empty_like(out)
+    rl.lowrank_apply(c, dev(x["q"]), dev(x["P_q"]), C, dev(x["gate"]), o_s, o, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(kv, kv2)
+    assert torch.equal(out, o)
+
+
 def test_forward_is_deterministic_and_stays_in_bounds(rl):
     """Two runs are bitwise equal; bytes around the output are never written."""
     cfg = SMALL["ragged_585_r64"]
