@@ -91,9 +91,26 @@ typedef struct {
     int32_t debug_flags;       /* 0 normally.  ROLA_DEBUG_SKIP_FIRST_K_COPY makes each CTA of the
                                   bf16 sparse kernel skip its first K copy, so a bounded wait runs
                                   out and the call reports ROLA_ERR_TIMEOUT (tests the timeout path) */
+    int32_t lowrank_rope;      /* where the truncated RoPE sits in the low-rank features; one of
+                                  rola_lowrank_rope_t, default ROLA_LOWRANK_ROPE_OUTSIDE */
 } rola_config_t;
 
 #define ROLA_DEBUG_SKIP_FIRST_K_COPY 1
+
+/*
+ * Placement of the truncated rotation R_r in the low-rank features (the three
+ * orderings the paper compares in its RoPE-placement study, Tab. mechanism):
+ *   OUTSIDE  k~_q = R_r(q) SiLU(P_k k^n_q)   Eq. (qklr), the RoLA branch
+ *   INSIDE   k~_q = SiLU(R_r(q) P_k k^n_q)   Prop. inside (App. inside): no
+ *            exact relative factorisation, the summary leaks absolute position
+ *   NONE     k~_q = SiLU(P_k k^n_q)          position-blind low-rank branch
+ * and the same for q~_p.  The sparse branch always uses the full RoPE.
+ */
+typedef enum {
+    ROLA_LOWRANK_ROPE_OUTSIDE = 0,
+    ROLA_LOWRANK_ROPE_INSIDE = 1,
+    ROLA_LOWRANK_ROPE_NONE = 2
+} rola_lowrank_rope_t;
 
 /* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
 rola_status_t rola_config_init(rola_config_t* cfg);
@@ -138,7 +155,8 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
 
 /*
  * Kernel (3): low-rank summary, Eq. (qklr) and Eq. (ctx):
- *   k~_q = R_r(q) SiLU(P_k k^n_q),   C = sum_q k~_q v_q^T,   z = sum_q k~_q.
+ *   k~_q = R_r(q) SiLU(P_k k^n_q),   C = sum_q k~_q v_q^T,   z = sum_q k~_q
+ * (k~ as cfg->lowrank_rope places the rotation).
  * R_r keeps the first r coordinates (r/2 complete pairs) of the native RoPE
  * ordering (Sec. 4.2).  The reduction over N is split across CTAs (one
  * contiguous token range each) and combined in a fixed order, so results are
@@ -152,7 +170,7 @@ rola_status_t rola_lowrank_summary(const rola_config_t* cfg, const void* k, cons
 
 /*
  * Kernel (4): low-rank readout and gated fusion, Eq. (ctx) and Eq. (gate):
- *   q~_p   = R_r(p) SiLU(P_q q^n_p)
+ *   q~_p   = R_r(p) SiLU(P_q q^n_p)            (as cfg->lowrank_rope places R_r)
  *   O^lr_p = y_p / sqrt(mean_i y_{p,i}^2 + eps_lr),   y_p = q~_p^T C
  *   r_p    = sqrt(mean_i (O^s_{p,i})^2 + eps_fuse)
  *   O_p    = (O^s_p / r_p + g_p O^lr_p) r_p

@@ -42,6 +42,8 @@ rola_status_t validate(const rola_config_t* c)
         if (c->pos_offset[a] < -(1 << 20) || c->pos_offset[a] > (1 << 20)) return ROLA_ERR_INVALID_ARG;
     if (c->wait_limit_ms < 0 || c->wait_limit_ms > 60000) return ROLA_ERR_INVALID_ARG;
     if (c->debug_flags & ~ROLA_DEBUG_SKIP_FIRST_K_COPY) return ROLA_ERR_INVALID_ARG;
+    if (c->lowrank_rope < ROLA_LOWRANK_ROPE_OUTSIDE || c->lowrank_rope > ROLA_LOWRANK_ROPE_NONE)
+        return ROLA_ERR_INVALID_ARG;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
     if ((int64_t)c->B * c->H * c->N * c->d_h > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
@@ -63,6 +65,7 @@ Shape make_shape(const rola_config_t& c)
     s.sm_scale_log2 = (float)(1.4426950408889634 / sqrt((double)kDh));
     s.wait_limit_ns = (uint64_t)(c.wait_limit_ms > 0 ? c.wait_limit_ms : 2000) * 1000000ull;
     s.debug_flags = c.debug_flags;
+    s.lr_rope = c.lowrank_rope;
     return s;
 }
 

@@ -39,6 +39,7 @@ struct Shape {
     float sm_scale_log2;      // log2(e) / sqrt(128)
     uint64_t wait_limit_ns;   // bound of every device-side wait
     int debug_flags;          // ROLA_DEBUG_* test hooks
+    int lr_rope;              // rola_lowrank_rope_t
 };
 
 // Rotation (cos, sin) of pair m for the token at flat index n.
@@ -58,6 +59,21 @@ __device__ __forceinline__ float2 rope_cs(const float2* __restrict__ tab, const 
 __device__ __forceinline__ float2 rope_rotate(float x0, float x1, float2 cs)
 {
     return make_float2(__fmaf_rn(x0, cs.x, -__fmul_rn(x1, cs.y)), __fmaf_rn(x0, cs.y, __fmul_rn(x1, cs.x)));
+}
+
+// One pair of low-rank features from the projected pair (u0, u1) = the pair's
+// two rows of P x: R_r after SiLU (Eq. qklr, ROLA_LOWRANK_ROPE_OUTSIDE), before
+// it (Prop. inside, ROLA_LOWRANK_ROPE_INSIDE) or not at all (ROLA_LOWRANK_ROPE_NONE).
+// `act` is the SiLU evaluation the caller uses.
+template <typename Act>
+__device__ __forceinline__ float2 lowrank_pair(float u0, float u1, float2 cs, int mode, Act act)
+{
+    if (mode == ROLA_LOWRANK_ROPE_INSIDE) {
+        const float2 r = rope_rotate(u0, u1, cs);
+        return make_float2(act(r.x), act(r.y));
+    }
+    const float a0 = act(u0), a1 = act(u1);
+    return mode == ROLA_LOWRANK_ROPE_NONE ? make_float2(a0, a1) : rope_rotate(a0, a1, cs);
 }
 
 // ---------------------------------------------------------------- host side

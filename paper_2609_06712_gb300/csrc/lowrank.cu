@@ -14,6 +14,17 @@
 
 namespace rola {
 
+// SiLU evaluations: IEEE exp and divide (fp32 validation mode) and the
+// MUFU-based one of the bf16 readout
+struct SiluIeee {
+    __device__ float operator()(float x) const { return x / (1.0f + expf(-x)); }
+};
+struct SiluMufu {
+    __device__ float operator()(float x) const { return silu(x); }
+};
+__device__ constexpr SiluIeee silu_ieee{};
+__device__ constexpr SiluMufu silu_mufu{};
+
 // ===========================================================================
 // Split-N partitioning of the fp32 summary: CTA = (split, head).
 
@@ -82,10 +93,10 @@ __global__ void __launch_bounds__(256) summary_f32_kernel(Shape s, int tokens_pe
                 u0 = fmaf(Ks[r * (kDh + 1) + c], Ps[(2 * m) * (kDh + 1) + c], u0);
                 u1 = fmaf(Ks[r * (kDh + 1) + c], Ps[(2 * m + 1) * (kDh + 1) + c], u1);
             }
-            float x0 = u0 / (1.0f + expf(-u0)), x1 = u1 / (1.0f + expf(-u1));
             float2 cs = n < n_end ? rope_cs(tab, s, n, m) : make_float2(0.0f, 0.0f);
-            Us[r * (R + 1) + 2 * m] = x0 * cs.x - x1 * cs.y;
-            Us[r * (R + 1) + 2 * m + 1] = x0 * cs.y + x1 * cs.x;
+            const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, silu_ieee);
+            Us[r * (R + 1) + 2 * m] = f.x;
+            Us[r * (R + 1) + 2 * m + 1] = f.y;
         }
         __syncthreads();
         for (int r = 0; r < kF32Tile; ++r) {
@@ -214,10 +225,10 @@ __global__ void __launch_bounds__(128, 4) apply_bf16_kernel(Shape s, const __nv_
     for (int nt = 0; nt < NT; ++nt) {
         const int m = nt * 4 + t4;
         float2 c0 = rope_cs(tab, s, n_lo_c, m), c1 = rope_cs(tab, s, n_hi_c, m);
-        float x0 = silu(u[nt][0]), x1 = silu(u[nt][1]);
-        float x2 = silu(u[nt][2]), x3 = silu(u[nt][3]);
-        qf[nt][0] = pack_bf16(x0 * c0.x - x1 * c0.y, x0 * c0.y + x1 * c0.x);
-        qf[nt][1] = pack_bf16(x2 * c1.x - x3 * c1.y, x2 * c1.y + x3 * c1.x);
+        const float2 f0 = lowrank_pair(u[nt][0], u[nt][1], c0, s.lr_rope, silu_mufu);
+        const float2 f1 = lowrank_pair(u[nt][2], u[nt][3], c1, s.lr_rope, silu_mufu);
+        qf[nt][0] = pack_bf16(f0.x, f0.y);
+        qf[nt][1] = pack_bf16(f1.x, f1.y);
     }
     float y[16][4];
 #pragma unroll
@@ -311,10 +322,10 @@ __global__ void __launch_bounds__(256) apply_f32_kernel(Shape s, const float* __
             u0 = fmaf(Qs[r * (kDh + 1) + c], Ps[(2 * m) * (kDh + 1) + c], u0);
             u1 = fmaf(Qs[r * (kDh + 1) + c], Ps[(2 * m + 1) * (kDh + 1) + c], u1);
         }
-        float x0 = u0 / (1.0f + expf(-u0)), x1 = u1 / (1.0f + expf(-u1));
         float2 cs = rope_cs(tab, s, n, m);
-        Us[r * (R + 1) + 2 * m] = x0 * cs.x - x1 * cs.y;
-        Us[r * (R + 1) + 2 * m + 1] = x0 * cs.y + x1 * cs.x;
+        const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, silu_ieee);
+        Us[r * (R + 1) + 2 * m] = f.x;
+        Us[r * (R + 1) + 2 * m + 1] = f.y;
     }
     __syncthreads();
     const int row = tid >> 2, quarter = tid & 3;

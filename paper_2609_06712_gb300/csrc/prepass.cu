@@ -103,7 +103,9 @@ __device__ __forceinline__ void rotate8(const uint4& w, const float2 (&cs)[4], _
 }
 
 // SiLU with the approximate divide (the features enter the MMA in bf16)
-__device__ __forceinline__ float silu_fast(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
+struct SiluFast {
+    __device__ float operator()(float x) const { return __fdividef(x, 1.0f + __expf(-x)); }
+};
 
 template <int R>
 __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_constant__ CUtensorMap map_q,
@@ -352,9 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
 #pragma unroll
                 for (int j = 0; j < NTW; ++j) {
                     const int nt = nh * NTW + j;
-                    const float x0 = silu_fast(uacc[j][2 * hr]), x1 = silu_fast(uacc[j][2 * hr + 1]);
                     const float2 cs = valid ? kcs[hr][j] : make_float2(0.0f, 0.0f);
-                    const float2 y = rope_rotate(x0, x1, cs);
+                    const float2 y = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], cs, s.lr_rope, SiluFast{});
                     zacc[j][0] += y.x;
                     zacc[j][1] += y.y;
                     asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(ktb + tl * L::KT + (nt * 8 + t4 * 2) * 2),

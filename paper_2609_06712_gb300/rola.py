@@ -36,10 +36,13 @@ class RolaConfig(ctypes.Structure):
         ("dtype", ctypes.c_int32),
         ("wait_limit_ms", ctypes.c_int32),
         ("debug_flags", ctypes.c_int32),
+        ("lowrank_rope", ctypes.c_int32),
     ]
 
 
 ROLA_DEBUG_SKIP_FIRST_K_COPY = 1
+# rola_lowrank_rope_t: where the truncated RoPE sits in the low-rank features
+ROLA_LOWRANK_ROPE_OUTSIDE, ROLA_LOWRANK_ROPE_INSIDE, ROLA_LOWRANK_ROPE_NONE = 0, 1, 2
 
 
 class RolaError(RuntimeError):
@@ -103,6 +106,7 @@ def make_config(cfg: dict, dtype: int = ROLA_BF16) -> RolaConfig:
     c.eps_fuse = float(cfg.get("eps_fuse", 1e-6))
     c.gate_bias = float(cfg.get("gate_bias", -1.946))
     c.dtype = dtype
+    c.lowrank_rope = int(cfg.get("lowrank_rope", ROLA_LOWRANK_ROPE_OUTSIDE))
     return c
 
 

@@ -52,6 +52,7 @@ def test_defaults_and_sizes(rl):
     assert rl.library().rola_config_init(ctypes.byref(c)) == rl.ROLA_OK
     assert (c.d_h, c.block, list(c.rope_split), c.rope_theta) == (128, 64, [44, 42, 42], 10000.0)
     assert c.gate_bias == pytest.approx(-1.946) and c.eps_lr == pytest.approx(1e-6)
+    assert c.lowrank_rope == rl.ROLA_LOWRANK_ROPE_OUTSIDE and c.wait_limit_ms == 0 and c.debug_flags == 0
     from paper_2609_06712_gb300 import configs
     for name, nb, nk in [("tiny", 16, 2), ("wan13b_480p", 512, 51), ("wan14b_720p", 1182, 118),
                          ("wan14b_720p_long", 2307, 231)]:
@@ -91,6 +92,8 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
     ("wait_limit_ms", -1, 1),
     ("wait_limit_ms", 60001, 1),
     ("debug_flags", 2, 1),
+    ("lowrank_rope", 3, 1),
+    ("lowrank_rope", -1, 1),
 ])
 def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
     c = cfg_tiny(rl, **{field: value})
