@@ -253,7 +253,10 @@ def main():
         over["keep"] = args.keep
     if args.r is not None:
         over["r"] = args.r
-    cfg = configs.get(args.workload, **over)
+    if args.workload == "sweep":          # the rank x sparsity sweep at the 720p shape (seed of the sweep)
+        cfg = configs.sweep_config(args.r if args.r is not None else 32, args.keep if args.keep is not None else 0.1)
+    else:
+        cfg = configs.get(args.workload, **over)
     ws, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, cfg, ws, rank)
@@ -306,6 +309,9 @@ def main():
     stage_names = ["prepass", "select", "sparse_attn", "apply_fuse"]
     stage_ms = {n: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K))
                 for j, n in enumerate(stage_names)}
+    per_step = sorted(evs[i][0].elapsed_time(evs[i][4]) for i in range(K))
+    step_stats = {"median": statistics.median(per_step), "min": per_step[0],
+                  "p90": per_step[min(K - 1, int(round(0.9 * (K - 1))))]}
     assert rola.get_device_status(wsb) == rola.ROLA_OK
     tokens = cfg["B"] * cfg["N"]
     value = job_throughput(tokens, ms_step, ws)
@@ -457,6 +463,7 @@ def main():
                        "l2": "no flush: q, k, v are each larger than L2 (774 MB vs 129 MB)",
                        "parallelism": f"replica per GPU x{ws}"},
             "stage_ms": stage_ms,
+            "step_ms": step_stats,
             "roofline": roofline,
             "roofline_other": secondary,
             "dense": dense,

@@ -64,7 +64,6 @@ constexpr int kWGThreads = 128;
 constexpr uint32_t kQBytes = 64 * 128 * 2;          // one query block
 constexpr uint32_t kKVBytes = 128 * 128 * 2;        // a pair of key blocks
 constexpr uint32_t kPBytes = 128 * 64 * 2;          // P^T tile
-constexpr uint32_t kOBytes = 64 * 128 * 2;          // output staging
 constexpr int KS = 3;                               // K ring: pairs of key blocks ([chunk][block][row])
 constexpr int VB = 5;                               // V ring: single key blocks (16 KB, [chunk][row])
 constexpr uint32_t kVBlockBytes = 64 * 128 * 2;
@@ -72,9 +71,7 @@ constexpr uint32_t kSmemQ = 0;
 constexpr uint32_t kSmemK = kSmemQ + kQBytes;
 constexpr uint32_t kSmemV = kSmemK + KS * kKVBytes;
 constexpr uint32_t kSmemP = kSmemV + VB * kVBlockBytes;
-constexpr uint32_t kSmemO = kSmemP;                 // output staging reuses P buffer 0 (free at the epilogue)
 constexpr uint32_t kSmemTiles = kSmemP + 2 * kPBytes;   // 224 KB, 1024-aligned pieces
-static_assert(kOBytes <= kPBytes, "output staging fits a P buffer");
 constexpr uint32_t kTmemCols = 256;                 // S^T x2 (64 cols each), O^T x2
 constexpr float kRescaleThreshold = 8.0f;           // log2 units
 
@@ -510,36 +507,26 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 if (lane == 0) mbar_arrive(bar(P_FULL + sb));
             }
             if (!ok) break;
-            // ---- epilogue: O^s = O^T / l, transposed through shared memory
-            if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
-            fence_after_sync();
+            // ---- epilogue: O^s = O^T / l.  l is final after the last tile, so its
+            // reduction overlaps the last P V; then thread wtid writes d = wtid of
+            // this warpgroup's 32 query rows, so each warp store is one 64-byte segment
             column_reduce<false>(l, sm, wg, wtid, sm.inv_l + col0);
             if (wtid < kCols) sm.inv_l[col0 + wtid] = 1.0f / sm.inv_l[col0 + wtid];
             bar_sync(1 + wg, kWGThreads);
+            if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
+            fence_after_sync();
             {
                 float ov[kCols];
                 tmem_ld_cols<kCols>(tmem + lane_off + 128 + ob * 64 + col0, ov);
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
-                __nv_bfloat16* ostage = reinterpret_cast<__nv_bfloat16*>(tiles + kSmemO);
+                __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + wtid;
+                const int rows = min(64, s.N - qb * 64) - col0;     // rows of this warpgroup inside the sequence
 #pragma unroll
                 for (int q = 0; q < kCols; ++q)
-                    ostage[(col0 + q) * 128 + wtid] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
+                    if (q < rows) dst[(size_t)q * kDh] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
             }
-            bar_sync(1 + kSoftmaxWG, kSoftmaxWarps * 32);                  // both halves staged
-            {
-                const uint4* src = reinterpret_cast<const uint4*>(tiles + kSmemO);
-                __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64) * kDh;
-#pragma unroll
-                for (int it = 0; it < 1024 / (kSoftmaxWarps * 32); ++it) {
-                    const int e = it * kSoftmaxWarps * 32 + tid;
-                    const int row = e >> 4, c = e & 15;
-                    if (qb * 64 + row < s.N)
-                        *reinterpret_cast<uint4*>(dst + (size_t)row * kDh + c * 8) = src[e];
-                }
-            }
-            bar_sync(1 + kSoftmaxWG, kSoftmaxWarps * 32);
         }
         if (!ok) record_timeout(p, 3);
     }
