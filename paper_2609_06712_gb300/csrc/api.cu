@@ -268,7 +268,8 @@ rola_status_t rola_lowrank_apply(const rola_config_t* cfg, const void* q, const 
     ROLA_CHECK(prologue(*cfg, ws, w, st));
     __nv_bfloat16* Cbf = at<__nv_bfloat16>(ws, w.Cbf);
     if (cfg->dtype == ROLA_BF16) ROLA_TRY(launch_c_to_bf16(s, C, Cbf, st));
-    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, C, Cbf, gate, o_s, o, at<float2>(ws, w.table), st));
+    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, C, Cbf, gate, o_s, o, at<float2>(ws, w.table),
+                                  at<DeviceStatus>(ws, w.status), st));
     return ROLA_OK;
 }
 
@@ -316,7 +317,7 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                 at<DeviceStatus>(ws, w.status), st));
     ROLA_TRY(mark(3));
     ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, o,
-                                  o, at<float2>(ws, w.table), st));
+                                  o, at<float2>(ws, w.table), at<DeviceStatus>(ws, w.status), st));
     ROLA_TRY(mark(4));
     return ROLA_OK;
 }

@@ -103,7 +103,12 @@ cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, 
 cudaError_t launch_c_to_bf16(const Shape& s, const float* C, __nv_bfloat16* Cbf, cudaStream_t st);
 cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q, const void* P_q,
                                  const float* C, const __nv_bfloat16* Cbf, const float* gate,
-                                 const void* o_s, void* o, const float2* tab, cudaStream_t st);
+                                 const void* o_s, void* o, const float2* tab, DeviceStatus* status,
+                                 cudaStream_t st);
+// bf16 readout + fusion (readout.cu): persistent, TMA in and out, P_q and C once per head
+cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const __nv_bfloat16* Cbf,
+                           const float* gate, const void* o_s, void* o, const float2* tab, DeviceStatus* status,
+                           cudaStream_t st);
 
 // Number of N-splits of the summary reduction for this shape (fp32 kernel).
 int summary_splits(const Shape& s);

@@ -370,19 +370,16 @@ static cudaError_t launch_apply_bf16_r(const Shape& s, const void* q, const void
 
 cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q, const void* P_q, const float* C,
                                  const __nv_bfloat16* Cbf, const float* gate, const void* o_s, void* o,
-                                 const float2* tab, cudaStream_t st)
+                                 const float2* tab, DeviceStatus* status, cudaStream_t st)
 {
     if (dt == ROLA_BF16) {
+        // small r: one CTA per block, four per SM (P_q and C re-read from L2 are cheap);
+        // large r: the persistent kernel, which loads P_q and C once per head
         switch (s.r) {
             case 16: return launch_apply_bf16_r<16>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
             case 32: return launch_apply_bf16_r<32>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
             case 48: return launch_apply_bf16_r<48>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 64: return launch_apply_bf16_r<64>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 80: return launch_apply_bf16_r<80>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 96: return launch_apply_bf16_r<96>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 112: return launch_apply_bf16_r<112>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 128: return launch_apply_bf16_r<128>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            default: return cudaErrorInvalidValue;
+            default: return launch_readout(s, q, P_q, Cbf, gate, o_s, o, tab, status, st);
         }
     }
     size_t smem = sizeof(float) * ((size_t)s.r * (kDh + 1) + (size_t)s.r * kDh + kBlock * (kDh + 1) +
