@@ -82,7 +82,8 @@ typedef struct {
     double rope_theta;         /* RoPE base; default 10000 */
     int32_t block;             /* block size for queries and keys; 64 */
     float keep_ratio;          /* n_keep = clamp(floor(keep_ratio*nKB + 0.5), 1, nKB) */
-    int32_t r;                 /* low-rank width, even, 16 <= r <= d_h, r % 16 == 0 */
+    int32_t r;                 /* low-rank width (Sec. 4.2), 8 <= r <= d_h, r % 8 == 0; the bf16
+                                  kernels run at r rounded up to 16 with zero rows of P */
     float eps_lr;              /* RMSNorm epsilon of the low-rank readout; default 1e-6 */
     float eps_fuse;            /* epsilon of the sparse-output RMS r_p, Eq. (gate); default 1e-6 */
     float gate_bias;           /* g = sigmoid(gate_bias) when gate == NULL; default -1.946 */

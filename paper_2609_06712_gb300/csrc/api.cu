@@ -34,7 +34,7 @@ rola_status_t validate(const rola_config_t* c)
     if (!(c->rope_theta > 0.0) || !isfinite(c->rope_theta)) return ROLA_ERR_INVALID_ARG;
     if (!(c->keep_ratio >= 0.0f && c->keep_ratio <= 1.0f)) return ROLA_ERR_INVALID_ARG;
     if (c->r < 2 || (c->r & 1) || c->r > c->d_h) return ROLA_ERR_INVALID_ARG;
-    if (c->r % 16 != 0) return ROLA_ERR_UNSUPPORTED;
+    if (c->r % 8 != 0) return ROLA_ERR_UNSUPPORTED;
     if (!(c->eps_lr >= 0.0f) || !(c->eps_fuse >= 0.0f) || !isfinite(c->eps_lr) || !isfinite(c->eps_fuse))
         return ROLA_ERR_INVALID_ARG;
     if (!isfinite(c->gate_bias)) return ROLA_ERR_INVALID_ARG;
@@ -54,6 +54,7 @@ Shape make_shape(const rola_config_t& c)
 {
     Shape s;
     s.B = c.B; s.H = c.H; s.N = c.N; s.r = c.r;
+    s.rp = (c.r + 15) & ~15;
     s.nB = num_blocks_of(c);
     s.n_keep = num_keep_of(c);
     s.T = c.T; s.Hh = c.Hh; s.Ww = c.Ww;
@@ -97,12 +98,12 @@ Workspace layout(const rola_config_t& c)
     w.kv_idx = off; off = align_up(off + 4 * bh * s.nB * s.n_keep);
     w.C = off; off = align_up(off + 4 * bh * c.r * kDh);
     w.z = off; off = align_up(off + 4 * bh * c.r);
-    w.Cbf = off; off = align_up(off + 2 * bh * c.r * kDh);
+    w.Cbf = off; off = align_up(off + 2 * bh * s.rp * kDh);           // zero-padded to rp rows
     // summary partials: fp32 split-N slots, or the bf16 pre-pass's per-(CTA, head) slots
     const size_t units = bh * s.nB;
     w.prepass_slots = (units < (size_t)kMaxPrepassCtas ? units : (size_t)kMaxPrepassCtas) + bh - 1;
     const size_t slots = c.dtype == ROLA_BF16 ? w.prepass_slots : bh * w.nsplit;
-    w.partials = off; off = align_up(off + 4 * slots * ((size_t)c.r * kDh + c.r));
+    w.partials = off; off = align_up(off + 4 * slots * ((size_t)s.rp * kDh + s.rp));
     w.total = off;
     return w;
 }

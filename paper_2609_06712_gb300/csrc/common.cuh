@@ -32,6 +32,8 @@ struct DeviceStatus {
 // Kernel-side view of a validated configuration.
 struct Shape {
     int B, H, N, nB, n_keep, r;
+    int rp;                   // r rounded up to a multiple of 16: the width the bf16 kernels run at
+                              // (rows r .. rp-1 of P are read as zero, so those features are zero)
     int T, Hh, Ww;
     int pt, px;               // pairs on the temporal / height axis (rest: width)
     float eps_lr, eps_fuse;

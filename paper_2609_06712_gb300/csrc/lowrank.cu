@@ -136,16 +136,19 @@ __global__ void summary_combine_kernel(Shape s, int nsplit, const float* __restr
     }
 }
 
-__global__ void c_to_bf16_kernel(int n, const float* __restrict__ C, __nv_bfloat16* __restrict__ Cbf)
+// C [B*H][r][128] fp32 -> bf16 [B*H][rp][128], rows r .. rp-1 zero
+__global__ void c_to_bf16_kernel(int r, int rp, int n, const float* __restrict__ C, __nv_bfloat16* __restrict__ Cbf)
 {
-    int e = blockIdx.x * blockDim.x + threadIdx.x;
-    if (e < n) Cbf[e] = __float2bfloat16_rn(C[e]);
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;     // index into the padded copy
+    if (e >= n) return;
+    const int bh = e / (rp * kDh), rest = e - bh * rp * kDh, row = rest / kDh;
+    Cbf[e] = row < r ? __float2bfloat16_rn(C[((size_t)bh * r) * kDh + rest]) : __float2bfloat16_rn(0.0f);
 }
 
 cudaError_t launch_c_to_bf16(const Shape& s, const float* C, __nv_bfloat16* Cbf, cudaStream_t st)
 {
-    int n = s.B * s.H * s.r * kDh;
-    c_to_bf16_kernel<<<(n + 255) / 256, 256, 0, st>>>(n, C, Cbf);
+    int n = s.B * s.H * s.rp * kDh;
+    c_to_bf16_kernel<<<(n + 255) / 256, 256, 0, st>>>(s.r, s.rp, n, C, Cbf);
     return cudaGetLastError();
 }
 
@@ -195,8 +198,8 @@ __global__ void __launch_bounds__(128, 4) apply_bf16_kernel(Shape s, const __nv_
     const uint32_t sO = sQ + kBlock * 256;
     uint8_t* o_gen = smem + 2 * R * 256 + kBlock * 256;
     const size_t head = (size_t)bh * s.N * kDh;
-    load_rows_async(sP, Pq + (size_t)h * R * kDh, 0, R, R, tid, 128);
-    load_rows_async(sC, Cbf + (size_t)bh * R * kDh, 0, R, R, tid, 128);
+    load_rows_async(sP, Pq + (size_t)h * s.r * kDh, 0, R, s.r, tid, 128);     // rows past r read as zero
+    load_rows_async(sC, Cbf + (size_t)bh * R * kDh, 0, R, R, tid, 128);       // rp rows, zero-padded
     load_rows_async(sQ, q + head, blk * kBlock, kBlock, s.N, tid, 128);
     load_rows_async(sO, o_s + head, blk * kBlock, kBlock, s.N, tid, 128);
     cp_async_commit();
@@ -375,7 +378,7 @@ cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q,
     if (dt == ROLA_BF16) {
         // small r: one CTA per block, four per SM (P_q and C re-read from L2 are cheap);
         // large r: the persistent kernel, which loads P_q and C once per head
-        switch (s.r) {
+        switch (s.rp) {
             case 16: return launch_apply_bf16_r<16>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
             case 32: return launch_apply_bf16_r<32>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
             case 48: return launch_apply_bf16_r<48>(s, q, P_q, Cbf, gate, o_s, o, tab, st);

@@ -75,7 +75,7 @@ extern "C" rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, c
     // fewer CTAs (bf16) or splits (fp32) if needed to fit, but at least one slot per head
     const size_t head = align256(sizeof(DeviceStatus));
     const size_t table = align256(sizeof(float2) * (size_t)(cfg->T + cfg->Hh + cfg->Ww) * kPairs);
-    const size_t slot = sizeof(float) * ((size_t)s.r * kDh + s.r);
+    const size_t slot = sizeof(float) * ((size_t)s.rp * kDh + s.rp);
     const size_t bh = (size_t)s.B * s.H;
     if (head + table + bh * slot > kStaticScratchBytes) return ROLA_ERR_UNSUPPORTED;   // layer too large
     const size_t fit = (kStaticScratchBytes - head - table) / slot;                   // slots available

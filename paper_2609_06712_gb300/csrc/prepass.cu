@@ -253,9 +253,9 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
                 clear();
             }
             // P_k of the new head (every reader of the old one has passed the last barrier)
-            const __nv_bfloat16* src = p.Pk + (size_t)(bh % s.H) * R * kDh;
+            const __nv_bfloat16* src = p.Pk + (size_t)(bh % s.H) * s.r * kDh;
             for (int e = tid; e < R * 16; e += kConsumers) {
-                const uint4 w = __ldg(reinterpret_cast<const uint4*>(src) + e);
+                const uint4 w = (e >> 4) < s.r ? __ldg(reinterpret_cast<const uint4*>(src) + e) : make_uint4(0, 0, 0, 0);
                 asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(sP + sw128(e >> 4, e & 15)), "r"(w.x),
                              "r"(w.y), "r"(w.z), "r"(w.w)
                              : "memory");
@@ -414,7 +414,7 @@ __global__ void prepass_combine_kernel(Shape s, int ctas, int units, const float
                                        float* __restrict__ C, float* __restrict__ z, __nv_bfloat16* __restrict__ Cbf)
 {
     const int bh = blockIdx.y;
-    const int per = s.r * kDh + s.r;
+    const int per = s.rp * kDh + s.rp;                 // one partial slot (rp rows)
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= per) return;
     // CTAs whose unit ranges meet head bh: those holding its first and last unit, and all between
@@ -422,11 +422,12 @@ __global__ void prepass_combine_kernel(Shape s, int ctas, int units, const float
     const int c1 = (int)((((long long)(bh + 1) * s.nB) * ctas - 1) / units);
     float x = 0.0f;
     for (int c = c0; c <= c1; ++c) x += partials[(size_t)(c + bh) * per + e];
-    if (e < s.r * kDh) {
-        C[(size_t)bh * s.r * kDh + e] = x;
-        if (Cbf) Cbf[(size_t)bh * s.r * kDh + e] = __float2bfloat16_rn(x);
-    } else if (z) {
-        z[(size_t)bh * s.r + (e - s.r * kDh)] = x;
+    // C and z have r rows; the bf16 copy keeps all rp (rows past r are exactly zero)
+    if (e < s.rp * kDh) {
+        if (e < s.r * kDh) C[(size_t)bh * s.r * kDh + e] = x;
+        if (Cbf) Cbf[(size_t)bh * s.rp * kDh + e] = __float2bfloat16_rn(x);
+    } else if (z && e - s.rp * kDh < s.r) {
+        z[(size_t)bh * s.r + (e - s.rp * kDh)] = x;
     }
 }
 
@@ -482,7 +483,7 @@ cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* 
     p.partials = partials;
     p.status = status;
     p.units = s.B * s.H * s.nB;
-    switch (s.r) {
+    switch (s.rp) {
         case 16: return launch_r<16>(mq, mk, mv, p, ctas, fuse, st);
         case 32: return launch_r<32>(mq, mk, mv, p, ctas, fuse, st);
         case 48: return launch_r<48>(mq, mk, mv, p, ctas, fuse, st);
@@ -498,7 +499,7 @@ cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* 
 cudaError_t launch_prepass_combine(const Shape& s, int ctas, const float* partials, float* C, float* z,
                                    __nv_bfloat16* Cbf, cudaStream_t st)
 {
-    const int per = s.r * kDh + s.r;
+    const int per = s.rp * kDh + s.rp;
     const int units = s.B * s.H * s.nB;
     prepass_combine_kernel<<<dim3((per + 255) / 256, s.B * s.H), 256, 0, st>>>(s, ctas, units, partials, C, z, Cbf);
     return cudaGetLastError();

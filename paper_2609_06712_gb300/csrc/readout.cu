@@ -126,10 +126,10 @@ __global__ void __launch_bounds__(kThreads, 1) readout_kernel(const __grid_const
         const int st = i % kStages;
         if (bh != hb) {
             // P_q of the head and C of (batch, head); every reader of the old ones has passed the last barrier
-            const uint4* srcP = reinterpret_cast<const uint4*>(p.Pq + (size_t)(bh % s.H) * R * kDh);
-            const uint4* srcC = reinterpret_cast<const uint4*>(p.Cbf + (size_t)bh * R * kDh);
+            const uint4* srcP = reinterpret_cast<const uint4*>(p.Pq + (size_t)(bh % s.H) * s.r * kDh);
+            const uint4* srcC = reinterpret_cast<const uint4*>(p.Cbf + (size_t)bh * R * kDh);   // rp rows
             for (int e = tid; e < R * 16; e += kThreads) {
-                const uint4 a = __ldg(srcP + e), c = __ldg(srcC + e);
+                const uint4 a = (e >> 4) < s.r ? __ldg(srcP + e) : make_uint4(0, 0, 0, 0), c = __ldg(srcC + e);
                 const uint32_t off = sw128(e >> 4, e & 15);
                 asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(sP + off), "r"(a.x), "r"(a.y), "r"(a.z),
                              "r"(a.w)
@@ -344,7 +344,7 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
     p.tab = tab;
     p.status = status;
     p.units = units;
-    switch (s.r) {
+    switch (s.rp) {
         case 16: return launch_r<16>(mq, mos, mo, p, ctas, st);
         case 32: return launch_r<32>(mq, mos, mo, p, ctas, st);
         case 48: return launch_r<48>(mq, mos, mo, p, ctas, st);

@@ -81,7 +81,7 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
     ("B", 0, 1),
     ("d_h", 64, 2),            # valid shape, not built
     ("block", 128, 2),
-    ("r", 24, 2),              # even but not a multiple of 16
+    ("r", 12, 2),              # even but not a multiple of 8
     ("r", 15, 1),
     ("r", 256, 1),             # r > d_h
     ("keep_ratio", 1.5, 1),

@@ -37,6 +37,7 @@ CASES = {
     "ragged_585_r64": layer(T=5, Hh=9, Ww=13, H=2, r=64, keep=0.3, seed=22),
     "r48_gate": layer(T=3, Hh=10, Ww=20, H=2, r=48, keep=0.2, seed=24, dist="normal_gate"),
     "r128": layer(T=2, Hh=12, Ww=16, H=2, r=128, keep=0.25, seed=27),
+    "r8": layer(T=3, Hh=7, Ww=11, H=2, r=8, keep=0.25, seed=28),
 }
 MODES = {"inside": (1, O.ROPE_INSIDE), "none": (2, O.ROPE_NONE)}
 DTYPES = [("bf16", torch.bfloat16), ("fp32", torch.float32)]

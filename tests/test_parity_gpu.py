@@ -42,6 +42,9 @@ SMALL = {
     "r48_gate": layer(T=3, Hh=10, Ww=20, H=2, r=48, keep=0.2, seed=24, dist="normal_gate"),
     "rmsnorm_gain_b2": layer(T=4, Hh=8, Ww=9, B=2, H=2, r=32, keep=0.25, seed=25, dist="rmsnorm_gain"),
     "offset": layer(T=3, Hh=8, Ww=8, H=2, r=32, keep=0.25, seed=26, pos_offset=(5, -3, 7)),
+    # ranks that are not multiples of 16 (the paper's sweep starts at r = 8)
+    "r8_ragged": layer(T=3, Hh=7, Ww=11, H=2, r=8, keep=0.25, seed=28),
+    "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=29, dist="normal_gate"),
 }
 
 
