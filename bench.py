@@ -348,6 +348,28 @@ def main():
                        "bytes": 3 * tensor_bytes, "note": "read q and O^s, write O"},
     }
 
+    # ---- the token gate g = sigmoid(X w_g + b_g) from the block input X [B][N][H*128]
+    # (an input of the layer step above; timed on its own)
+    d_model = cfg["H"] * 128
+    xg = inputs.make_gate_inputs(cfg["B"], cfg["N"], d_model, dtype=torch.bfloat16, device=dev, seed=7)
+    gbuf = torch.empty((cfg["B"], cfg["N"]), dtype=torch.float32, device=dev)
+    for _ in range(3):
+        rola.gate(c, xg["X"], xg["w_g"], xg["b_g"], gbuf)
+    torch.cuda.synchronize()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record(stream)
+    for _ in range(10):
+        rola.gate(c, xg["X"], xg["w_g"], xg["b_g"], gbuf)
+    g1.record(stream)
+    torch.cuda.synchronize()
+    gate_ms = g0.elapsed_time(g1) / 10
+    gate_bytes = float(xg["X"].numel() * 2 + d_model * 2 + gbuf.numel() * 4)
+    secondary["gate"] = {"bound": "hbm", "ms": gate_ms, "bytes": gate_bytes,
+                         "achieved_gbs": gate_bytes / (gate_ms * 1e-3) / 1e9, "peak_gbs": hbm,
+                         "frac": gate_bytes / (gate_ms * 1e-3) / 1e9 / hbm,
+                         "note": f"X [B][N][{d_model}] bf16 read once ({xg['X'].numel() * 2 / 1e6:.0f} MB)"}
+    del xg, gbuf
+
     # ---- end to end through the public API with host buffers
     # Every step copies its inputs from pinned host memory and reads its output
     # back.  Serial: copy in, layer, copy out on one stream.  Pipelined (the

@@ -213,6 +213,20 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                  void* const* stage_events);
 
 /*
+ * Token gate of the gated fusion (Sec. fusion; Alg. 1, token-wise scalar gate):
+ *   g_p = sigmoid(x_p . w_g + b_g)
+ * one scalar per token from the attention block's input hidden states; the
+ * result is the `gate` argument of rola_forward / rola_lowrank_apply.
+ *   X       : [B][N][d_model], cfg->dtype (bf16 or fp32);  w_g : [d_model], cfg->dtype
+ *   b_g     : the gate bias (the paper initialises it to -1.946, so g starts near 1/8)
+ *   gate    : out, fp32 [B][N]
+ * d_model must be a multiple of 8 and at least 8; X and w_g 16-byte aligned.
+ * Uses cfg->B, cfg->N and cfg->dtype; needs no workspace.  Accumulates in fp32.
+ */
+rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g, float b_g,
+                        int32_t d_model, float* gate, void* stream);
+
+/*
  * rola_lowrank_summary_static: the low-rank summary (C and optionally z, as
  * rola_lowrank_summary computes them) for callers that cannot give the
  * library any device scratch -- e.g. a plugin whose host framework owns the

@@ -77,6 +77,7 @@ def _get():
             lib.orc_block_mask.argtypes = [cfgp, P, P, P, P, P, P]
             lib.orc_sparse_attn.argtypes = [cfgp, P, P, P, P, ctypes.c_int, P, P]
             lib.orc_forward.argtypes = [cfgp, P, P, P, P, P, P, P, P, P, P, P, P, P]
+            lib.orc_gate.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, ctypes.c_double, P]
             _lib = lib
     return _lib
 
@@ -198,6 +199,17 @@ def lowrank_readout(cfg: dict, q, Pq, C, rope_mode: int = ROPE_OUTSIDE) -> np.nd
     y = np.empty((c.B, c.H, c.N, c.dh))
     _get().orc_lowrank_readout(ctypes.byref(c), qp, Pqp, C.ctypes.data, y.ctypes.data)
     return y
+
+
+def gate(X, w, b: float) -> np.ndarray:
+    """Token gate g = sigmoid(X w_g + b_g) of the gated fusion (Sec. fusion); X [B][N][D], w [D] -> [B][N]."""
+    X, Xp = _f32(X)
+    w, wp = _f32(w)
+    B, N, D = X.shape
+    assert w.shape == (D,)
+    g = np.empty((B, N))
+    _get().orc_gate(B, N, D, Xp, wp, float(b), g.ctypes.data)
+    return g
 
 
 def lowrank_explicit(cfg: dict, q, k, v, Pq, Pk, rope_mode: int = ROPE_OUTSIDE) -> np.ndarray:

@@ -588,3 +588,18 @@ void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* 
     free(z);
     free(mask);
 }
+
+/* Token gate of the gated fusion (Sec. fusion, Alg. 1 "token-wise scalar
+ * gate"): g_p = sigmoid(x_p . w_g + b_g), one scalar per token from the
+ * attention block's input hidden state x_p (d_model wide).  X is [B][N][D],
+ * w [D], g [B][N]. */
+void orc_gate(int B, int N, int D, const float* X, const float* w, double b, double* g)
+{
+#pragma omp parallel for schedule(static)
+    for (long p = 0; p < (long)B * N; ++p) {
+        const float* x = X + (size_t)p * D;
+        double logit = b;
+        for (int d = 0; d < D; ++d) logit += (double)x[d] * (double)w[d];
+        g[p] = 1.0 / (1.0 + exp(-logit));
+    }
+}

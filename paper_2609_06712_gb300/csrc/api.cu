@@ -330,6 +330,17 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
     return rola_forward_timed(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, ws_bytes, stream, nullptr);
 }
 
+rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g, float b_g, int32_t d_model,
+                        float* gate, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!X || !w_g || !gate || d_model < 8 || d_model % 8 != 0 || !isfinite(b_g)) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(w_g) || (reinterpret_cast<uintptr_t>(gate) & 3u)) return ROLA_ERR_INVALID_ARG;
+    ROLA_TRY(launch_gate(cfg->dtype, (long long)cfg->B * cfg->N, d_model, X, w_g, b_g, gate,
+                         static_cast<cudaStream_t>(stream)));
+    return ROLA_OK;
+}
+
 rola_status_t rola_get_device_status(const void* ws, void* stream)
 {
     if (!ws) return ROLA_ERR_WORKSPACE;

@@ -112,6 +112,10 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
                            const float* gate, const void* o_s, void* o, const float2* tab, DeviceStatus* status,
                            cudaStream_t st);
 
+// Token gate g = sigmoid(X w_g + b) over `rows` rows of D features (gate.cu).
+cudaError_t launch_gate(rola_dtype_t dt, long long rows, int D, const void* X, const void* w, float b, float* g,
+                        cudaStream_t st);
+
 // Number of N-splits of the summary reduction for this shape (fp32 kernel).
 int summary_splits(const Shape& s);
 

@@ -58,3 +58,16 @@ def make_inputs(cfg: dict, dtype: torch.dtype = torch.bfloat16, device="cpu", se
     out = dict(q=q.to(dtype), k=k.to(dtype), v=v.to(dtype), P_q=P_q.to(dtype), P_k=P_k.to(dtype),
                gate=gate)
     return out
+
+
+def make_gate_inputs(B: int, N: int, d_model: int, dtype: torch.dtype = torch.bfloat16, device="cpu",
+                     seed: int = 0) -> dict:
+    """Inputs of the token gate g = sigmoid(X w_g + b_g): the attention block's input hidden states
+    X ~ N(0, 1) [B][N][d_model] (a stand-in for the normalised block input), w_g ~ N(0, 1/d_model)
+    (so the logit is ~N(0, 1) around the bias) and the paper's initial bias b_g = -1.946."""
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    f32 = dict(dtype=torch.float32, device=device, generator=g)
+    X = torch.randn((B, N, d_model), **f32)
+    w = torch.randn((d_model,), **f32) * (1.0 / d_model) ** 0.5
+    return dict(X=X.to(dtype), w_g=w.to(dtype), b_g=-1.946)

@@ -71,6 +71,7 @@ def _load():
         "rola_lowrank_apply": (st, [cfgp, P, P, P, P, P, P, P, S, P]),
         "rola_forward": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P]),
         "rola_forward_timed": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P, P]),
+        "rola_gate": (st, [cfgp, P, P, ctypes.c_float, ctypes.c_int32, P, P]),
         "rola_get_device_status": (st, [P, P]),
         "rola_status_string": (ctypes.c_char_p, [st]),
     }
@@ -177,6 +178,12 @@ def lowrank_apply(c, q, P_q, C, gate, o_s, o, ws, stream=None):
 def forward(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, stream=None):
     _check(_lib.rola_forward(ctypes.byref(c), _p(q), _p(k), _p(v), _p(P_q), _p(P_k), _p(gate), _p(o),
                              _p(kv_idx_out), _p(ws), ws.numel(), _stream(stream)), "rola_forward")
+
+
+def gate(c, X, w_g, b_g: float, gate_out, stream=None):
+    """Token gate g = sigmoid(X w_g + b_g) into gate_out (fp32 [B][N]); X [B][N][d_model]."""
+    _check(_lib.rola_gate(ctypes.byref(c), _p(X), _p(w_g), float(b_g), int(X.shape[-1]), _p(gate_out),
+                          _stream(stream)), "rola_gate")
 
 
 def forward_timed(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, events, stream=None):

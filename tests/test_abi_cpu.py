@@ -128,3 +128,19 @@ def test_status_strings(rl):
     for code in range(6):
         assert L.rola_status_string(code).decode().startswith("ROLA_")
     assert b"unknown" in L.rola_status_string(42)
+
+
+def test_gate_arguments_are_checked_before_launch(rl):
+    """Every call here is rejected by validation, so no kernel is launched on the dummy pointers."""
+    L = rl.library()
+    c = rl.make_config({"B": 1, "H": 2, "N": 1024, "T": 4, "Hh": 16, "Ww": 16, "keep": 0.125, "r": 16})
+    P = ctypes.c_void_p
+    ok, mis = P(0x10000), P(0x10004)
+    b = ctypes.byref(c)
+    for d_model in (0, 4, 12, -8):
+        assert L.rola_gate(b, ok, ok, -1.946, d_model, ok, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_gate(b, None, ok, -1.946, 128, ok, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_gate(b, mis, ok, -1.946, 128, ok, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_gate(b, ok, ok, float("nan"), 128, ok, None) == rl.ROLA_ERR_INVALID_ARG
+    c.N = 1000                                   # N != T * Hh * Ww
+    assert L.rola_gate(b, ok, ok, -1.946, 128, ok, None) == rl.ROLA_ERR_INVALID_ARG

@@ -36,6 +36,9 @@ MUTATIONS = {
     "fusion_norm": ("out[d] = (os[d] / rp + g * olr[d]) * rp;", "out[d] = (os[d] + g * olr[d]) * rp;"),
     "rmsnorm_mean": ("double inv = 1.0 / sqrt(ss / (double)dh + c->eps_lr);",
                      "double inv = 1.0 / sqrt(ss + c->eps_lr);"),
+    "gate_bias_dropped": ("double logit = b;", "double logit = 0.0;"),
+    "gate_sigmoid_sign": ("g[p] = 1.0 / (1.0 + exp(-logit));", "g[p] = 1.0 / (1.0 + exp(logit));"),
+    "gate_last_feature": ("for (int d = 0; d < D; ++d) logit +=", "for (int d = 0; d < D - 1; ++d) logit +="),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 

@@ -372,3 +372,32 @@ def test_default_gate_is_one_eighth(oracle):
     a = O.lowrank_apply(cfg, x["q"], x["P_q"], C, None, o_s)
     bb = O.lowrank_apply(cfg, x["q"], x["P_q"], C, g, o_s)
     np.testing.assert_allclose(a, bb, rtol=1e-7)
+
+
+# ------------------------------------------------------------------ token gate (Sec. fusion)
+
+
+def test_gate_pins(oracle):
+    """g = sigmoid(X w_g + b_g): with zero input the gate is sigmoid(b_g), 1/8 at the paper's initial bias;
+    flipping the signs of w_g and b_g gives 1 - g; the logit is additive in X and moves by delta * w_d when
+    one input feature moves by delta."""
+    import json
+    O = oracle
+    b0 = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "paper_constants.json")))[
+        "gate_bias_init"]["value"]
+    rng = np.random.default_rng(7)
+    B, N, D = 2, 37, 96
+    # multiples of 1/8 and 1/64: every product and the sums below are exact in fp32 and fp64
+    X = (rng.integers(-16, 17, (B, N, D)) / 8.0).astype(np.float32)
+    X2 = (rng.integers(-16, 17, (B, N, D)) / 8.0).astype(np.float32)
+    w = (rng.integers(-8, 9, D) / 64.0).astype(np.float32)
+    logit = lambda g: np.log(g / (1.0 - g))
+    g = O.gate(X, w, b0)
+    assert ((g > 0) & (g < 1)).all()
+    assert np.abs(O.gate(np.zeros_like(X), w, b0) - 0.125).max() < 1e-4
+    assert np.allclose(O.gate(X, -w, -b0), 1.0 - g, rtol=0, atol=1e-14)
+    assert np.allclose(logit(O.gate(X + X2, w, b0)), logit(g) + logit(O.gate(X2, w, b0)) - b0, rtol=0, atol=1e-9)
+    for d in (0, 41, D - 1):
+        Xd = X.copy()
+        Xd[:, :, d] += 0.5
+        assert np.allclose(logit(O.gate(Xd, w, b0)) - logit(g), 0.5 * float(w[d]), rtol=0, atol=1e-9)
