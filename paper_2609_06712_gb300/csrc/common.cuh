@@ -125,8 +125,8 @@ int summary_splits(const Shape& s);
 // always writes the summary partials, one slot per (CTA c, head bh) at index
 // c + bh, which launch_prepass_combine adds in CTA order.  With `ctas` CTAs
 // the partial buffer needs ctas + B*H - 1 slots of r*128 + r floats.
-constexpr int kMaxPrepassCtas = 256;
-int prepass_ctas(const Shape& s, int max_ctas);     // one per SM of the current device, at most max_ctas
+constexpr int kMaxPrepassCtas = 512;
+int prepass_ctas(const Shape& s, int max_ctas);     // its CTAs per SM x the SMs of the current device, at most max_ctas
 cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* k, const void* v,
                            const void* P_k, const float2* tab, void* qr, void* kr, float* qbar, float* kbar,
                            float* partials, DeviceStatus* status, cudaStream_t st);

@@ -6,30 +6,34 @@
 //       k~_n = R_r(n) SiLU(P_k k^n_n),  C = sum_n k~_n v_n^T,  z = sum_n k~_n.
 // Without q the kernel computes (2) alone (the summary entry point).
 //
-// Work unit = (head, 64-token block).  G persistent CTAs (one per SM) take
-// contiguous unit ranges [c U / G, (c + 1) U / G), so every CTA moves the same
-// number of bytes to within one unit and no wave is left partly empty.  A
-// range spans one or more heads; the CTA keeps C and z of the current head in
-// registers and writes them to partial slot c + head when the head changes or
-// the range ends.  The slots of one head belong to consecutive CTAs, and the
-// combine kernel adds them in CTA order, so C is bitwise reproducible.
+// Work unit = (head, 64-token block).  G persistent CTAs take contiguous unit
+// ranges [c U / G, (c + 1) U / G), so every CTA moves the same number of bytes
+// to within one unit and no wave is left partly empty.  A range spans one or
+// more heads; the CTA keeps C and z of the current head in registers and
+// writes them to partial slot c + head when the head changes or the range
+// ends.  The slots of one head belong to consecutive CTAs, and the combine
+// kernel adds them in CTA order, so C is bitwise reproducible on a GPU model.
 //
-// Threads (256 = 8 warps, no producer warp): each unit's k, v (and q)
-// blocks arrive by TMA, one 16 KB [chunk][row][64] box each, in a ring of S
-// stages; the loads of unit i + S - 1 are issued (by lane 0 of warps 0-2, one
-// box each) right after unit i's barrier, when every thread is done with unit
-// i - 1 and its stage is free.  Per unit:
+// A unit is processed as two 32-token halves, each a stage of the TMA ring
+// (k, v and q boxes of 32 x 128, 8 KB each), which keeps a CTA small enough
+// that two fit on an SM for r <= 48 (16 warps per SM hide the latency of the
+// dependent MMA and rotation chains).  Per half, 8 warps:
 //   rotate q, k (thread = token row mod 16 x 8 coordinates), store q^r, k^r,
-//   pool; U = K P_k^T (mma.sync, warp = 16 tokens x half of the r columns);
-//   k~ = R_r SiLU(U) to shared memory; the unit's barrier; block means;
-//   C^T += V^T k~ (warp = 16 of the 128 d columns, all r rows).
-// The rotation, the pooling order and the divisions are those of the
-// stand-alone rotate + pool kernel, so both produce the same bits.
+//   pool into registers; U = K P_k^T (mma.sync; warp = 16 tokens x a quarter
+//   or half of the r columns); k~ = R_r SiLU(U) to shared memory; the half's
+//   barrier; C^T += V^T k~ (warp = 16 of the 128 d columns, all r rows).
+// After the second half the row partials of the pooling are summed into the
+// block means.  The rotation, the pooling order (a thread adds its tokens
+// rs, rs + 16, rs + 32, rs + 48 in that order, then the 16 row partials are
+// added in order) and the divisions are those of the stand-alone rotate +
+// pool kernel, so both produce the same bits.
 //
-// Every wait on an mbarrier is bounded; a wait that gives up records
-// ROLA_ERR_TIMEOUT, the threads agree on it at the unit's barrier (a barrier
-// reduction, so none is left waiting), and the copies still in flight are
-// waited for before the CTA exits.
+// The loads of half-stage i + S - 1 are issued (by lane 0 of warps 0-2, one
+// box each) right after half-stage i's barrier, when every thread is done
+// with half-stage i - 1 and its stage is free.  Every wait on an mbarrier is
+// bounded; a wait that gives up records ROLA_ERR_TIMEOUT, the threads agree on
+// it at the half's barrier (a barrier reduction, so none is left waiting),
+// and the copies still in flight are waited for before the CTA exits.
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -41,28 +45,41 @@ namespace {
 
 using namespace tc;
 
-constexpr int kConsumerWarps = 8;
-constexpr int kConsumers = 32 * kConsumerWarps;
-constexpr int kThreads = kConsumers;
-constexpr uint32_t kBox = 64 * 128 * 2;              // one 64-token block of one tensor
-constexpr int kMaxStages = 4;
+constexpr int kWarps = 8;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kHalfRows = 32;
+constexpr uint32_t kHalf = kHalfRows * 128 * 2;      // one 32-token half of one tensor
+constexpr int kMaxStages = 8;
+
+// Byte offset of 16-byte chunk c (0..15) of row r (0..31) in a 32-row half
+// tile as a [chunk][row][64] TMA box with 128-byte swizzle writes it.
+__device__ __forceinline__ uint32_t hsw(int r, int c)
+{
+    return (c >> 3) * (kHalfRows * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4);
+}
 
 template <int R>
+struct Cfg {
+    static constexpr int NT = R / 8;                             // n-tiles of U
+    static constexpr int NSPLIT = NT % 4 == 0 ? 4 : 2;           // column groups of U
+    static constexpr int NTW = NT / NSPLIT;                      // n-tiles per warp
+    static constexpr int KT = 2 * R + 16;                        // bytes per k~ row (padded)
+    static constexpr int kCtasPerSm = R <= 48 ? 2 : 1;
+};
+
 struct Layout {
-    static constexpr int NT = R / 8;                  // n-tiles of U
-    static constexpr int NTW = NT / 2;                // per warp (two warps share 16 tokens)
-    static constexpr int KT = 2 * R + 16;             // bytes per k~ row (padded against bank conflicts)
     int stages;
     uint32_t stage_bytes, P, kt, part, zsm, bars, total;
-    __host__ __device__ explicit Layout(bool fuse)
+    __host__ __device__ Layout(int R, bool fuse)
     {
-        stages = fuse ? (R <= 64 ? 3 : 2) : 4;
-        stage_bytes = fuse ? 3 * kBox : 2 * kBox;
-        P = stages * stage_bytes;                     // P_k of the current head, r rows x 256 B
-        kt = P + R * 256;                             // k~, two buffers of 64 rows
-        part = kt + 2 * 64 * KT;                      // pooling partials [buf][q|k][16][128] fp32
-        zsm = part + (fuse ? 2 * 2 * 16 * 128 * 4 : 0);
-        bars = zsm + 4 * R * 4;                       // full[kMaxStages], abort
+        const bool two = R <= 48;                                 // two CTAs per SM
+        stages = two ? (fuse ? 3 : 4) : (fuse ? 6 : 8);
+        stage_bytes = fuse ? 3 * kHalf : 2 * kHalf;
+        P = stages * stage_bytes;                                 // P_k of the current head, r rows x 256 B
+        kt = P + R * 256;                                         // k~, two buffers of 32 rows
+        part = kt + 2 * kHalfRows * (2 * R + 16);                 // pooling partials [q|k][16][128] fp32
+        zsm = part + (fuse ? 2 * 16 * 128 * 4 : 0);
+        bars = zsm + 2 * R * 4;                                   // full[kMaxStages], abort
         total = bars + kMaxStages * 8 + 16;
     }
 };
@@ -102,22 +119,28 @@ __device__ __forceinline__ void rotate8(const uint4& w, const float2 (&cs)[4], _
     *reinterpret_cast<uint4*>(dst) = make_uint4(out[0], out[1], out[2], out[3]);
 }
 
+__device__ __forceinline__ uint4 lds128(uint32_t a)
+{
+    uint4 w;
+    asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];\n" : "=r"(w.x), "=r"(w.y), "=r"(w.z), "=r"(w.w) : "r"(a));
+    return w;
+}
+
 // SiLU with the approximate divide (the features enter the MMA in bf16)
 struct SiluFast {
     __device__ float operator()(float x) const { return __fdividef(x, 1.0f + __expf(-x)); }
 };
 
 template <int R>
-__global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_constant__ CUtensorMap map_q,
-                                                              const __grid_constant__ CUtensorMap map_k,
-                                                              const __grid_constant__ CUtensorMap map_v,
-                                                              const Params p)
+__global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
+    const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+    const __grid_constant__ CUtensorMap map_v, const Params p)
 {
-    using L = Layout<R>;
-    constexpr int NTW = L::NTW;
+    using C = Cfg<R>;
+    constexpr int NTW = C::NTW;
     extern __shared__ __align__(1024) uint8_t smem[];
     const bool fuse = p.qr != nullptr;
-    const L lay(fuse);
+    const Layout lay(R, fuse);
     if (smem_u32(smem) & 1023u) {          // the 128-byte swizzle of the TMA boxes needs 1024-byte alignment
         if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
         return;
@@ -133,42 +156,40 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int u0 = (int)((long long)blockIdx.x * p.units / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * p.units / gridDim.x);
-    const int count = u1 - u0;
+    const int count = 2 * (u1 - u0);                // half-stages of this CTA
 
     if (tid == 0) {
         *abort = 0;
         for (int i = 0; i < S; ++i) mbar_init(full0 + 8 * i, 1);
         fence_mbar_init();
-    }
-    __syncthreads();
-
-    // loads of the j-th unit of the range into stage j % S: lane 0 of warps
-    // 0, 1, 2 issue the k, v, q boxes; thread 0 also arms the barrier
-    const uint32_t bytes = fuse ? 3 * kBox : 2 * kBox;
-    auto issue = [&](int j) {
-        const int u = u0 + j, bh = u / s.nB, blk = u - bh * s.nB, st = j % S;
-        const uint32_t dst = sbase + st * lay.stage_bytes, bar = full0 + 8 * st;
-        if (tid == 0) {
-            mbar_expect_tx(bar, bytes);
-            tma_load_4d(dst, &map_k, bar, 0, blk * 64, 0, bh);
-        } else if (tid == 32) {
-            tma_load_4d(dst + kBox, &map_v, bar, 0, blk * 64, 0, bh);
-        } else if (tid == 64 && fuse) {
-            tma_load_4d(dst + 2 * kBox, &map_q, bar, 0, blk * 64, 0, bh);
-        }
-    };
-    if (tid == 0) {
         tma_prefetch_desc(&map_k);
         tma_prefetch_desc(&map_v);
         if (fuse) tma_prefetch_desc(&map_q);
     }
+    __syncthreads();
+
+    // loads of the j-th half-stage of the range into stage j % S: lane 0 of
+    // warps 0, 1, 2 issue the k, v, q boxes; thread 0 also arms the barrier
+    const uint32_t bytes = fuse ? 3 * kHalf : 2 * kHalf;
+    auto issue = [&](int j) {
+        const int u = u0 + (j >> 1), bh = u / s.nB, row = (u - bh * s.nB) * 64 + (j & 1) * kHalfRows;
+        const uint32_t dst = sbase + (j % S) * lay.stage_bytes, bar = full0 + 8 * (j % S);
+        if (tid == 0) {
+            mbar_expect_tx(bar, bytes);
+            tma_load_4d(dst, &map_k, bar, 0, row, 0, bh);
+        } else if (tid == 32) {
+            tma_load_4d(dst + kHalf, &map_v, bar, 0, row, 0, bh);
+        } else if (tid == 64 && fuse) {
+            tma_load_4d(dst + 2 * kHalf, &map_q, bar, 0, row, 0, bh);
+        }
+    };
     int issued = count < S ? count : S;
     for (int j = 0; j < issued; ++j) issue(j);
 
-    // ---------------------------------------------------------------- consumers
     const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
-    const int mt = warp & 3, nh = warp >> 2;        // U: tokens 16 mt .. +15, n-tiles nh * NTW ..
-    const int rs = tid >> 4, c8 = tid & 15;         // rotation: rows rs + 16 j, coordinates 8 c8 .. +7
+    const int mt = warp & 1, cg = warp >> 1;        // U: tokens 16 mt .. +15 of the half, column group cg
+    const bool u_warp = cg < C::NSPLIT;             // (with two column groups, warps 4-7 skip U)
+    const int rs = tid >> 4, c8 = tid & 15;         // rotation: rows rs, rs + 16 of the half; 8 coordinates
     const int hw = s.Hh * s.Ww;
     int axis[4];
 #pragma unroll
@@ -176,11 +197,10 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
         const int m = c8 * 4 + q;
         axis[q] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
     }
-
     int kaxis[NTW];                                 // axis of pair nt * 4 + t4 of each of this warp's n-tiles
 #pragma unroll
     for (int j = 0; j < NTW; ++j) {
-        const int m = (nh * NTW + j) * 4 + t4;
+        const int m = (cg * NTW + j) * 4 + t4;
         kaxis[j] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
     }
     // grid position (t, x, y) of flat token n, and of the token `step` further on
@@ -214,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
 #pragma unroll
         for (int j = 0; j < NTW; ++j) zacc[j][0] = zacc[j][1] = 0.0f;
     };
-    // partial C [r][128] and z [r] of head hb -> slot blockIdx.x + hb
+    // partial C [R][128] and z [R] of head hb -> slot blockIdx.x + hb
     auto flush = [&](int hb) {
         float* dst = p.partials + (size_t)(blockIdx.x + hb) * (size_t)(R * kDh + R);
 #pragma unroll
@@ -234,164 +254,169 @@ __global__ void __launch_bounds__(kThreads, 1) prepass_kernel(const __grid_const
                 x += __shfl_xor_sync(0xffffffffu, x, 4);
                 x += __shfl_xor_sync(0xffffffffu, x, 8);
                 x += __shfl_xor_sync(0xffffffffu, x, 16);
-                if (g == 0) zsm[mt * R + (nh * NTW + j) * 8 + t4 * 2 + e] = x;
+                if (g == 0 && u_warp) zsm[mt * R + (cg * NTW + j) * 8 + t4 * 2 + e] = x;
             }
-        bar_sync(1, kConsumers);
-        if (tid < R) dst[R * kDh + tid] = (zsm[tid] + zsm[R + tid]) + (zsm[2 * R + tid] + zsm[3 * R + tid]);
+        bar_sync(1, kThreads);
+        if (tid < R) dst[R * kDh + tid] = zsm[tid] + zsm[R + tid];
     };
 
     clear();
     int hb = -1;
     bool failed = false;
-    int i = 0;
-    for (int u = u0; u < u1; ++u, ++i) {
+    float accq[8], acck[8];                         // pooling partials of the current block (both halves)
+    int i = 0;                                      // half-stage index
+    for (; i < count; ++i) {
+        const int u = u0 + (i >> 1), h = i & 1;
         const int bh = u / s.nB, blk = u - bh * s.nB;
         const int st = i % S, buf = i & 1;
-        if (bh != hb) {
+        if (h == 0 && bh != hb) {
             if (hb >= 0) {
                 flush(hb);
                 clear();
             }
             // P_k of the new head (every reader of the old one has passed the last barrier)
             const __nv_bfloat16* src = p.Pk + (size_t)(bh % s.H) * s.r * kDh;
-            for (int e = tid; e < R * 16; e += kConsumers) {
+            for (int e = tid; e < R * 16; e += kThreads) {
                 const uint4 w = (e >> 4) < s.r ? __ldg(reinterpret_cast<const uint4*>(src) + e) : make_uint4(0, 0, 0, 0);
                 asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(sP + sw128(e >> 4, e & 15)), "r"(w.x),
                              "r"(w.y), "r"(w.z), "r"(w.w)
                              : "memory");
             }
-            bar_sync(1, kConsumers);
+            bar_sync(1, kThreads);
             hb = bh;
         }
+        if (h == 0) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) accq[e] = acck[e] = 0.0f;
+        }
         const uint32_t stage = sbase + st * lay.stage_bytes;
-        const uint32_t kb = stage, vb = stage + kBox, qb = stage + 2 * kBox;
-        const uint32_t ktb = sKt + buf * (64 * L::KT);
-        const int n_base = blk * kBlock;
+        const uint32_t kb = stage, vb = stage + kHalf, qb = stage + 2 * kHalf;
+        const uint32_t ktb = sKt + buf * (kHalfRows * C::KT);
+        const int n_half = blk * kBlock + h * kHalfRows;          // first token of this half
+        // (cos, sin) of the k~ pairs of this thread's two tokens, needed after U
+        float2 kcs[2][NTW];
+        {
+            int t, x, y;
+            position(n_half + mt * 16 + g, t, x, y);
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+#pragma unroll
+                for (int j = 0; j < NTW; ++j)
+                    kcs[hr][j] = __ldg(p.tab + table_row(kaxis[j], t, x, y) * kPairs + (cg * NTW + j) * 4 + t4);
+                advance(8, t, x, y);
+            }
+        }
+        // (cos, sin) of the rotation's pairs for this thread's two rows
+        float2 cs[2][4];
+        if (fuse) {
+            int t, x, y;
+            position(n_half + rs, t, x, y);
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) cs[j][q] = __ldg(p.tab + table_row(axis[q], t, x, y) * kPairs + c8 * 4 + q);
+                advance(16, t, x, y);
+            }
+        }
         const bool ok = mbar_wait(full0 + 8 * st, (i / S) & 1, abort, s.wait_limit_ns);
         if (ok) {
-            // (cos, sin) of the k~ pairs of this thread's two tokens, needed after U
-            float2 kcs[2][NTW];
-            {
-                int t, x, y;
-                position(n_base + mt * 16 + g, t, x, y);
-#pragma unroll
-                for (int hr = 0; hr < 2; ++hr) {
-#pragma unroll
-                    for (int j = 0; j < NTW; ++j)
-                        kcs[hr][j] = __ldg(p.tab + table_row(kaxis[j], t, x, y) * kPairs + (nh * NTW + j) * 4 + t4);
-                    advance(8, t, x, y);
-                }
-            }
             if (fuse) {
                 // ---- rotate q and k, store q^r and k^r, pool (same order as the stand-alone kernel)
-                float2 cs[4][4];
-                uint4 wq[4], wk[4];
-                {
-                    int t, x, y;
-                    position(n_base + rs, t, x, y);
+                uint4 wq[2], wk[2];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const int tl = rs + 16 * j;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q)
-                            cs[j][q] = __ldg(p.tab + table_row(axis[q], t, x, y) * kPairs + c8 * 4 + q);
-                        asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];\n"
-                                     : "=r"(wq[j].x), "=r"(wq[j].y), "=r"(wq[j].z), "=r"(wq[j].w)
-                                     : "r"(qb + tsw(tl, c8)));
-                        asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];\n"
-                                     : "=r"(wk[j].x), "=r"(wk[j].y), "=r"(wk[j].z), "=r"(wk[j].w)
-                                     : "r"(kb + tsw(tl, c8)));
-                        advance(16, t, x, y);
-                    }
+                for (int j = 0; j < 2; ++j) {
+                    wq[j] = lds128(qb + hsw(rs + 16 * j, c8));
+                    wk[j] = lds128(kb + hsw(rs + 16 * j, c8));
                 }
-                float accq[8], acck[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) accq[e] = acck[e] = 0.0f;
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const int n = n_base + rs + 16 * j;
+                for (int j = 0; j < 2; ++j) {
+                    const int n = n_half + rs + 16 * j;
                     if (n < s.N) {
                         const size_t go = ((size_t)bh * s.N + n) * kDh + c8 * 8;
                         rotate8(wq[j], cs[j], p.qr + go, accq);
                         rotate8(wk[j], cs[j], p.kr + go, acck);
                     }
                 }
-                float* pq = part + ((buf * 2 + 0) * 16 + rs) * kDh + c8 * 8;
-                float* pk = part + ((buf * 2 + 1) * 16 + rs) * kDh + c8 * 8;
-                reinterpret_cast<float4*>(pq)[0] = make_float4(accq[0], accq[1], accq[2], accq[3]);
-                reinterpret_cast<float4*>(pq)[1] = make_float4(accq[4], accq[5], accq[6], accq[7]);
-                reinterpret_cast<float4*>(pk)[0] = make_float4(acck[0], acck[1], acck[2], acck[3]);
-                reinterpret_cast<float4*>(pk)[1] = make_float4(acck[4], acck[5], acck[6], acck[7]);
-            }
-            // ---- U = K P_k^T for tokens 16 mt .. +15 and this warp's n-tiles
-            float uacc[NTW][4];
-#pragma unroll
-            for (int j = 0; j < NTW; ++j) uacc[j][0] = uacc[j][1] = uacc[j][2] = uacc[j][3] = 0.0f;
-#pragma unroll
-            for (int kc = 0; kc < 8; ++kc) {
-                uint32_t a0, a1, a2, a3;
-                ldsm_x4(kb + tsw(mt * 16 + (lane & 7) + (mi & 1) * 8, kc * 2 + (mi >> 1)), a0, a1, a2, a3);
-#pragma unroll
-                for (int np = 0; np < NTW / 2; ++np) {
-                    const int nt = nh * NTW + 2 * np;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(sP + sw128(nt * 8 + (mi >> 1) * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1, b2, b3);
-                    mma_bf16(uacc[2 * np], a0, a1, a2, a3, b0, b1);
-                    mma_bf16(uacc[2 * np + 1], a0, a1, a2, a3, b2, b3);
-                }
-                if (NTW & 1) {
-                    const int nt = nh * NTW + NTW - 1;
-                    uint32_t b0, b1;
-                    ldsm_x2(sP + sw128(nt * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1);
-                    mma_bf16(uacc[NTW - 1], a0, a1, a2, a3, b0, b1);
+                if (h == 1) {
+                    float* pq = part + (0 * 16 + rs) * kDh + c8 * 8;
+                    float* pk = part + (1 * 16 + rs) * kDh + c8 * 8;
+                    reinterpret_cast<float4*>(pq)[0] = make_float4(accq[0], accq[1], accq[2], accq[3]);
+                    reinterpret_cast<float4*>(pq)[1] = make_float4(accq[4], accq[5], accq[6], accq[7]);
+                    reinterpret_cast<float4*>(pk)[0] = make_float4(acck[0], acck[1], acck[2], acck[3]);
+                    reinterpret_cast<float4*>(pk)[1] = make_float4(acck[4], acck[5], acck[6], acck[7]);
                 }
             }
-            // ---- k~ = R_r SiLU(U); tokens past N contribute nothing
+            if (u_warp) {
+                // ---- U = K P_k^T for tokens 16 mt .. +15 of the half and this warp's n-tiles
+                float uacc[NTW][4];
 #pragma unroll
-            for (int hr = 0; hr < 2; ++hr) {
-                const int tl = mt * 16 + g + hr * 8, n = n_base + tl;
-                const bool valid = n < s.N;
+                for (int j = 0; j < NTW; ++j) uacc[j][0] = uacc[j][1] = uacc[j][2] = uacc[j][3] = 0.0f;
 #pragma unroll
-                for (int j = 0; j < NTW; ++j) {
-                    const int nt = nh * NTW + j;
-                    const float2 cs = valid ? kcs[hr][j] : make_float2(0.0f, 0.0f);
-                    const float2 y = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], cs, s.lr_rope, SiluFast{});
-                    zacc[j][0] += y.x;
-                    zacc[j][1] += y.y;
-                    asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(ktb + tl * L::KT + (nt * 8 + t4 * 2) * 2),
-                                 "r"(pack_bf16(y.x, y.y))
-                                 : "memory");
+                for (int kc = 0; kc < 8; ++kc) {
+                    uint32_t a0, a1, a2, a3;
+                    ldsm_x4(kb + hsw(mt * 16 + (lane & 7) + (mi & 1) * 8, kc * 2 + (mi >> 1)), a0, a1, a2, a3);
+#pragma unroll
+                    for (int np = 0; np < NTW / 2; ++np) {
+                        const int nt = cg * NTW + 2 * np;
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4(sP + sw128(nt * 8 + (mi >> 1) * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1, b2, b3);
+                        mma_bf16(uacc[2 * np], a0, a1, a2, a3, b0, b1);
+                        mma_bf16(uacc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+                    }
+                    if (NTW & 1) {
+                        const int nt = cg * NTW + NTW - 1;
+                        uint32_t b0, b1;
+                        ldsm_x2(sP + sw128(nt * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1);
+                        mma_bf16(uacc[NTW - 1], a0, a1, a2, a3, b0, b1);
+                    }
+                }
+                // ---- k~ = R_r SiLU(U) (or the placement cfg selects); tokens past N contribute nothing
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    const int tl = mt * 16 + g + hr * 8, n = n_half + tl;
+                    const bool valid = n < s.N;
+#pragma unroll
+                    for (int j = 0; j < NTW; ++j) {
+                        const int nt = cg * NTW + j;
+                        const float2 cs2 = valid ? kcs[hr][j] : make_float2(0.0f, 0.0f);
+                        const float2 y = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], cs2, s.lr_rope, SiluFast{});
+                        zacc[j][0] += y.x;
+                        zacc[j][1] += y.y;
+                        asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(ktb + tl * C::KT + (nt * 8 + t4 * 2) * 2),
+                                     "r"(pack_bf16(y.x, y.y))
+                                     : "memory");
+                    }
                 }
             }
         }
-        // every thread reaches this barrier once per unit; it also settles a timeout
-        if (bar_red_or(1, kConsumers, !ok)) {
+        // every thread reaches this barrier once per half; it also settles a timeout
+        if (bar_red_or(1, kThreads, !ok)) {
             failed = true;
             break;
         }
-        if (i >= 1 && issued < count) {       // unit i - 1 is done everywhere: refill its stage
+        if (i >= 1 && issued < count) {       // half-stage i - 1 is done everywhere: refill its stage
             issue(issued);
             ++issued;
         }
-        if (fuse) {
+        if (fuse && h == 1) {
             // ---- block means: threads 0-127 q, 128-255 k; 16 row partials in order
             const int which = tid >> 7, d = tid & 127;
-            const float* src = part + ((buf * 2 + which) * 16) * kDh + d;
+            const float* src = part + (which * 16) * kDh + d;
             float sum = 0.0f;
 #pragma unroll
             for (int r = 0; r < 16; ++r) sum += src[r * kDh];
-            const int cnt = min(kBlock, s.N - n_base);
+            const int cnt = min(kBlock, s.N - blk * kBlock);
             (which ? p.kbar : p.qbar)[((size_t)bh * s.nB + blk) * kDh + d] = sum / (float)cnt;
         }
-        // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 64 tokens
+        // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 32 tokens
 #pragma unroll
-        for (int kc = 0; kc < kBlock / 16; ++kc) {
+        for (int kc = 0; kc < kHalfRows / 16; ++kc) {
             uint32_t b0, b1, b2, b3;
-            ldsm_x4_t(vb + tsw(kc * 16 + (mi & 1) * 8 + (lane & 7), warp * 2 + (mi >> 1)), b0, b1, b2, b3);
+            ldsm_x4_t(vb + hsw(kc * 16 + (mi & 1) * 8 + (lane & 7), warp * 2 + (mi >> 1)), b0, b1, b2, b3);
 #pragma unroll
             for (int a = 0; a < R / 16; ++a) {
                 uint32_t a0, a1, a2, a3;
-                ldsm_x4_t(ktb + (kc * 16 + (mi >> 1) * 8 + (lane & 7)) * L::KT + (a * 2 + (mi & 1)) * 16, a0, a1, a2,
+                ldsm_x4_t(ktb + (kc * 16 + (mi >> 1) * 8 + (lane & 7)) * C::KT + (a * 2 + (mi & 1)) * 16, a0, a1, a2,
                           a3);
                 mma_bf16(cacc[a][0], a0, a1, a2, a3, b0, b1);
                 mma_bf16(cacc[a][1], a0, a1, a2, a3, b2, b3);
@@ -435,7 +460,7 @@ template <int R>
 cudaError_t launch_r(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv, const Params& p, int ctas,
                      bool fuse, cudaStream_t st)
 {
-    const Layout<R> lay(fuse);
+    const Layout lay(R, fuse);
     cudaError_t e = cudaFuncSetAttribute(prepass_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)lay.total);
     if (e != cudaSuccess) return e;
@@ -452,7 +477,7 @@ int prepass_ctas(const Shape& s, int max_ctas)
                                                    cudaSuccess)
         return 0;
     const long long units = (long long)s.B * s.H * s.nB;
-    long long g = nsm;
+    long long g = (long long)nsm * (s.rp <= 48 ? 2 : 1);     // CTAs per SM as Cfg<R>::kCtasPerSm
     if (g > max_ctas) g = max_ctas;
     if (g > kMaxPrepassCtas) g = kMaxPrepassCtas;
     if (g > units) g = units;
@@ -466,9 +491,9 @@ cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* 
     if (ctas <= 0 || ctas > kMaxPrepassCtas || ctas > s.B * s.H * s.nB) return cudaErrorInvalidValue;
     const bool fuse = q != nullptr;
     CUtensorMap mq, mk, mv;
-    if (!make_block_map(&mk, k, s) || !make_block_map(&mv, v, s)) return cudaErrorInvalidValue;
+    if (!make_block_map(&mk, k, s, kHalfRows) || !make_block_map(&mv, v, s, kHalfRows)) return cudaErrorInvalidValue;
     if (fuse) {
-        if (!make_block_map(&mq, q, s)) return cudaErrorInvalidValue;
+        if (!make_block_map(&mq, q, s, kHalfRows)) return cudaErrorInvalidValue;
     } else {
         mq = mk;
     }

@@ -331,8 +331,12 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
                            cudaStream_t st)
 {
     const int units = s.B * s.H * s.nB;
-    const int ctas = prepass_ctas(s, kMaxPrepassCtas);
-    if (ctas <= 0) return cudaErrorInvalidValue;
+    int dev = 0, nsm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int ctas = units < nsm ? units : nsm;             // one CTA per SM
     CUtensorMap mq, mos, mo;
     if (!make_block_map(&mq, q, s) || !make_block_map(&mos, o_s, s) || !make_block_map(&mo, o, s))
         return cudaErrorInvalidValue;

@@ -570,13 +570,13 @@ bool make_chunk_map(CUtensorMap* m, const void* ptr, const Shape& s)
 // The same tensor viewed as 4-D (d within chunk, token, d-chunk, head) so that
 // one 64 x 64 x 2 box brings a whole key block in as [chunk][row][64]: 16 KB,
 // 128-byte swizzle, rows past N read as zero.
-bool make_block_map(CUtensorMap* m, const void* ptr, const Shape& s)
+bool make_block_map(CUtensorMap* m, const void* ptr, const Shape& s, int rows)
 {
     auto enc = encode_fn();
     if (!enc) return false;
     cuuint64_t dims[4] = {64, (cuuint64_t)s.N, 2, (cuuint64_t)s.B * s.H};
     cuuint64_t strides[3] = {(cuuint64_t)kDh * 2, 128, (cuuint64_t)s.N * kDh * 2};
-    cuuint32_t box[4] = {64, 64, 2, 1};
+    cuuint32_t box[4] = {64, (cuuint32_t)rows, 2, 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
