@@ -263,6 +263,15 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     clear();
     int hb = -1;
     bool failed = false;
+    // grid positions of this thread's first k~ token and first rotation row in
+    // the current half; carried 32 tokens forward per half (a division only at
+    // the start of the range, since consecutive units are consecutive blocks)
+    int kt_t, kt_x, kt_y, rt_t, rt_x, rt_y;
+    {
+        const int blk0 = u0 - (u0 / s.nB) * s.nB;
+        position(blk0 * kBlock + mt * 16 + g, kt_t, kt_x, kt_y);
+        position(blk0 * kBlock + rs, rt_t, rt_x, rt_y);
+    }
     float accq[8], acck[8];                         // pooling partials of the current block (both halves)
     int i = 0;                                      // half-stage index
     for (; i < count; ++i) {
@@ -283,6 +292,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
                              : "memory");
             }
             bar_sync(1, kThreads);
+            if (hb >= 0) {                         // a new head starts at its block 0
+                position(mt * 16 + g, kt_t, kt_x, kt_y);
+                position(rs, rt_t, rt_x, rt_y);
+            }
             hb = bh;
         }
         if (h == 0) {
@@ -296,8 +309,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
         // (cos, sin) of the k~ pairs of this thread's two tokens, needed after U
         float2 kcs[2][NTW];
         {
-            int t, x, y;
-            position(n_half + mt * 16 + g, t, x, y);
+            int t = kt_t, x = kt_x, y = kt_y;
 #pragma unroll
             for (int hr = 0; hr < 2; ++hr) {
 #pragma unroll
@@ -309,8 +321,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
         // (cos, sin) of the rotation's pairs for this thread's two rows
         float2 cs[2][4];
         if (fuse) {
-            int t, x, y;
-            position(n_half + rs, t, x, y);
+            int t = rt_t, x = rt_x, y = rt_y;
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
 #pragma unroll
@@ -318,6 +329,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
                 advance(16, t, x, y);
             }
         }
+        advance(kHalfRows, kt_t, kt_x, kt_y);          // the next half's positions
+        advance(kHalfRows, rt_t, rt_x, rt_y);
         const bool ok = mbar_wait(full0 + 8 * st, (i / S) & 1, abort, s.wait_limit_ns);
         if (ok) {
             if (fuse) {
