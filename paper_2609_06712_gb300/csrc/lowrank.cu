@@ -1,5 +1,6 @@
-// Low-rank branch: the fp32 summary of the validation mode (the bf16 summary
-// is part of the pre-pass, prepass.cu) and readout + gated fusion (kernel 4).
+// Low-rank branch of the fp32 validation mode: the summary (kernel 3) and the
+// readout + gated fusion (kernel 4).  The bf16 path has them in prepass.cu and
+// readout.cu.
 //
 // Eq. (qklr):  k~_q = R_r(q) SiLU(P_k k^n_q),   q~_p = R_r(p) SiLU(P_q q^n_p)
 // Eq. (ctx):   C = sum_q k~_q v_q^T,            O^lr_p = RMSNorm(q~_p^T C)   (no gain)
@@ -14,16 +15,11 @@
 
 namespace rola {
 
-// SiLU evaluations: IEEE exp and divide (fp32 validation mode) and the
-// MUFU-based one of the bf16 readout
+// SiLU with the IEEE exp and divide (fp32 validation mode)
 struct SiluIeee {
     __device__ float operator()(float x) const { return x / (1.0f + expf(-x)); }
 };
-struct SiluMufu {
-    __device__ float operator()(float x) const { return silu(x); }
-};
 __device__ constexpr SiluIeee silu_ieee{};
-__device__ constexpr SiluMufu silu_mufu{};
 
 // ===========================================================================
 // Split-N partitioning of the fp32 summary: CTA = (split, head).
@@ -40,16 +36,6 @@ int summary_splits(const Shape& s)
     return (tiles + per - 1) / per;
 }
 
-__device__ __forceinline__ void load_rows_async(uint32_t sbase, const __nv_bfloat16* g, int row0, int nrows,
-                                                int limit, int tid, int nthreads)
-{
-    for (int e = tid; e < nrows * 16; e += nthreads) {
-        int r = e >> 4, c = e & 15;
-        int n = row0 + r;
-        const __nv_bfloat16* src = g + (size_t)min(n, limit - 1) * kDh + c * 8;
-        cp_async16(sbase + sw128(r, c), src, n < limit ? 16 : 0);
-    }
-}
 
 // ===========================================================================
 // summary, fp32 validation mode: CTA = (split, head), 256 threads, 64-token tiles.
@@ -173,127 +159,6 @@ cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, 
 }
 
 // ===========================================================================
-// apply, bf16: CTA = (64-token block, head), 4 warps x 16 tokens.
-//   U = Q P_q^T -> q~ = R_r SiLU(U) (registers, never stored) -> y = q~ C (MMA,
-//   C in bf16) -> O^lr = y / sqrt(mean y^2 + eps_lr) -> fuse with O^s.
-// Shared memory: P_q r x 256 B | C r x 256 B | Q 16 KB | O^s 16 KB, all 256-byte
-// rows, swizzled.  O^s comes in and O goes out through the shared tile with
-// 16-byte accesses.
-
-template <int R>
-__global__ void __launch_bounds__(128, 4) apply_bf16_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
-                                                         const __nv_bfloat16* __restrict__ Pq,
-                                                         const __nv_bfloat16* __restrict__ Cbf,
-                                                         const float* __restrict__ gate,
-                                                         const __nv_bfloat16* o_s, __nv_bfloat16* o,
-                                                         const float2* __restrict__ tab)
-{
-    extern __shared__ __align__(128) uint8_t smem[];
-    constexpr int NT = R / 8;
-    const int blk = blockIdx.x, bh = blockIdx.y, h = bh % s.H, b = bh / s.H;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t4 = lane & 3;
-    const uint32_t sP = smem_u32(smem);
-    const uint32_t sC = sP + R * 256;
-    const uint32_t sQ = sC + R * 256;
-    const uint32_t sO = sQ + kBlock * 256;
-    uint8_t* o_gen = smem + 2 * R * 256 + kBlock * 256;
-    const size_t head = (size_t)bh * s.N * kDh;
-    load_rows_async(sP, Pq + (size_t)h * s.r * kDh, 0, R, s.r, tid, 128);     // rows past r read as zero
-    load_rows_async(sC, Cbf + (size_t)bh * R * kDh, 0, R, R, tid, 128);       // rp rows, zero-padded
-    load_rows_async(sQ, q + head, blk * kBlock, kBlock, s.N, tid, 128);
-    load_rows_async(sO, o_s + head, blk * kBlock, kBlock, s.N, tid, 128);
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-    const int mi = lane >> 3;
-    float u[NT][4];
-#pragma unroll
-    for (int a = 0; a < NT; ++a) u[a][0] = u[a][1] = u[a][2] = u[a][3] = 0.0f;
-#pragma unroll
-    for (int kc = 0; kc < 8; ++kc) {
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4(sQ + sw128(warp * 16 + (lane & 7) + (mi & 1) * 8, kc * 2 + (mi >> 1)), a0, a1, a2, a3);
-#pragma unroll
-        for (int np = 0; np < NT / 2; ++np) {
-            uint32_t b0, b1, b2, b3;
-            ldsm_x4(sP + sw128(np * 16 + (mi >> 1) * 8 + (lane & 7), kc * 2 + (mi & 1)), b0, b1, b2, b3);
-            mma_bf16(u[2 * np], a0, a1, a2, a3, b0, b1);
-            mma_bf16(u[2 * np + 1], a0, a1, a2, a3, b2, b3);
-        }
-    }
-    const int n_lo = blk * kBlock + warp * 16 + g, n_hi = n_lo + 8;
-    const int n_lo_c = min(n_lo, s.N - 1), n_hi_c = min(n_hi, s.N - 1);
-    uint32_t qf[NT][2];
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-        const int m = nt * 4 + t4;
-        float2 c0 = rope_cs(tab, s, n_lo_c, m), c1 = rope_cs(tab, s, n_hi_c, m);
-        const float2 f0 = lowrank_pair(u[nt][0], u[nt][1], c0, s.lr_rope, silu_mufu);
-        const float2 f1 = lowrank_pair(u[nt][2], u[nt][3], c1, s.lr_rope, silu_mufu);
-        qf[nt][0] = pack_bf16(f0.x, f0.y);
-        qf[nt][1] = pack_bf16(f1.x, f1.y);
-    }
-    float y[16][4];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) y[i][0] = y[i][1] = y[i][2] = y[i][3] = 0.0f;
-#pragma unroll
-    for (int kc = 0; kc < R / 16; ++kc) {
-#pragma unroll
-        for (int dp = 0; dp < 8; ++dp) {
-            uint32_t b0, b1, b2, b3;
-            ldsm_x4_t(sC + sw128(kc * 16 + (mi & 1) * 8 + (lane & 7), dp * 2 + (mi >> 1)), b0, b1, b2, b3);
-            mma_bf16(y[2 * dp], qf[2 * kc][0], qf[2 * kc][1], qf[2 * kc + 1][0], qf[2 * kc + 1][1], b0, b1);
-            mma_bf16(y[2 * dp + 1], qf[2 * kc][0], qf[2 * kc][1], qf[2 * kc + 1][0], qf[2 * kc + 1][1], b2, b3);
-        }
-    }
-    // per-row RMS of y and of O^s (the 4 lanes of a quad share a row); O^s stays
-    // in shared memory and is read again for the fusion
-    const int r_lo = warp * 16 + g, r_hi = r_lo + 8;                 // rows within the tile
-    float ssy[2] = {0.0f, 0.0f}, sso[2] = {0.0f, 0.0f};
-#pragma unroll
-    for (int dt = 0; dt < 16; ++dt) {
-        const uint32_t lo_off = sw128(r_lo, dt) + t4 * 4, hi_off = sw128(r_hi, dt) + t4 * 4;
-        float2 lo = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + lo_off));
-        float2 hi = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_gen + hi_off));
-        ssy[0] += y[dt][0] * y[dt][0] + y[dt][1] * y[dt][1];
-        ssy[1] += y[dt][2] * y[dt][2] + y[dt][3] * y[dt][3];
-        sso[0] += lo.x * lo.x + lo.y * lo.y;
-        sso[1] += hi.x * hi.x + hi.y * hi.y;
-    }
-    float coef[2];
-#pragma unroll
-    for (int hr = 0; hr < 2; ++hr) {
-        ssy[hr] += __shfl_xor_sync(0xffffffffu, ssy[hr], 1);
-        ssy[hr] += __shfl_xor_sync(0xffffffffu, ssy[hr], 2);
-        sso[hr] += __shfl_xor_sync(0xffffffffu, sso[hr], 1);
-        sso[hr] += __shfl_xor_sync(0xffffffffu, sso[hr], 2);
-        int n = hr ? n_hi_c : n_lo_c;
-        float gp = gate ? __ldg(gate + (size_t)b * s.N + n) : s.default_gate;
-        float rp = sqrtf(sso[hr] * (1.0f / kDh) + s.eps_fuse);
-        coef[hr] = gp * rp * rsqrtf(ssy[hr] * (1.0f / kDh) + s.eps_lr);
-    }
-    // fused rows back into the shared tile (each thread rewrites what it read), then 16-byte stores
-#pragma unroll
-    for (int dt = 0; dt < 16; ++dt) {
-        uint32_t* lo_p = reinterpret_cast<uint32_t*>(o_gen + sw128(r_lo, dt) + t4 * 4);
-        uint32_t* hi_p = reinterpret_cast<uint32_t*>(o_gen + sw128(r_hi, dt) + t4 * 4);
-        const float2 lo = unpack_bf16(*lo_p), hi = unpack_bf16(*hi_p);
-        *lo_p = pack_bf16(lo.x + coef[0] * y[dt][0], lo.y + coef[0] * y[dt][1]);
-        *hi_p = pack_bf16(hi.x + coef[1] * y[dt][2], hi.y + coef[1] * y[dt][3]);
-    }
-    __syncthreads();
-#pragma unroll
-    for (int it = 0; it < 8; ++it) {
-        const int e = it * 128 + tid;
-        const int row = e >> 4, c = e & 15;
-        const int n = blk * kBlock + row;
-        if (n < s.N)
-            *reinterpret_cast<uint4*>(o + head + (size_t)n * kDh + c * 8) =
-                *reinterpret_cast<const uint4*>(o_gen + sw128(row, c));
-    }
-}
-
-// ===========================================================================
 // apply, fp32 validation mode: CTA = (64-token block, head), 256 threads.
 
 __global__ void __launch_bounds__(256) apply_f32_kernel(Shape s, const float* __restrict__ q,
@@ -358,33 +223,11 @@ __global__ void __launch_bounds__(256) apply_f32_kernel(Shape s, const float* __
         for (int i = 0; i < 32; ++i) o[head + (size_t)n * kDh + quarter + 4 * i] = os[i] + coef * y[i];
 }
 
-template <int R>
-static cudaError_t launch_apply_bf16_r(const Shape& s, const void* q, const void* P_q, const __nv_bfloat16* Cbf,
-                                       const float* gate, const void* o_s, void* o, const float2* tab, cudaStream_t st)
-{
-    size_t smem = (size_t)R * 512 + 2 * kBlock * 256;
-    cudaError_t e = cudaFuncSetAttribute(apply_bf16_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    apply_bf16_kernel<R><<<dim3(s.nB, s.B * s.H), 128, smem, st>>>(
-        s, (const __nv_bfloat16*)q, (const __nv_bfloat16*)P_q, Cbf, gate, (const __nv_bfloat16*)o_s,
-        (__nv_bfloat16*)o, tab);
-    return cudaGetLastError();
-}
-
 cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q, const void* P_q, const float* C,
                                  const __nv_bfloat16* Cbf, const float* gate, const void* o_s, void* o,
                                  const float2* tab, DeviceStatus* status, cudaStream_t st)
 {
-    if (dt == ROLA_BF16) {
-        // small r: one CTA per block, four per SM (P_q and C re-read from L2 are cheap);
-        // large r: the persistent kernel, which loads P_q and C once per head
-        switch (s.rp) {
-            case 16: return launch_apply_bf16_r<16>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 32: return launch_apply_bf16_r<32>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            case 48: return launch_apply_bf16_r<48>(s, q, P_q, Cbf, gate, o_s, o, tab, st);
-            default: return launch_readout(s, q, P_q, Cbf, gate, o_s, o, tab, status, st);
-        }
-    }
+    if (dt == ROLA_BF16) return launch_readout(s, q, P_q, Cbf, gate, o_s, o, tab, status, st);
     size_t smem = sizeof(float) * ((size_t)s.r * (kDh + 1) + (size_t)s.r * kDh + kBlock * (kDh + 1) +
                                    kBlock * (s.r + 1));
     cudaError_t e = cudaFuncSetAttribute(apply_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -4,7 +4,8 @@
 //   r_p    = sqrt(mean_i (O^s_{p,i})^2 + eps_fuse)
 //   O_p    = O^s_p + g_p r_p O^lr_p                     Eq. (gate), (O^s/r_p + g O^lr) r_p
 //
-// Work unit = (head, 64-token block); G persistent CTAs (one per SM) take
+// Work unit = (head, 64-token block); G persistent CTAs (two per SM for
+// r <= 48, else one) take
 // contiguous unit ranges, so P_q and C (bf16) are loaded once per head a CTA
 // meets instead of once per block.  Each unit's q and O^s blocks arrive by TMA
 // (one 16 KB [chunk][row][64] box each) in a ring of stages; the fused O is
@@ -31,7 +32,15 @@ using namespace tc;
 constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr uint32_t kBox = 64 * 128 * 2;
-constexpr int kStages = 4;
+constexpr int kMaxStages = 4;
+
+// r <= 48: two CTAs per SM (16 warps) with a 2-deep ring; wider r: one CTA
+// with a 4-deep ring (P_q and C take more shared memory and registers)
+template <int R>
+struct Occupancy {
+    static constexpr int ctas = R <= 48 ? 2 : 1;
+    static constexpr int stages = R <= 48 ? 2 : 4;
+};
 
 template <int R>
 struct Layout {
@@ -39,12 +48,12 @@ struct Layout {
     static constexpr int NTW = NT / 2;               // n-tiles of U per warp
     static constexpr int QT = 2 * R + 16;            // bytes per q~ row (padded against bank conflicts)
     static constexpr uint32_t stage_bytes = 2 * kBox;   // q | O^s
-    static constexpr uint32_t P = kStages * stage_bytes;
+    static constexpr uint32_t P = Occupancy<R>::stages * stage_bytes;
     static constexpr uint32_t C = P + R * 256;
     static constexpr uint32_t qt = C + R * 256;
     static constexpr uint32_t red = qt + 64 * QT;    // [y^2 | O^s^2][half][64 rows] fp32
     static constexpr uint32_t bars = red + 2 * 2 * 64 * 4;
-    static constexpr uint32_t total = bars + kStages * 8 + 16;
+    static constexpr uint32_t total = bars + kMaxStages * 8 + 16;
 };
 
 struct Params {
@@ -62,13 +71,14 @@ struct SiluMufu {
 };
 
 template <int R>
-__global__ void __launch_bounds__(kThreads, 1) readout_kernel(const __grid_constant__ CUtensorMap map_q,
+__global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(const __grid_constant__ CUtensorMap map_q,
                                                               const __grid_constant__ CUtensorMap map_os,
                                                               const __grid_constant__ CUtensorMap map_o,
                                                               const Params p)
 {
     using L = Layout<R>;
     constexpr int NTW = L::NTW;
+    constexpr int kStages = Occupancy<R>::stages;
     extern __shared__ __align__(1024) uint8_t smem[];
     if (smem_u32(smem) & 1023u) {
         if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
@@ -78,7 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1) readout_kernel(const __grid_const
     const uint32_t sbase = smem_u32(smem), sP = sbase + L::P, sC = sbase + L::C, sQt = sbase + L::qt;
     float* red = reinterpret_cast<float*>(smem + L::red);
     const uint32_t full0 = sbase + L::bars;
-    volatile int* abort = reinterpret_cast<volatile int*>(smem + L::bars + kStages * 8);
+    volatile int* abort = reinterpret_cast<volatile int*>(smem + L::bars + kMaxStages * 8);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
     const int mt = warp & 3, half = warp >> 2;
@@ -336,7 +346,8 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    const int ctas = units < nsm ? units : nsm;             // one CTA per SM
+    const int per_sm = s.rp <= 48 ? 2 : 1;                   // Occupancy<R>::ctas
+    const int ctas = units < nsm * per_sm ? units : nsm * per_sm;
     CUtensorMap mq, mos, mo;
     if (!make_block_map(&mq, q, s) || !make_block_map(&mos, o_s, s) || !make_block_map(&mo, o, s))
         return cudaErrorInvalidValue;
