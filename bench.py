@@ -232,6 +232,47 @@ def run_reference(args, cfg, ws, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank):
+    """Times one per-stage entry point of the C ABI on the layer (inputs resident in HBM)."""
+    import torch
+    from paper_2609_06712_gb300 import rola
+    C = torch.empty((cfg["B"], cfg["H"], cfg["r"], 128), dtype=torch.float32, device=o.device)
+    rola.forward(c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kv, wsb)    # a mask and O^s to use
+    tensor_bytes = 2.0 * cfg["B"] * cfg["H"] * cfg["N"] * 128
+    calls = {
+        "mask": (lambda: rola.block_mask(c, x["q"], x["k"], kv, wsb), 4 * tensor_bytes,
+                 "read q, k; write q^r, k^r (rotate + pool), then scores and top-k"),
+        "summary": (lambda: rola.lowrank_summary(c, x["k"], x["v"], x["P_k"], C, None, wsb), 2 * tensor_bytes,
+                    "read k, v"),
+        "sparse": (lambda: rola.sparse_attn(c, x["q"], x["k"], x["v"], kv, o, wsb), 6 * tensor_bytes,
+                   "rotate q, k (read q, k; write q^r, k^r), then the sparse kernel (read q^r, k^r, v; write O^s)"),
+        "apply": (lambda: rola.lowrank_apply(c, x["q"], x["P_q"], C, x["gate"], o, o, wsb), 3 * tensor_bytes,
+                  "read q, O^s; write O"),
+    }
+    fn, nbytes, what = calls[args.entry]
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    barrier(ws)
+    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        fn()
+    z.record(stream)
+    torch.cuda.synchronize()
+    ms = reduce_max(a.elapsed_time(z) / args.steps, ws)
+    assert rola.get_device_status(wsb) == rola.ROLA_OK
+    if rank == 0:
+        peaks, src = load_peaks()
+        hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+        names = {"mask": "rola_block_mask", "summary": "rola_lowrank_summary", "sparse": "rola_sparse_attn",
+                 "apply": "rola_lowrank_apply"}
+        print(json.dumps({"entry": names[args.entry], "ms_per_call": ms, "unit": "ms", "steps": args.steps, "warmup": args.warmup,
+                          "bytes_per_call": nbytes, "achieved_gbs": nbytes / (ms * 1e-3) / 1e9, "hbm_peak_gbs": hbm,
+                          "note": what, "config": {"workload": cfg["name"], "H": cfg["H"], "N": cfg["N"],
+                                                   "r": cfg["r"], "keep": cfg["keep"]}}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -244,6 +285,8 @@ def main():
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--entry", default="forward", choices=["forward", "mask", "summary", "sparse", "apply"],
+                    help="time one per-stage entry point alone instead of the layer")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -282,6 +325,9 @@ def main():
         for e in row:
             e.record(stream)
     args_fw = (c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kv, wsb)
+    if args.entry != "forward":
+        run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank)
+        return
 
     for _ in range(args.warmup):
         rola.forward(*args_fw)
