@@ -280,9 +280,14 @@ def test_forward_layer_shapes_sampled(rl, name, r, keep, nsample):
     nB = (cfg["N"] + 63) // 64
     blocks = sample_blocks(nB, nsample, seed=cfg["seed"])
     res = compare_forward(cfg, x, h, out, kv, "bf16", qblocks=blocks)
-    # the summary in full
     c = rl.make_config(cfg)
     ws = rl.workspace(c)
+    # the fused pre-pass and the stand-alone rotate + pool give the same mask, bit for bit, in full
+    kv2 = torch.empty_like(kv)
+    rl.block_mask(c, dev(x["q"]), dev(x["k"]), kv2, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(kv, kv2)
+    # the summary in full
     C = torch.empty((cfg["B"], cfg["H"], cfg["r"], 128), dtype=torch.float32, device="cuda")
     rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, None, ws)
     torch.cuda.synchronize()
