@@ -14,8 +14,9 @@ namespace rola {
 // tile per CTA, 256 threads with 8 x 8 register tiles (rows ty + 16 u, columns
 // tx + 16 w), d staged through shared memory in chunks of 16, transposed and
 // double-buffered: the next chunk's global loads are in flight while the
-// current chunk is multiplied.  Every score is the same ascending-d FMA chain
-// whatever the tiling.
+// current chunk is multiplied.  Two neighbouring columns go through one packed
+// fma.rn.f32x2 (each element an IEEE fma), so every score is the same
+// ascending-d fp32 FMA chain whatever the tiling.
 
 constexpr int kSTile = 128, kSChunk = 16;
 
@@ -72,7 +73,15 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
 #pragma unroll
             for (int u = 0; u < 8; ++u)
 #pragma unroll
-                for (int w = 0; w < 8; ++w) acc[u][w] = fmaf(av[u], bv[w], acc[u][w]);
+                for (int w = 0; w < 8; w += 2)
+                    asm("{\n.reg .b64 ra, rb, rc;\n"
+                        "mov.b64 ra, {%2, %2};\n"
+                        "mov.b64 rb, {%3, %4};\n"
+                        "mov.b64 rc, {%0, %1};\n"
+                        "fma.rn.f32x2 rc, ra, rb, rc;\n"
+                        "mov.b64 {%0, %1}, rc;\n}\n"
+                        : "+f"(acc[u][w]), "+f"(acc[u][w + 1])
+                        : "f"(av[u]), "f"(bv[w]), "f"(bv[w + 1]));
         }
         // the other buffer was last read in chunk c - 1, before the previous barrier
         if (c + 1 < kDh / kSChunk) stash(buf ^ 1);

@@ -148,6 +148,22 @@ __device__ __forceinline__ void column_reduce(float (&v)[kCols], Smem& sm, int w
     bar_sync(1 + wg, kWGThreads);
 }
 
+// Two neighbouring query columns in one packed f32x2 instruction (each element
+// an IEEE fma / add, so the results are those of the scalar forms):
+// (a, b) = (a * m0 + c0, b * m1 + c1) and (a, b) += (p, q)
+__device__ __forceinline__ void ffma2(float& a, float& b, float m0, float m1, float c0, float c1)
+{
+    asm("{\n.reg .b64 ra, rm, rc;\nmov.b64 ra, {%0, %1};\nmov.b64 rm, {%2, %3};\nmov.b64 rc, {%4, %5};\n"
+        "fma.rn.f32x2 ra, ra, rm, rc;\nmov.b64 {%0, %1}, ra;\n}\n"
+        : "+f"(a), "+f"(b) : "f"(m0), "f"(m1), "f"(c0), "f"(c1));
+}
+__device__ __forceinline__ void fadd2(float& a, float& b, float p, float q)
+{
+    asm("{\n.reg .b64 ra, rp;\nmov.b64 ra, {%0, %1};\nmov.b64 rp, {%2, %3};\n"
+        "add.rn.f32x2 ra, ra, rp;\nmov.b64 {%0, %1}, ra;\n}\n"
+        : "+f"(a), "+f"(b) : "f"(p), "f"(q));
+}
+
 template <int NC>
 __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[NC])
 {
@@ -429,10 +445,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
 #pragma unroll
                     for (int q = 0; q < kCols; q += 4) {
                         const float4 nm = *reinterpret_cast<const float4*>(&sm.m[col0 + q]);
-                        x[q] = fmaf(x[q], c_log2, nm.x);
-                        x[q + 1] = fmaf(x[q + 1], c_log2, nm.y);
-                        x[q + 2] = fmaf(x[q + 2], c_log2, nm.z);
-                        x[q + 3] = fmaf(x[q + 3], c_log2, nm.w);
+                        ffma2(x[q], x[q + 1], c_log2, c_log2, nm.x, nm.y);
+                        ffma2(x[q + 2], x[q + 3], c_log2, c_log2, nm.z, nm.w);
                         need |= (x[q] > kRescaleThreshold) | (x[q + 1] > kRescaleThreshold) |
                                 (x[q + 2] > kRescaleThreshold) | (x[q + 3] > kRescaleThreshold);
                     }
@@ -488,8 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 for (int q = 0; q < kCols; q += 2) {
                     const float p0 = fast_exp2(x[q]);
                     const float p1 = fast_exp2(x[q + 1]);
-                    l[q] += p0;
-                    l[q + 1] += p1;
+                    fadd2(l[q], l[q + 1], p0, p1);
                     pk[q >> 1] = pack_bf16(p0, p1);
                 }
                 if (g >= 2 && !(ok = mbar_wait(bar(PV_DONE + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns))) break;
