@@ -8,7 +8,7 @@ using namespace rola;
 
 namespace rola {
 
-int num_blocks_of(const rola_config_t& c) { return (c.N + c.block - 1) / c.block; }
+int num_blocks_of(const rola_config_t& c) { return (int)(((int64_t)c.N + c.block - 1) / c.block); }
 
 int num_keep_of(const rola_config_t& c)
 {
@@ -46,6 +46,8 @@ rola_status_t validate(const rola_config_t* c)
         return ROLA_ERR_INVALID_ARG;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
+    // the sparse kernel counts a CTA's kept blocks in 32 bits (ring slots and phases)
+    if ((int64_t)c->B * c->H * num_blocks_of(*c) * num_keep_of(*c) >= ((int64_t)1 << 31)) return ROLA_ERR_UNSUPPORTED;
     if ((int64_t)c->B * c->H * c->N * c->d_h > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
     return ROLA_OK;
 }

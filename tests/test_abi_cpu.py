@@ -101,6 +101,16 @@ def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
     assert rl.workspace_bytes(c) == 0 and rl.num_keep(c) == 0
 
 
+def test_kept_block_count_limit(rl):
+    """B*H*nB*n_keep must stay below 2^31: the sparse kernel counts a CTA's kept blocks in 32 bits."""
+    N = 5793 * 64                                    # nB = 5793; 64 * 5793^2 just exceeds 2^31
+    big = cfg_tiny(rl, H=64, N=N, T=1, Hh=1, Ww=N, keep_ratio=1.0)
+    assert all(s == rl.ROLA_ERR_UNSUPPORTED for s in call_all(rl, big))
+    assert rl.workspace_bytes(big) == 0
+    half = cfg_tiny(rl, H=64, N=N, T=1, Hh=1, Ww=N, keep_ratio=0.5)
+    assert rl.num_keep(half) == 2897 and rl.workspace_bytes(half) > 0
+
+
 def test_rope_split_must_sum_to_head_dim(rl):
     c = cfg_tiny(rl)
     c.rope_split[:] = [44, 42, 40]
