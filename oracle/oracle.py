@@ -47,10 +47,13 @@ class OracleConfig(ctypes.Structure):
         ("eps_lr", ctypes.c_double), ("eps_f", ctypes.c_double),
         ("gate_bias", ctypes.c_double),
         ("rope_mode", ctypes.c_int32),
+        ("act", ctypes.c_int32),
     ]
 
 
 ROPE_OUTSIDE, ROPE_INSIDE, ROPE_NONE = 0, 1, 2
+# feature maps of the activation ablation (Tab. abl_activation), by the name a config dict uses
+ACTIVATIONS = {"silu": 0, "identity": 1, "tanh": 2, "relu": 3, "gelu": 4}
 
 
 def _get():
@@ -67,6 +70,8 @@ def _get():
             lib.orc_position.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.restype = ctypes.c_double
+            lib.orc_activation.argtypes = [cfgp, ctypes.c_double]
+            lib.orc_activation.restype = ctypes.c_double
             lib.orc_rotate.argtypes = [cfgp, ctypes.c_int, P, P, P, ctypes.c_int]
             lib.orc_lowrank_features.argtypes = [cfgp, P, P, P]
             lib.orc_lowrank_summary.argtypes = [cfgp, P, P, P, P, P]
@@ -98,6 +103,7 @@ def make_config(cfg: dict, rope_mode: int = ROPE_OUTSIDE) -> OracleConfig:
     c.eps_f = float(np.float32(cfg.get("eps_fuse", 1e-6)))
     c.gate_bias = float(np.float32(cfg.get("gate_bias", -1.946)))
     c.rope_mode = rope_mode
+    c.act = ACTIVATIONS[cfg.get("lowrank_act", "silu")]
     return c
 
 
@@ -108,6 +114,13 @@ def _f32(a):
 
 def _ptr(a):
     return None if a is None else a.ctypes.data
+
+
+def activation(name: str, x: float) -> float:
+    """The feature map phi of Eq. (qklr) (Tab. abl_activation), one fp64 value."""
+    c = make_config({"B": 1, "H": 1, "N": 1, "T": 1, "Hh": 1, "Ww": 1, "keep": 1.0, "r": 2,
+                     "lowrank_act": name})
+    return _get().orc_activation(ctypes.byref(c), float(x))
 
 
 def num_blocks(cfg: dict) -> int:

@@ -31,7 +31,10 @@
  *   fusion           Eq. (gate): r_p = sqrt(mean_i O^s_{p,i}^2 + eps),
  *                    O = (O^s / r_p + g_p O^lr) r_p.
  *   variants         Prop. (inside): SiLU(R_r(p) P x) ("inside"), and the
- *                    no-RoPE ablation (Sec. 5.2) SiLU(P x).
+ *                    no-RoPE ablation (Sec. 5.2) SiLU(P x); the feature map
+ *                    of the activation ablation (Tab. abl_activation):
+ *                    SiLU (default), identity, tanh, ReLU, GELU (the exact
+ *                    x Phi(x) form; the paper does not say which GELU).
  *
  * Layouts: q, k, v, o: [B][H][N][d_h]; P_q, P_k: [H][r][d_h];
  * C: [B][H][r][d_h]; z: [B][H][r]; gate: [B][N] (NULL -> sigmoid(gate_bias));
@@ -54,6 +57,7 @@ typedef struct {
     double eps_lr, eps_f;
     double gate_bias;     /* g = sigmoid(gate_bias) when gate == NULL */
     int32_t rope_mode;    /* 0: RoPE outside SiLU (RoLA), 1: inside, 2: none */
+    int32_t act;          /* 0: SiLU, 1: identity, 2: tanh, 3: ReLU, 4: GELU */
 } orc_cfg;
 
 /* ------------------------------------------------------------------ */
@@ -150,6 +154,20 @@ static double* token_cs(const orc_cfg* c)
 
 static double silu(double x) { return x / (1.0 + exp(-x)); }
 
+/* The feature map phi of Eq. (qklr): SiLU by default, or one of the
+ * activations of the ablation (Tab. abl_activation).  GELU is x * Phi(x)
+ * with Phi the standard normal CDF, Phi(x) = (1 + erf(x / sqrt 2)) / 2. */
+double orc_activation(const orc_cfg* c, double x)
+{
+    switch (c->act) {
+        case 1: return x;
+        case 2: return tanh(x);
+        case 3: return x > 0.0 ? x : 0.0;
+        case 4: return 0.5 * x * (1.0 + erf(x / sqrt(2.0)));
+        default: return silu(x);
+    }
+}
+
 /* ------------------------------------------------------------------ */
 /* low-rank features, Eq. (qklr) and its two ablations                */
 /* ------------------------------------------------------------------ */
@@ -165,14 +183,14 @@ static void lowrank_feature(const orc_cfg* c, const double* cs, const float* x, 
         for (int d = 0; d < dh; ++d) s += (double)P[(size_t)a * dh + d] * (double)x[d];
         u[a] = s;
     }
-    if (c->rope_mode == 0) {            /* R_r(p) SiLU(P x) */
-        for (int a = 0; a < r; ++a) u[a] = silu(u[a]);
+    if (c->rope_mode == 0) {            /* R_r(p) phi(P x) */
+        for (int a = 0; a < r; ++a) u[a] = orc_activation(c, u[a]);
         rotate_pairs(r / 2, cs, u, feat, r);
-    } else if (c->rope_mode == 1) {     /* SiLU(R_r(p) P x) */
+    } else if (c->rope_mode == 1) {     /* phi(R_r(p) P x) */
         rotate_pairs(r / 2, cs, u, feat, r);
-        for (int a = 0; a < r; ++a) feat[a] = silu(feat[a]);
-    } else {                            /* SiLU(P x) */
-        for (int a = 0; a < r; ++a) feat[a] = silu(u[a]);
+        for (int a = 0; a < r; ++a) feat[a] = orc_activation(c, feat[a]);
+    } else {                            /* phi(P x) */
+        for (int a = 0; a < r; ++a) feat[a] = orc_activation(c, u[a]);
     }
     free(u);
 }

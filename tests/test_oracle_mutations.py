@@ -39,6 +39,11 @@ MUTATIONS = {
     "gate_bias_dropped": ("double logit = b;", "double logit = 0.0;"),
     "gate_sigmoid_sign": ("g[p] = 1.0 / (1.0 + exp(-logit));", "g[p] = 1.0 / (1.0 + exp(logit));"),
     "gate_last_feature": ("for (int d = 0; d < D; ++d) logit +=", "for (int d = 0; d < D - 1; ++d) logit +="),
+    "gelu_scale": ("return 0.5 * x * (1.0 + erf(x / sqrt(2.0)));", "return 0.5 * x * (1.0 + erf(x / 2.0));"),
+    "tanh_for_identity": ("case 1: return x;", "case 1: return tanh(x);"),
+    "relu_leaky": ("case 3: return x > 0.0 ? x : 0.0;", "case 3: return x > 0.0 ? x : 0.01 * x;"),
+    "activation_before_rotation_only": ("for (int a = 0; a < r; ++a) u[a] = orc_activation(c, u[a]);",
+                                        "for (int a = 0; a < r; ++a) u[a] = silu(u[a]);"),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 

@@ -284,6 +284,77 @@ def test_projection_is_a_matmul(oracle):
     np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-13)
 
 
+ACTS = ["silu", "identity", "tanh", "relu", "gelu"]
+
+
+def test_activation_pins(oracle):
+    """The feature maps of the activation ablation (Tab. abl_activation) against closed forms:
+    phi(x) - phi(-x) = x for SiLU (sigma(x) + sigma(-x) = 1), ReLU and GELU (Phi(x) + Phi(-x) = 1);
+    SiLU(ln 3) = (3/4) ln 3; tanh odd, tanh(ln 2) = 3/5 and tanh(x) = 2 sigma(2x) - 1 with
+    sigma(2x) = SiLU(2x) / 2x; GELU(1) = Phi(1) from the normal table and x Phi(x) on a grid
+    (scipy's ndtr, an implementation independent of the C library's erf)."""
+    O = oracle
+    xs = np.linspace(-6.0, 6.0, 49)
+    phi = {n: np.array([O.activation(n, v) for v in xs]) for n in ACTS}
+    for n in ("silu", "relu", "gelu"):
+        np.testing.assert_allclose(phi[n] - phi[n][::-1], xs, rtol=0, atol=1e-14)
+    np.testing.assert_array_equal(phi["identity"], xs)
+    np.testing.assert_array_equal(phi["relu"], np.where(xs > 0, xs, 0.0))
+    assert O.activation("silu", math.log(3.0)) == pytest.approx(0.75 * math.log(3.0), abs=1e-15)
+    np.testing.assert_allclose(phi["tanh"], -phi["tanh"][::-1], rtol=0, atol=1e-16)
+    assert O.activation("tanh", math.log(2.0)) == pytest.approx(0.6, abs=1e-15)
+    nz = xs != 0
+    sig2 = np.array([O.activation("silu", 2 * v) / (2 * v) for v in xs[nz]])
+    np.testing.assert_allclose(phi["tanh"][nz], 2 * sig2 - 1, rtol=0, atol=1e-14)
+    assert O.activation("gelu", 1.0) == pytest.approx(0.8413447460685429, abs=1e-15)
+    special = pytest.importorskip("scipy.special")
+    np.testing.assert_allclose(phi["gelu"], xs * special.ndtr(xs), rtol=1e-14, atol=1e-15)
+
+
+def closed_form_act(name):
+    special = pytest.importorskip("scipy.special")
+    return {"silu": lambda a: a / (1.0 + np.exp(-a)), "identity": lambda a: a, "tanh": np.tanh,
+            "relu": lambda a: np.maximum(a, 0.0), "gelu": lambda a: a * special.ndtr(a)}[name]
+
+
+@pytest.mark.parametrize("act", ACTS)
+def test_features_apply_the_chosen_activation(oracle, act):
+    """With r = d_h and P = I the features of Eq. (qklr) are R(p) phi(x) (outside), phi(R(p) x)
+    (inside) and phi(x) (none), for every feature map of Tab. abl_activation."""
+    O = oracle
+    cfg = small_cfg(r=128, lowrank_act=act)
+    x = draw(cfg)
+    phi = closed_form_act(act)
+    P = np.broadcast_to(np.eye(128, dtype=np.float32), (cfg["H"], 128, 128)).copy()
+    k = x["k"].astype(np.float64)
+    none = O.lowrank_features(cfg, x["k"], P, rope_mode=O.ROPE_NONE)
+    np.testing.assert_allclose(none, phi(k), rtol=1e-13, atol=1e-14)
+    inside = O.lowrank_features(cfg, x["k"], P, rope_mode=O.ROPE_INSIDE)
+    np.testing.assert_allclose(inside, phi(O.rope_full(cfg, x["k"])), rtol=1e-13, atol=1e-14)
+    outside = O.lowrank_features(cfg, x["k"], P)
+    pk = phi(k)
+    want = np.stack([np.stack([O.rotate(cfg, 64, O.position(cfg, n), pk[0, h, n])
+                               for n in range(cfg["N"])]) for h in range(cfg["H"])])[None]
+    np.testing.assert_allclose(outside, want, rtol=1e-13, atol=1e-14)
+
+
+def test_identity_activation_is_rotary_linear_attention(oracle):
+    """Identity feature map, r = d_h, P = I: the summary form is plain (unnormalised) linear
+    attention on the fully rotated q and k, y = R q (R k)^T V (numpy matmuls); and the inside
+    placement equals the outside one, since a rotation commutes with the identity."""
+    O = oracle
+    cfg = small_cfg(r=128, lowrank_act="identity")
+    x = draw(cfg)
+    P = np.broadcast_to(np.eye(128, dtype=np.float32), (cfg["H"], 128, 128)).copy()
+    C, _ = O.lowrank_summary(cfg, x["k"], x["v"], P)
+    y = O.lowrank_readout(cfg, x["q"], P, C)
+    qr, kr = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"])
+    want = qr @ np.swapaxes(kr, -1, -2) @ x["v"].astype(np.float64)
+    np.testing.assert_allclose(y, want, rtol=1e-10, atol=1e-9)
+    Ci, _ = O.lowrank_summary(cfg, x["k"], x["v"], P, rope_mode=O.ROPE_INSIDE)
+    np.testing.assert_allclose(Ci, C, rtol=1e-12, atol=1e-11)
+
+
 def shift_residual(O, cfg, x, rope_mode, delta):
     a = O.forward(cfg, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], rope_mode=rope_mode)
     b = O.forward(dict(cfg, pos_offset=delta), x["q"], x["k"], x["v"], x["P_q"], x["P_k"],
@@ -307,6 +378,20 @@ def test_module_shift_invariance_outside_vs_inside(oracle):
     assert out < 1e-12
     assert non < 1e-12
     assert ins > 1e-3
+
+
+@pytest.mark.parametrize("act", ["identity", "tanh", "relu", "gelu"])
+def test_shift_invariance_for_every_activation(oracle, act):
+    """T5 for each feature map of Tab. abl_activation: with RoPE outside the activation the
+    module is shift-invariant whatever phi is (Prop. exact needs only a pointwise map before the
+    rotation); inside, a nonlinear phi breaks it (Prop. inside) while the identity does not."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=6, Ww=8, r=16, keep=0.25, lowrank_act=act)
+    x = draw(cfg)
+    x["gate"] = np.full((1, cfg["N"]), 0.9, np.float32)
+    assert shift_residual(O, cfg, x, O.ROPE_OUTSIDE, (7, 3, -2)) < 1e-12
+    ins = shift_residual(O, cfg, x, O.ROPE_INSIDE, (7, 3, -2))
+    assert ins < 1e-12 if act == "identity" else ins > 1e-3
 
 
 def test_truncation_bound(oracle):
