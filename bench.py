@@ -224,7 +224,8 @@ def run_reference(args, cfg, ws, rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * est["layer_s_est"],
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": cfg["name"], "B": cfg["B"], "H": cfg["H"], "N": cfg["N"],
-                   "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "keep": cfg["keep"], "r": cfg["r"]},
+                   "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "keep": cfg["keep"], "r": cfg["r"],
+                   "lowrank_act": cfg.get("lowrank_act", "silu")},
         "cpu_baseline": {"value": est["value"], "unit": "tokens/s", "cores": est["cores"], "kind": "oracle",
                          "sample": est["sample"], "wall_s_per_step": statistics.median(times)},
         "e2e": {"value": est["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -282,6 +283,8 @@ def main():
     ap.add_argument("--workload", default="wan14b_720p")
     ap.add_argument("--keep", type=float, default=None)
     ap.add_argument("--r", type=int, default=None)
+    ap.add_argument("--lowrank-act", default=None, choices=["silu", "identity", "tanh", "relu", "gelu"],
+                    help="feature map of the low-rank branch (the activation ablation); default SiLU")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -300,6 +303,8 @@ def main():
         cfg = configs.sweep_config(args.r if args.r is not None else 32, args.keep if args.keep is not None else 0.1)
     else:
         cfg = configs.get(args.workload, **over)
+    if args.lowrank_act is not None:
+        cfg["lowrank_act"] = args.lowrank_act
     ws, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, cfg, ws, rank)
@@ -527,7 +532,7 @@ def main():
             "dtype": "bf16", "data": "synthetic",
             "config": {"workload": cfg["name"], "B": cfg["B"], "H": cfg["H"], "N": cfg["N"],
                        "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "block": 64, "keep": cfg["keep"],
-                       "n_keep": nk, "r": cfg["r"], "d_h": 128,
+                       "n_keep": nk, "r": cfg["r"], "d_h": 128, "lowrank_act": cfg.get("lowrank_act", "silu"),
                        "l2": "no flush: q, k, v are each larger than L2 (774 MB vs 129 MB)",
                        "parallelism": f"replica per GPU x{ws}"},
             "stage_ms": stage_ms,

@@ -94,6 +94,8 @@ typedef struct {
                                   out and the call reports ROLA_ERR_TIMEOUT (tests the timeout path) */
     int32_t lowrank_rope;      /* where the truncated RoPE sits in the low-rank features; one of
                                   rola_lowrank_rope_t, default ROLA_LOWRANK_ROPE_OUTSIDE */
+    int32_t lowrank_act;       /* feature map phi of the low-rank features; one of
+                                  rola_lowrank_act_t, default ROLA_LOWRANK_ACT_SILU */
 } rola_config_t;
 
 #define ROLA_DEBUG_SKIP_FIRST_K_COPY 1
@@ -112,6 +114,24 @@ typedef enum {
     ROLA_LOWRANK_ROPE_INSIDE = 1,
     ROLA_LOWRANK_ROPE_NONE = 2
 } rola_lowrank_rope_t;
+
+/*
+ * Feature map phi of the low-rank branch (SiLU in Eq. qklr; the others are
+ * the activation ablation, Tab. abl_activation), applied coordinatewise to
+ * P x wherever SiLU appears in the formulas of this header:
+ *   SILU      x / (1 + exp(-x))              the RoLA default
+ *   IDENTITY  x                              plain (rotary) linear features
+ *   TANH      tanh(x)
+ *   RELU      max(x, 0)
+ *   GELU      x Phi(x) = x (1 + erf(x / sqrt 2)) / 2   (the exact form)
+ */
+typedef enum {
+    ROLA_LOWRANK_ACT_SILU = 0,
+    ROLA_LOWRANK_ACT_IDENTITY = 1,
+    ROLA_LOWRANK_ACT_TANH = 2,
+    ROLA_LOWRANK_ACT_RELU = 3,
+    ROLA_LOWRANK_ACT_GELU = 4
+} rola_lowrank_act_t;
 
 /* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
 rola_status_t rola_config_init(rola_config_t* cfg);
@@ -157,7 +177,7 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
 /*
  * Kernel (3): low-rank summary, Eq. (qklr) and Eq. (ctx):
  *   k~_q = R_r(q) SiLU(P_k k^n_q),   C = sum_q k~_q v_q^T,   z = sum_q k~_q
- * (k~ as cfg->lowrank_rope places the rotation).
+ * (k~ as cfg->lowrank_rope places the rotation, with cfg->lowrank_act's feature map).
  * R_r keeps the first r coordinates (r/2 complete pairs) of the native RoPE
  * ordering (Sec. 4.2).  The reduction over N is split across CTAs (one
  * contiguous token range each) and combined in a fixed order, so results are
@@ -171,7 +191,8 @@ rola_status_t rola_lowrank_summary(const rola_config_t* cfg, const void* k, cons
 
 /*
  * Kernel (4): low-rank readout and gated fusion, Eq. (ctx) and Eq. (gate):
- *   q~_p   = R_r(p) SiLU(P_q q^n_p)            (as cfg->lowrank_rope places R_r)
+ *   q~_p   = R_r(p) SiLU(P_q q^n_p)            (as cfg->lowrank_rope places R_r; SiLU or
+ *                                               cfg->lowrank_act's feature map)
  *   O^lr_p = y_p / sqrt(mean_i y_{p,i}^2 + eps_lr),   y_p = q~_p^T C
  *   r_p    = sqrt(mean_i (O^s_{p,i})^2 + eps_fuse)
  *   O_p    = (O^s_p / r_p + g_p O^lr_p) r_p

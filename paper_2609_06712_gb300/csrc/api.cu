@@ -44,6 +44,7 @@ rola_status_t validate(const rola_config_t* c)
     if (c->debug_flags & ~ROLA_DEBUG_SKIP_FIRST_K_COPY) return ROLA_ERR_INVALID_ARG;
     if (c->lowrank_rope < ROLA_LOWRANK_ROPE_OUTSIDE || c->lowrank_rope > ROLA_LOWRANK_ROPE_NONE)
         return ROLA_ERR_INVALID_ARG;
+    if (c->lowrank_act < ROLA_LOWRANK_ACT_SILU || c->lowrank_act > ROLA_LOWRANK_ACT_GELU) return ROLA_ERR_INVALID_ARG;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
     // the sparse kernel counts a CTA's kept blocks in 32 bits (ring slots and phases)
@@ -69,6 +70,7 @@ Shape make_shape(const rola_config_t& c)
     s.wait_limit_ns = (uint64_t)(c.wait_limit_ms > 0 ? c.wait_limit_ms : 2000) * 1000000ull;
     s.debug_flags = c.debug_flags;
     s.lr_rope = c.lowrank_rope;
+    s.lr_act = c.lowrank_act;
     return s;
 }
 

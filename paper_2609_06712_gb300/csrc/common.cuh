@@ -42,6 +42,7 @@ struct Shape {
     uint64_t wait_limit_ns;   // bound of every device-side wait
     int debug_flags;          // ROLA_DEBUG_* test hooks
     int lr_rope;              // rola_lowrank_rope_t
+    int lr_act;               // rola_lowrank_act_t
 };
 
 // Rotation (cos, sin) of pair m for the token at flat index n.
@@ -66,7 +67,7 @@ __device__ __forceinline__ float2 rope_rotate(float x0, float x1, float2 cs)
 // One pair of low-rank features from the projected pair (u0, u1) = the pair's
 // two rows of P x: R_r after SiLU (Eq. qklr, ROLA_LOWRANK_ROPE_OUTSIDE), before
 // it (Prop. inside, ROLA_LOWRANK_ROPE_INSIDE) or not at all (ROLA_LOWRANK_ROPE_NONE).
-// `act` is the SiLU evaluation the caller uses.
+// `act` is the feature-map evaluation the caller uses (SiLU, or ActAblation).
 template <typename Act>
 __device__ __forceinline__ float2 lowrank_pair(float u0, float u1, float2 cs, int mode, Act act)
 {
@@ -200,6 +201,22 @@ __device__ __forceinline__ float fast_exp2(float x)
 }
 
 __device__ __forceinline__ float silu(float x) { return x / (1.0f + __expf(-x)); }
+
+// The feature maps of the activation ablation other than SiLU (Tab. abl_activation),
+// chosen at run time by `kind` (a rola_lowrank_act_t).  tanhf and erff are CUDA's
+// accurate functions; GELU is the exact x Phi(x) form.
+struct ActAblation {
+    int kind;
+    __device__ float operator()(float x) const
+    {
+        switch (kind) {
+            case ROLA_LOWRANK_ACT_IDENTITY: return x;
+            case ROLA_LOWRANK_ACT_TANH: return tanhf(x);
+            case ROLA_LOWRANK_ACT_RELU: return fmaxf(x, 0.0f);
+            default: return 0.5f * x * (1.0f + erff(x * 0.7071067811865476f));
+        }
+    }
+};
 
 // Byte offset of 16-byte chunk c of row r in a [rows][128 bf16] tile with the
 // chunk index XOR-swizzled by the row (conflict-free ldmatrix on 8-row groups).

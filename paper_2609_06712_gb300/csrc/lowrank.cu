@@ -15,11 +15,15 @@
 
 namespace rola {
 
-// SiLU with the IEEE exp and divide (fp32 validation mode)
-struct SiluIeee {
-    __device__ float operator()(float x) const { return x / (1.0f + expf(-x)); }
+// The feature map in the fp32 validation mode: SiLU with the IEEE exp and
+// divide, or one of the ablation's activations.
+struct ActIeee {
+    int kind;
+    __device__ float operator()(float x) const
+    {
+        return kind == ROLA_LOWRANK_ACT_SILU ? x / (1.0f + expf(-x)) : ActAblation{kind}(x);
+    }
 };
-__device__ constexpr SiluIeee silu_ieee{};
 
 // ===========================================================================
 // Split-N partitioning of the fp32 summary: CTA = (split, head).
@@ -80,7 +84,7 @@ __global__ void __launch_bounds__(256) summary_f32_kernel(Shape s, int tokens_pe
                 u1 = fmaf(Ks[r * (kDh + 1) + c], Ps[(2 * m + 1) * (kDh + 1) + c], u1);
             }
             float2 cs = n < n_end ? rope_cs(tab, s, n, m) : make_float2(0.0f, 0.0f);
-            const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, silu_ieee);
+            const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, ActIeee{s.lr_act});
             Us[r * (R + 1) + 2 * m] = f.x;
             Us[r * (R + 1) + 2 * m + 1] = f.y;
         }
@@ -191,7 +195,7 @@ __global__ void __launch_bounds__(256) apply_f32_kernel(Shape s, const float* __
             u1 = fmaf(Qs[r * (kDh + 1) + c], Ps[(2 * m + 1) * (kDh + 1) + c], u1);
         }
         float2 cs = rope_cs(tab, s, n, m);
-        const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, silu_ieee);
+        const float2 f = lowrank_pair(u0, u1, cs, s.lr_rope, ActIeee{s.lr_act});
         Us[r * (R + 1) + 2 * m] = f.x;
         Us[r * (R + 1) + 2 * m + 1] = f.y;
     }

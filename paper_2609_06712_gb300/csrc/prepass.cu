@@ -126,12 +126,14 @@ __device__ __forceinline__ uint4 lds128(uint32_t a)
     return w;
 }
 
-// SiLU with the approximate divide (the features enter the MMA in bf16)
+// SiLU with the approximate divide (the features enter the MMA in bf16).  The
+// kernel is instantiated for it and for ActAblation (the other feature maps).
 struct SiluFast {
+    int kind;    // always ROLA_LOWRANK_ACT_SILU
     __device__ float operator()(float x) const { return __fdividef(x, 1.0f + __expf(-x)); }
 };
 
-template <int R>
+template <int R, typename Act>
 __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
     const __grid_constant__ CUtensorMap map_v, const Params p)
@@ -392,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
                     for (int j = 0; j < NTW; ++j) {
                         const int nt = cg * NTW + j;
                         const float2 cs2 = valid ? kcs[hr][j] : make_float2(0.0f, 0.0f);
-                        const float2 y = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], cs2, s.lr_rope, SiluFast{});
+                        const float2 y = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], cs2, s.lr_rope, Act{s.lr_act});
                         zacc[j][0] += y.x;
                         zacc[j][1] += y.y;
                         asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(ktb + tl * C::KT + (nt * 8 + t4 * 2) * 2),
@@ -469,16 +471,24 @@ __global__ void prepass_combine_kernel(Shape s, int ctas, int units, const float
     }
 }
 
+template <int R, typename Act>
+cudaError_t launch_ra(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv, const Params& p, int ctas,
+                      bool fuse, cudaStream_t st)
+{
+    const Layout lay(R, fuse);
+    cudaError_t e = cudaFuncSetAttribute(prepass_kernel<R, Act>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)lay.total);
+    if (e != cudaSuccess) return e;
+    prepass_kernel<R, Act><<<ctas, kThreads, lay.total, st>>>(mq, mk, mv, p);
+    return cudaGetLastError();
+}
+
 template <int R>
 cudaError_t launch_r(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv, const Params& p, int ctas,
                      bool fuse, cudaStream_t st)
 {
-    const Layout lay(R, fuse);
-    cudaError_t e = cudaFuncSetAttribute(prepass_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)lay.total);
-    if (e != cudaSuccess) return e;
-    prepass_kernel<R><<<ctas, kThreads, lay.total, st>>>(mq, mk, mv, p);
-    return cudaGetLastError();
+    return p.s.lr_act == ROLA_LOWRANK_ACT_SILU ? launch_ra<R, SiluFast>(mq, mk, mv, p, ctas, fuse, st)
+                                               : launch_ra<R, ActAblation>(mq, mk, mv, p, ctas, fuse, st);
 }
 
 }  // namespace

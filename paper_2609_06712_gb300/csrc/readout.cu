@@ -66,11 +66,14 @@ struct Params {
     int units;
 };
 
+// SiLU with the MUFU exponential; the kernel is instantiated for it and for
+// ActAblation (the other feature maps of the activation ablation).
 struct SiluMufu {
+    int kind;    // always ROLA_LOWRANK_ACT_SILU
     __device__ float operator()(float x) const { return silu(x); }
 };
 
-template <int R>
+template <int R, typename Act>
 __global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(const __grid_constant__ CUtensorMap map_q,
                                                               const __grid_constant__ CUtensorMap map_os,
                                                               const __grid_constant__ CUtensorMap map_o,
@@ -218,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(c
                 for (int j = 0; j < NTW; ++j) {
                     const int nt = half * NTW + j;
                     const float2 f = lowrank_pair(uacc[j][2 * hr], uacc[j][2 * hr + 1], kcs[hr][j], s.lr_rope,
-                                                  SiluMufu{});
+                                                  Act{s.lr_act});
                     asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(sQt + tl * L::QT + (nt * 8 + t4 * 2) * 2),
                                  "r"(pack_bf16(f.x, f.y))
                                  : "memory");
@@ -322,16 +325,25 @@ __global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(c
     }
 }
 
+template <int R, typename Act>
+cudaError_t launch_ra(const CUtensorMap& mq, const CUtensorMap& mos, const CUtensorMap& mo, const Params& p, int ctas,
+                      cudaStream_t st)
+{
+    using L = Layout<R>;
+    static_assert(L::total <= 232448, "fits the shared memory of one SM");
+    cudaError_t e =
+        cudaFuncSetAttribute(readout_kernel<R, Act>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
+    if (e != cudaSuccess) return e;
+    readout_kernel<R, Act><<<ctas, kThreads, L::total, st>>>(mq, mos, mo, p);
+    return cudaGetLastError();
+}
+
 template <int R>
 cudaError_t launch_r(const CUtensorMap& mq, const CUtensorMap& mos, const CUtensorMap& mo, const Params& p, int ctas,
                      cudaStream_t st)
 {
-    using L = Layout<R>;
-    static_assert(L::total <= 232448, "fits the shared memory of one SM");
-    cudaError_t e = cudaFuncSetAttribute(readout_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L::total);
-    if (e != cudaSuccess) return e;
-    readout_kernel<R><<<ctas, kThreads, L::total, st>>>(mq, mos, mo, p);
-    return cudaGetLastError();
+    return p.s.lr_act == ROLA_LOWRANK_ACT_SILU ? launch_ra<R, SiluMufu>(mq, mos, mo, p, ctas, st)
+                                               : launch_ra<R, ActAblation>(mq, mos, mo, p, ctas, st);
 }
 
 }  // namespace

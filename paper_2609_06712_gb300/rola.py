@@ -37,12 +37,18 @@ class RolaConfig(ctypes.Structure):
         ("wait_limit_ms", ctypes.c_int32),
         ("debug_flags", ctypes.c_int32),
         ("lowrank_rope", ctypes.c_int32),
+        ("lowrank_act", ctypes.c_int32),
     ]
 
 
 ROLA_DEBUG_SKIP_FIRST_K_COPY = 1
 # rola_lowrank_rope_t: where the truncated RoPE sits in the low-rank features
 ROLA_LOWRANK_ROPE_OUTSIDE, ROLA_LOWRANK_ROPE_INSIDE, ROLA_LOWRANK_ROPE_NONE = 0, 1, 2
+# rola_lowrank_act_t: the feature map of the low-rank features, and the names a config dict uses
+(ROLA_LOWRANK_ACT_SILU, ROLA_LOWRANK_ACT_IDENTITY, ROLA_LOWRANK_ACT_TANH, ROLA_LOWRANK_ACT_RELU,
+ ROLA_LOWRANK_ACT_GELU) = 0, 1, 2, 3, 4
+LOWRANK_ACTS = {"silu": ROLA_LOWRANK_ACT_SILU, "identity": ROLA_LOWRANK_ACT_IDENTITY,
+                "tanh": ROLA_LOWRANK_ACT_TANH, "relu": ROLA_LOWRANK_ACT_RELU, "gelu": ROLA_LOWRANK_ACT_GELU}
 
 
 class RolaError(RuntimeError):
@@ -108,6 +114,8 @@ def make_config(cfg: dict, dtype: int = ROLA_BF16) -> RolaConfig:
     c.gate_bias = float(cfg.get("gate_bias", -1.946))
     c.dtype = dtype
     c.lowrank_rope = int(cfg.get("lowrank_rope", ROLA_LOWRANK_ROPE_OUTSIDE))
+    act = cfg.get("lowrank_act", "silu")
+    c.lowrank_act = LOWRANK_ACTS[act] if isinstance(act, str) else int(act)
     return c
 
 

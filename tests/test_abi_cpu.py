@@ -39,6 +39,23 @@ def test_exports_every_declared_entry_point(rl):
         getattr(rl.library(), n)
 
 
+def test_config_struct_layout_matches_the_header(rl, tmp_path):
+    """The binding's RolaConfig has the size and field offsets that a C compiler gives rola_config_t."""
+    fields = [f[0] for f in rl.RolaConfig._fields_]
+    prog = tmp_path / "layout.c"
+    body = "".join(f'    printf("%s %zu\\n", "{n}", offsetof(rola_config_t, {n}));\n' for n in fields)
+    prog.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "rola.h"\nint main(void) {\n'
+                    '    printf("sizeof %zu\\n", sizeof(rola_config_t));\n' + body + "    return 0;\n}\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run(["gcc", "-std=c99", "-I", inc, str(prog), "-o", str(exe)], check=True)
+    got = dict(line.split() for line in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                       check=True).stdout.splitlines())
+    assert int(got["sizeof"]) == ctypes.sizeof(rl.RolaConfig)
+    for n in fields:
+        assert int(got[n]) == getattr(rl.RolaConfig, n).offset, n
+
+
 def cfg_tiny(rl, **kw):
     from paper_2609_06712_gb300 import configs
     c = rl.make_config(configs.get("tiny"))
@@ -52,6 +69,7 @@ def test_defaults_and_sizes(rl):
     assert rl.library().rola_config_init(ctypes.byref(c)) == rl.ROLA_OK
     assert (c.d_h, c.block, list(c.rope_split), c.rope_theta) == (128, 64, [44, 42, 42], 10000.0)
     assert c.gate_bias == pytest.approx(-1.946) and c.eps_lr == pytest.approx(1e-6)
+    assert c.lowrank_act == rl.ROLA_LOWRANK_ACT_SILU
     assert c.lowrank_rope == rl.ROLA_LOWRANK_ROPE_OUTSIDE and c.wait_limit_ms == 0 and c.debug_flags == 0
     from paper_2609_06712_gb300 import configs
     for name, nb, nk in [("tiny", 16, 2), ("wan13b_480p", 512, 51), ("wan14b_720p", 1182, 118),
@@ -94,6 +112,8 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
     ("debug_flags", 2, 1),
     ("lowrank_rope", 3, 1),
     ("lowrank_rope", -1, 1),
+    ("lowrank_act", 5, 1),
+    ("lowrank_act", -1, 1),
 ])
 def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
     c = cfg_tiny(rl, **{field: value})

@@ -1,0 +1,115 @@
+"""The feature maps of the paper's activation ablation (Tab. abl_activation):
+identity, tanh, ReLU and GELU in place of SiLU in Eq. (qklr).  CUDA path vs the
+fp64 oracle per kernel (summary, readout + fusion) and for the module, bf16 and
+fp32, in the outside placement and, for GELU, the inside one; and SiLU chosen
+explicitly is bit-identical to the default."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2609_06712_gb300 import configs, inputs
+from parity_util import assert_close, check_mask, dev, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rl():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2609_06712_gb300 import build
+    build.build()
+    from paper_2609_06712_gb300 import rola
+    O.build()
+    return rola
+
+
+def layer(**kw):
+    c = configs.get("tiny")
+    c.update(kw)
+    c["N"] = c["T"] * c["Hh"] * c["Ww"]
+    return c
+
+
+CASES = {
+    "ragged_585_r32": layer(T=5, Hh=9, Ww=13, H=2, r=32, keep=0.3, seed=31, dist="normal_gate"),
+    "r64": layer(T=2, Hh=12, Ww=16, H=2, r=64, keep=0.25, seed=32),
+}
+ACTS = ["identity", "tanh", "relu", "gelu"]
+DTYPES = [("bf16", torch.bfloat16), ("fp32", torch.float32)]
+
+
+def draw(cfg, dtype):
+    x = inputs.make_inputs(cfg, dtype=dtype)
+    return x, {k: (None if v is None else v.float().numpy()) for k, v in x.items()}
+
+
+def run_summary_apply(rl, cfg, x, c):
+    ws = rl.workspace(c)
+    C = torch.empty((cfg["B"], cfg["H"], cfg["r"], 128), dtype=torch.float32, device="cuda")
+    z = torch.empty((cfg["B"], cfg["H"], cfg["r"]), dtype=torch.float32, device="cuda")
+    rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, z, ws)
+    torch.cuda.synchronize()
+    assert rl.get_device_status(ws) == rl.ROLA_OK
+    return C, z, ws
+
+
+@pytest.mark.parametrize("case", sorted(CASES))
+@pytest.mark.parametrize("act", ACTS)
+@pytest.mark.parametrize("dname,tdt", DTYPES)
+@pytest.mark.parametrize("placement", ["outside", "inside"])
+def test_summary_and_apply(rl, case, act, dname, tdt, placement):
+    if placement == "inside" and act != "gelu":
+        pytest.skip("the inside placement is covered with GELU")
+    lr_mode, o_mode = (0, O.ROPE_OUTSIDE) if placement == "outside" else (1, O.ROPE_INSIDE)
+    cfg = dict(CASES[case], lowrank_act=act)
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(dict(cfg, lowrank_rope=lr_mode), rl.ROLA_BF16 if dname == "bf16" else rl.ROLA_FP32)
+    C, z, ws = run_summary_apply(rl, cfg, x, c)
+    Cw, zw = O.lowrank_summary(cfg, h["k"], h["v"], h["P_k"], rope_mode=o_mode)
+    tag = f"[{case},{act},{placement},{dname}]"
+    assert_close(to_np(C), Cw, dname == "bf16", "C" + tag, unit_rms=True)
+    assert_close(to_np(z), zw, dname == "bf16", "z" + tag, unit_rms=True)
+    g = torch.Generator().manual_seed(cfg["seed"] + 1000)
+    o_s = (0.02 * torch.randn(x["q"].shape, generator=g)).to(tdt)
+    C32 = torch.from_numpy(Cw.astype(np.float32))
+    o = torch.empty_like(dev(o_s))
+    rl.lowrank_apply(c, dev(x["q"]), dev(x["P_q"]), dev(C32), dev(x["gate"]), dev(o_s), o, ws)
+    torch.cuda.synchronize()
+    want = O.lowrank_apply(cfg, h["q"], h["P_q"], C32.double().numpy(), h["gate"], o_s.float().numpy(),
+                           rope_mode=o_mode)
+    assert_close(to_np(o), want, dname == "bf16", "O" + tag)
+
+
+@pytest.mark.parametrize("act", ACTS)
+@pytest.mark.parametrize("dname,tdt", DTYPES)
+def test_forward(rl, act, dname, tdt):
+    cfg = dict(CASES["ragged_585_r32"], lowrank_act=act)
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rl.ROLA_BF16 if dname == "bf16" else rl.ROLA_FP32)
+    ws = rl.workspace(c)
+    nB, nk = rl.num_blocks(c), rl.num_keep(c)
+    out = torch.empty_like(dev(x["q"]))
+    kv = torch.empty((cfg["B"], cfg["H"], nB, nk), dtype=torch.int32, device="cuda")
+    rl.forward(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), dev(x["P_q"]), dev(x["P_k"]), dev(x["gate"]), out, kv, ws)
+    torch.cuda.synchronize()
+    assert rl.get_device_status(ws) == rl.ROLA_OK
+    res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], mask_override=kv.cpu().numpy())
+    idx, scores, gap, tau = O.block_mask(cfg, h["q"], h["k"])
+    check_mask(kv.cpu().numpy(), idx, scores, gap, tau, nB)
+    assert_close(to_np(out), res["o"], dname == "bf16", f"O[forward,{act},{dname}]")
+
+
+def test_explicit_silu_is_the_default(rl):
+    cfg = CASES["ragged_585_r32"]
+    x, _ = draw(cfg, torch.bfloat16)
+    outs = []
+    for extra in ({}, {"lowrank_act": "silu"}):
+        c = rl.make_config(dict(cfg, **extra), rl.ROLA_BF16)
+        ws = rl.workspace(c)
+        out = torch.empty_like(dev(x["q"]))
+        rl.forward(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), dev(x["P_q"]), dev(x["P_k"]), dev(x["gate"]), out,
+                   None, ws)
+        torch.cuda.synchronize()
+        outs.append(out)
+    assert torch.equal(outs[0], outs[1])
