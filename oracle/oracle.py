@@ -48,12 +48,15 @@ class OracleConfig(ctypes.Structure):
         ("gate_bias", ctypes.c_double),
         ("rope_mode", ctypes.c_int32),
         ("act", ctypes.c_int32),
+        ("geometry", ctypes.c_int32),
     ]
 
 
 ROPE_OUTSIDE, ROPE_INSIDE, ROPE_NONE = 0, 1, 2
 # feature maps of the activation ablation (Tab. abl_activation), by the name a config dict uses
 ACTIVATIONS = {"silu": 0, "identity": 1, "tanh": 2, "relu": 3, "gelu": 4}
+# block geometries: contiguous 64-token chunks, or 4 x 4 x 4 cubes of the latent grid
+GEOMETRIES = {"flat": 0, "cube": 1}
 
 
 def _get():
@@ -67,6 +70,7 @@ def _get():
             cfgp = ctypes.POINTER(OracleConfig)
             lib.orc_num_blocks.argtypes = [cfgp]
             lib.orc_num_keep.argtypes = [cfgp]
+            lib.orc_block_of.argtypes = [cfgp, ctypes.c_int]
             lib.orc_position.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.restype = ctypes.c_double
@@ -104,6 +108,7 @@ def make_config(cfg: dict, rope_mode: int = ROPE_OUTSIDE) -> OracleConfig:
     c.gate_bias = float(np.float32(cfg.get("gate_bias", -1.946)))
     c.rope_mode = rope_mode
     c.act = ACTIVATIONS[cfg.get("lowrank_act", "silu")]
+    c.geometry = GEOMETRIES[cfg.get("block_geometry", "flat")]
     return c
 
 
@@ -131,6 +136,13 @@ def num_blocks(cfg: dict) -> int:
 def num_keep(cfg: dict) -> int:
     c = make_config(cfg)
     return _get().orc_num_keep(ctypes.byref(c))
+
+
+def block_of(cfg: dict) -> np.ndarray:
+    """Block id of every token [N]: its 64-token chunk, or its 4 x 4 x 4 cube (t-major cube numbering)."""
+    c = make_config(cfg)
+    lib = _get()
+    return np.array([lib.orc_block_of(ctypes.byref(c), n) for n in range(c.N)], dtype=np.int64)
 
 
 def position(cfg: dict, n: int) -> np.ndarray:

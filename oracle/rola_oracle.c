@@ -23,6 +23,12 @@
  *                    mean-pools the rotated q / k over each block, scores
  *                    q_bar . k_bar / sqrt(d_h) and keeps the n_keep largest
  *                    per query block (ties -> lower block index).
+ *   block geometry   not described by the paper either: contiguous chunks of
+ *                    `block` tokens of the t-major sequence (geometry 0), or
+ *                    4 x 4 x 4 cubes of the (t, x, y) latent grid (geometry
+ *                    1, the tiling of the sparse video attentions the paper
+ *                    builds on), numbered t-major over the cube grid; edge
+ *                    cubes hold the tokens that fall inside the grid.
  *   sparse branch    Sec. 3 (softmax(QK^T / sqrt d_h) V) restricted to the
  *                    kept key blocks; Alg. 1 sparse-branch steps.
  *   low-rank branch  Eq. (qklr): q~ = R_r(p) SiLU(P_q q^n), k~ = R_r(q)
@@ -58,13 +64,43 @@ typedef struct {
     double gate_bias;     /* g = sigmoid(gate_bias) when gate == NULL */
     int32_t rope_mode;    /* 0: RoPE outside SiLU (RoLA), 1: inside, 2: none */
     int32_t act;          /* 0: SiLU, 1: identity, 2: tanh, 3: ReLU, 4: GELU */
+    int32_t geometry;     /* 0: contiguous chunks of `block` tokens, 1: 4x4x4 cubes */
 } orc_cfg;
+
+enum { CUBE = 4 };        /* cube edge of geometry 1 (CUBE^3 == block == 64) */
 
 /* ------------------------------------------------------------------ */
 /* sizes                                                              */
 /* ------------------------------------------------------------------ */
 
-int orc_num_blocks(const orc_cfg* c) { return (c->N + c->block - 1) / c->block; }
+int orc_num_blocks(const orc_cfg* c)
+{
+    if (c->geometry == 1)
+        return ((c->T + CUBE - 1) / CUBE) * ((c->Hh + CUBE - 1) / CUBE) * ((c->Ww + CUBE - 1) / CUBE);
+    return (c->N + c->block - 1) / c->block;
+}
+
+/* The block token n belongs to: its chunk n / block, or its cube
+ * (t / 4, x / 4, y / 4) numbered t-major over the cube grid. */
+int orc_block_of(const orc_cfg* c, int n)
+{
+    if (c->geometry != 1) return n / c->block;
+    int t = n / (c->Hh * c->Ww), x = (n / c->Ww) % c->Hh, y = n % c->Ww;
+    int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;
+    return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;
+}
+
+/* Members of every block in ascending token order: list[b * block + i] for
+ * i < cnt[b] (a block never holds more than `block` tokens). */
+static void block_members(const orc_cfg* c, int* list, int* cnt)
+{
+    int nB = orc_num_blocks(c);
+    for (int b = 0; b < nB; ++b) cnt[b] = 0;
+    for (int n = 0; n < c->N; ++n) {
+        int b = orc_block_of(c, n);
+        list[(size_t)b * c->block + cnt[b]++] = n;
+    }
+}
 
 int orc_num_keep(const orc_cfg* c)
 {
@@ -289,7 +325,7 @@ static void fuse(const orc_cfg* c, const double* os, const double* olr, double g
 /* Token list helper: the tokens of the selected query blocks (all if NULL). */
 static int token_in_selection(const orc_cfg* c, int n, const uint8_t* qb_sel)
 {
-    return qb_sel == NULL || qb_sel[n / c->block];
+    return qb_sel == NULL || qb_sel[orc_block_of(c, n)];
 }
 
 /* O = fusion(O^s, RMSNorm(q~^T C)) for the tokens of the selected query
@@ -427,6 +463,9 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
     double isd = 1.0 / sqrt((double)dh);
     const double u = ldexp(1.0, -24);
     double* tcs = token_cs(c);
+    int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
+    int* count = (int*)malloc(sizeof(int) * (size_t)nB);
+    block_members(c, members, count);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
         size_t nbd = (size_t)nB * dh;
@@ -445,14 +484,14 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
                 size_t off = ((size_t)bh * N + n) * dh;
                 for (int d = 0; d < dh; ++d) xi[d] = (double)x[off + d];
                 rotate_pairs(dh / 2, tcs + (size_t)n * dh, xi, xr, dh);
-                int blk = n / bs;
+                int blk = orc_block_of(c, n);
                 for (int d = 0; d < dh; ++d) {
                     mean[(size_t)blk * dh + d] += xr[d];
                     mag[(size_t)blk * dh + d] += fabs(xi[d & ~1]) + fabs(xi[d | 1]);
                 }
             }
             for (int blk = 0; blk < nB; ++blk) {
-                int cnt = (blk + 1) * bs <= N ? bs : N - blk * bs;
+                int cnt = count[blk];
                 for (int d = 0; d < dh; ++d) {
                     mean[(size_t)blk * dh + d] /= (double)cnt;
                     mag[(size_t)blk * dh + d] /= (double)cnt;
@@ -490,6 +529,8 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
         free(qb); free(kb); free(qa); free(ka); free(xr); free(xi); free(row);
     }
     free(tcs);
+    free(members);
+    free(count);
 }
 
 /* ------------------------------------------------------------------ */
@@ -507,22 +548,23 @@ void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const
     int nB = orc_num_blocks(c);
     double isd = 1.0 / sqrt((double)dh);
     int ntask = BH * nB;
+    int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
+    int* count = (int*)malloc(sizeof(int) * (size_t)nB);
+    block_members(c, members, count);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int task = 0; task < ntask; ++task) {
         int bh = task / nB, i = task % nB;
         if (qb_sel && !qb_sel[i]) continue;
         const int32_t* kept = kv_idx + ((size_t)bh * nB + i) * n_keep;
         int nkeys = 0;
-        for (int t = 0; t < n_keep; ++t) {
-            int j = kept[t];
-            nkeys += (j + 1) * bs <= N ? bs : N - j * bs;
-        }
+        for (int t = 0; t < n_keep; ++t) nkeys += count[kept[t]];
         int* keys = (int*)malloc(sizeof(int) * (size_t)nkeys);
         double* s = (double*)malloc(sizeof(double) * (size_t)nkeys);
         int kk = 0;
         for (int t = 0; t < n_keep; ++t)
-            for (int qn = kept[t] * bs; qn < (kept[t] + 1) * bs && qn < N; ++qn) keys[kk++] = qn;
-        for (int p = i * bs; p < (i + 1) * bs && p < N; ++p) {
+            for (int m = 0; m < count[kept[t]]; ++m) keys[kk++] = members[(size_t)kept[t] * bs + m];
+        for (int mi = 0; mi < count[i]; ++mi) {
+            int p = members[(size_t)i * bs + mi];
             const double* qp = qr + ((size_t)bh * N + p) * dh;
             double mx = -INFINITY;
             for (int t = 0; t < nkeys; ++t) {
@@ -545,6 +587,8 @@ void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const
         free(keys);
         free(s);
     }
+    free(members);
+    free(count);
 }
 
 /* ------------------------------------------------------------------ */

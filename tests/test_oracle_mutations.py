@@ -32,7 +32,10 @@ MUTATIONS = {
     "pool_unrotated": ("mean[(size_t)blk * dh + d] += xr[d];", "mean[(size_t)blk * dh + d] += xi[d];"),
     "softmax_scale": ("double isd = 1.0 / sqrt((double)dh);\n    int ntask",
                       "double isd = 1.0;\n    int ntask"),
-    "ragged_keys": ("nkeys += (j + 1) * bs <= N ? bs : N - j * bs;", "nkeys += bs <= N ? bs : N;"),
+    "cube_axis_stride": ("return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;",
+                         "return ((t / CUBE) * ny + x / CUBE) * nx + y / CUBE;"),
+    "cube_grid_rounding": ("int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;",
+                           "int nx = c->Hh / CUBE + 1, ny = c->Ww / CUBE + 1;"),
     "fusion_norm": ("out[d] = (os[d] / rp + g * olr[d]) * rp;", "out[d] = (os[d] + g * olr[d]) * rp;"),
     "rmsnorm_mean": ("double inv = 1.0 / sqrt(ss / (double)dh + c->eps_lr);",
                      "double inv = 1.0 / sqrt(ss + c->eps_lr);"),

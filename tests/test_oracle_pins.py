@@ -238,6 +238,87 @@ def test_sparse_with_mask_is_masked_sdpa(oracle):
     assert np.isnan(sel[:, :, :64]).all()
 
 
+# ---------------------------------------------------------------- cube blocks -
+
+def cube_ids(T, Hh, Ww):
+    """Cube of every token by numpy: (t // 4, x // 4, y // 4), numbered t-major over the cube grid."""
+    t, x, y = np.meshgrid(np.arange(T), np.arange(Hh), np.arange(Ww), indexing="ij")
+    nx, ny = -(-Hh // 4), -(-Ww // 4)
+    return (((t // 4) * nx + x // 4) * ny + y // 4).reshape(-1)
+
+
+def test_cube_blocks_partition_the_grid(oracle):
+    """Cube geometry: every token lies in exactly one 4 x 4 x 4 cube of the latent grid, the cube
+    count is the product of the per-axis cube counts, and an edge cube holds the product of its
+    per-axis extents min(4, extent - 4 c)."""
+    O = oracle
+    cfg = small_cfg(T=5, Hh=9, Ww=13, block_geometry="cube")
+    ids = O.block_of(cfg)
+    np.testing.assert_array_equal(ids, cube_ids(5, 9, 13))
+    assert O.num_blocks(cfg) == 2 * 3 * 4
+    ext = lambda n: [min(4, n - 4 * c) for c in range(-(-n // 4))]
+    want = np.array([a * b * c for a in ext(5) for b in ext(9) for c in ext(13)])
+    np.testing.assert_array_equal(np.bincount(ids, minlength=24), want)
+    assert O.num_keep(dict(cfg, keep=0.25)) == 6
+
+
+def test_cube_pooled_scores_by_numpy(oracle):
+    """Cube geometry: the block scores are the means of the rotated q / k over each cube's real
+    tokens (numpy bincount over the cube ids), dotted and scaled by 1/sqrt(d_h)."""
+    O = oracle
+    cfg = small_cfg(T=5, Hh=9, Ww=13, block_geometry="cube", keep=0.25)
+    x = draw(cfg)
+    _, scores, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    ids = cube_ids(5, 9, 13)
+    cnt = np.bincount(ids)
+    for h in range(cfg["H"]):
+        qr, kr = O.rope_full(cfg, x["q"])[0, h], O.rope_full(cfg, x["k"])[0, h]
+        qb = np.stack([np.bincount(ids, weights=qr[:, d]) for d in range(128)], axis=1) / cnt[:, None]
+        kb = np.stack([np.bincount(ids, weights=kr[:, d]) for d in range(128)], axis=1) / cnt[:, None]
+        np.testing.assert_allclose(scores[0, h], qb @ kb.T / math.sqrt(128), rtol=1e-11, atol=1e-13)
+
+
+def test_cube_keep_all_is_dense_and_mask_is_shift_invariant(oracle):
+    """Cube geometry at keep = 1 is dense attention (torch fp64 SDPA) whatever the tiling; the cube
+    scores, like the chunk scores, depend only on relative positions (Eq. shiftinv)."""
+    O = oracle
+    cfg = small_cfg(T=5, Hh=6, Ww=7, block_geometry="cube", keep=1.0)
+    x = draw(cfg)
+    qr, kr = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"])
+    idx, _, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    assert (idx == np.arange(O.num_blocks(cfg))).all()
+    got = O.sparse_attn(cfg, qr, kr, x["v"], idx)
+    np.testing.assert_allclose(got, sdpa64(qr, kr, x["v"]), rtol=1e-11, atol=1e-12)
+    cfg = dict(cfg, keep=0.3)
+    _, s0, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    _, s1, _, _ = O.block_mask(dict(cfg, pos_offset=(5, -3, 11)), x["q"], x["k"])
+    np.testing.assert_allclose(s1, s0, atol=1e-13)
+
+
+def test_cube_sparse_equals_chunks_of_the_cube_ordered_sequence(oracle):
+    """On a grid of whole cubes, sorting the tokens by cube turns every cube into one contiguous
+    64-token chunk: the cube-geometry sparse branch equals the chunk-geometry branch run on the
+    permuted q^r, k^r, v with the same block mask, permuted back."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=8, Ww=12, block_geometry="cube", keep=0.5)
+    x = draw(cfg)
+    qr, kr, v = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"]), x["v"]
+    nb = O.num_blocks(cfg)
+    assert nb == 6
+    rng = np.random.default_rng(5)
+    idx = np.sort(np.stack([[rng.choice(nb, 3, replace=False) for _ in range(nb)]
+                            for _ in range(cfg["H"])]), axis=-1)[None].astype(np.int32)
+    got = O.sparse_attn(cfg, qr, kr, v, idx)
+    perm = np.argsort(cube_ids(4, 8, 12), kind="stable")
+    flat = dict(cfg, block_geometry="flat")
+    pf = O.sparse_attn(flat, qr[:, :, perm], kr[:, :, perm], v[:, :, perm], idx)
+    back = np.empty_like(pf)
+    back[:, :, perm] = pf
+    np.testing.assert_allclose(got, back, rtol=1e-13, atol=1e-14)
+    # a random cube mask differs from the chunk mask on the unpermuted sequence
+    assert np.abs(got - O.sparse_attn(flat, qr, kr, v, idx)).max() > 1e-3
+
+
 # ---------------------------------------------------------------- low-rank ----
 
 def test_summary_form_equals_explicit_quadratic_form(oracle):
