@@ -52,14 +52,22 @@ def load_peaks():
 
 # ----------------------------------------------------------------- accounting
 
-def sparse_flops_from_mask(kv_idx, N, block=64, d_h=128):
+def block_sizes(cfg, block=64):
+    """Tokens per block: 64-token chunks (the last one ragged), or the real tokens of each
+    4 x 4 x 4 cube of the latent grid (edge cubes hold fewer)."""
+    if cfg.get("block_geometry", "flat") == "cube":
+        ext = lambda n: [min(4, n - 4 * c) for c in range(-(-n // 4))]
+        return [a * b * c for a in ext(cfg["T"]) for b in ext(cfg["Hh"]) for c in ext(cfg["Ww"])]
+    nB = -(-cfg["N"] // block)
+    return [block] * (nB - 1) + [cfg["N"] - (nB - 1) * block]
+
+
+def sparse_flops_from_mask(kv_idx, sizes, d_h=128):
     """Algorithmic FLOPs of the sparse branch: 4 d_h sum_{h,i} |Q_i| sum_{j kept} |K_j|
-    (QK^T and PV, 2 flops per multiply-add), with the ragged last block counted
-    at its real size (App. D, C_sparse = 4 B H L^2 (1-S) d_h)."""
+    (QK^T and PV, 2 flops per multiply-add), every block counted at its real size
+    (App. D, C_sparse = 4 B H L^2 (1-S) d_h)."""
     import torch
-    nB = kv_idx.shape[-2]
-    sizes = torch.full((nB,), block, dtype=torch.float64, device=kv_idx.device)
-    sizes[-1] = N - (nB - 1) * block
+    sizes = torch.tensor(sizes, dtype=torch.float64, device=kv_idx.device)
     keys = sizes[kv_idx.long()].sum(dim=-1)            # [B,H,nQB] kept keys per query block
     return float(4.0 * d_h * (keys * sizes).sum().item())
 
@@ -70,8 +78,9 @@ def lowrank_flops(B, H, N, d_h, r):
 
 
 # kernels one bf16 forward launches: RoPE table, fused pre-pass, block scores,
-# top-k, summary combine, sparse attention, readout + fusion
-LAUNCHES_PER_FORWARD = 7
+# top-k, summary combine, sparse attention, readout + fusion; with cube blocks
+# the pre-pass splits into the cube rotate + pool and the summary-only pre-pass
+LAUNCHES_PER_FORWARD = {"flat": 7, "cube": 8}
 
 
 def summary_bytes(B, H, N, d_h, esize=2):
@@ -156,7 +165,7 @@ def cpu_oracle_estimate(cfg, heads=None, q_lo=8, q_hi=96):
     O.build()
     cores = os.cpu_count() or 1
     heads = heads or min(cfg["H"], cores)
-    nB = (cfg["N"] + cfg["block"] - 1) // cfg["block"]
+    nB = len(block_sizes(cfg, cfg["block"]))
     t_lo = oracle_sample_time(cfg, heads, list(range(q_lo)))
     t_hi = oracle_sample_time(cfg, heads, list(range(q_hi)))
     per_block = max(t_hi - t_lo, 0.0) / (q_hi - q_lo)
@@ -283,6 +292,8 @@ def main():
     ap.add_argument("--workload", default="wan14b_720p")
     ap.add_argument("--keep", type=float, default=None)
     ap.add_argument("--r", type=int, default=None)
+    ap.add_argument("--geometry", default=None, choices=["flat", "cube"],
+                    help="blocks of the sparse branch: 64-token chunks (default) or 4x4x4 cubes of the latent grid")
     ap.add_argument("--lowrank-act", default=None, choices=["silu", "identity", "tanh", "relu", "gelu"],
                     help="feature map of the low-rank branch (the activation ablation); default SiLU")
     ap.add_argument("--no-dense", action="store_true")
@@ -305,6 +316,8 @@ def main():
         cfg = configs.get(args.workload, **over)
     if args.lowrank_act is not None:
         cfg["lowrank_act"] = args.lowrank_act
+    if args.geometry is not None:
+        cfg["block_geometry"] = args.geometry
     ws, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, cfg, ws, rank)
@@ -369,12 +382,13 @@ def main():
 
     # ---- roofline of the dominant kernel (the sparse branch: tensor-core bound)
     peaks, peak_src = load_peaks()
-    fl = sparse_flops_from_mask(kv, cfg["N"])
+    geometry = cfg.get("block_geometry", "flat")
+    fl = sparse_flops_from_mask(kv, block_sizes(cfg))
     sp_ms = stage_ms["sparse_attn"]
     achieved = fl / (sp_ms * 1e-3) / 1e12
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
     traffic = None
-    if SPARSE_TRAFFIC_PER_HEAD_TOKEN is not None:
+    if SPARSE_TRAFFIC_PER_HEAD_TOKEN is not None and geometry == "flat":
         traffic = SPARSE_TRAFFIC_PER_HEAD_TOKEN * cfg["B"] * cfg["H"] * cfg["N"]
     roofline = {"bound": "tensor", "kernel": "sparse_attn", "achieved": achieved, "peak": peak,
                 "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
@@ -383,13 +397,19 @@ def main():
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     tensor_bytes = summary_bytes(cfg["B"], cfg["H"], cfg["N"], 128) / 2      # one [B,H,N,128] bf16 tensor
     pre_bytes = 5 * tensor_bytes                                                # read q, k, v; write q^r, k^r
+    pre_note = ("bytes = read q, k, v once + write the rotated q^r, k^r the sparse branch reads; "
+                "algorithmic_bytes = the reads alone")
+    if geometry == "cube":
+        # cube rotate + pool: read q, k, v, write q^r, k^r, v in padded cube order; then the summary reads k, v
+        pad = nB * 64 / cfg["N"]
+        pre_bytes = (3 + 3 * pad + 2) * tensor_bytes
+        pre_note = ("cube geometry: read q, k, v + write q^r, k^r, v in padded cube order (x%.3f) + the "
+                    "summary's second read of k, v; algorithmic_bytes = one read of q, k, v" % pad)
     select_flops = 2.0 * cfg["B"] * cfg["H"] * nB * nB * 128
     secondary = {
         "prepass": {"bound": "hbm", "achieved_gbs": pre_bytes / (stage_ms["prepass"] * 1e-3) / 1e9,
                     "peak_gbs": hbm, "frac": pre_bytes / (stage_ms["prepass"] * 1e-3) / 1e9 / hbm,
-                    "bytes": pre_bytes, "algorithmic_bytes": 3 * tensor_bytes,
-                    "note": "bytes = read q, k, v once + write the rotated q^r, k^r the sparse branch reads; "
-                            "algorithmic_bytes = the reads alone"},
+                    "bytes": pre_bytes, "algorithmic_bytes": 3 * tensor_bytes, "note": pre_note},
         "select": {"bound": "fp32", "ms": stage_ms["select"], "flops": select_flops,
                    "achieved_tflops": select_flops / (stage_ms["select"] * 1e-3) / 1e12,
                    "note": "block scores (fp32 FMA) + per-row top-k + summary combine"},
@@ -515,7 +535,7 @@ def main():
         t3.record(stream)
         torch.cuda.synchronize()
         d_ms = s3.elapsed_time(t3) / 2
-        flop_ratio = (sparse_flops_from_mask(kvd, cfg["N"]) + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"])) / \
+        flop_ratio = (sparse_flops_from_mask(kvd, block_sizes(cfg)) + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"])) / \
             (fl + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"]))
         dense = {"dense_ms": d_ms, "speedup": d_ms / ms_step, "flop_ratio": flop_ratio,
                  "target_speedup": 0.85 * flop_ratio}
@@ -533,6 +553,7 @@ def main():
             "config": {"workload": cfg["name"], "B": cfg["B"], "H": cfg["H"], "N": cfg["N"],
                        "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "block": 64, "keep": cfg["keep"],
                        "n_keep": nk, "r": cfg["r"], "d_h": 128, "lowrank_act": cfg.get("lowrank_act", "silu"),
+                       "block_geometry": cfg.get("block_geometry", "flat"),
                        "l2": "no flush: q, k, v are each larger than L2 (774 MB vs 129 MB)",
                        "parallelism": f"replica per GPU x{ws}"},
             "stage_ms": stage_ms,
@@ -542,7 +563,7 @@ def main():
             "dense": dense,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": LAUNCHES_PER_FORWARD * K,
+            "gpu_launches": LAUNCHES_PER_FORWARD[geometry] * K,
             "clocks": clk,
         }
         print(json.dumps(line), flush=True)

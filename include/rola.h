@@ -39,7 +39,9 @@
  *              must be ordered on one stream.
  *   Errors     argument validation happens on the host before any launch
  *              and returns ROLA_ERR_INVALID_ARG / ROLA_ERR_UNSUPPORTED /
- *              ROLA_ERR_WORKSPACE with nothing launched; a launch failure
+ *              ROLA_ERR_WORKSPACE with nothing launched (UNSUPPORTED also
+ *              for shapes past the kernels' limits: B*H > 65535, more than
+ *              7008 blocks, B*H*nB*n_keep >= 2^31); a launch failure
  *              returns ROLA_ERR_CUDA.  A device-side bounded wait that gives
  *              up records ROLA_ERR_TIMEOUT in the workspace status word,
  *              which rola_get_device_status reads.  No C++ exception
@@ -96,6 +98,8 @@ typedef struct {
                                   rola_lowrank_rope_t, default ROLA_LOWRANK_ROPE_OUTSIDE */
     int32_t lowrank_act;       /* feature map phi of the low-rank features; one of
                                   rola_lowrank_act_t, default ROLA_LOWRANK_ACT_SILU */
+    int32_t block_geometry;    /* which tokens form a block of the sparse branch; one of
+                                  rola_block_geometry_t, default ROLA_BLOCK_FLAT */
 } rola_config_t;
 
 #define ROLA_DEBUG_SKIP_FIRST_K_COPY 1
@@ -133,10 +137,27 @@ typedef enum {
     ROLA_LOWRANK_ACT_GELU = 4
 } rola_lowrank_act_t;
 
+/*
+ * Block geometry of the sparse branch (the paper does not describe it):
+ *   FLAT  block i = tokens 64 i .. 64 i + 63 of the t-major sequence (the
+ *         last block ragged); nQB = nKB = ceil(N / 64)
+ *   CUBE  block i = the 4 x 4 x 4 cube (ct, cx, cy) of the latent grid,
+ *         i = (ct * ceil(Hh/4) + cx) * ceil(Ww/4) + cy, holding the tokens
+ *         (t, x, y) with t / 4 = ct, x / 4 = cx, y / 4 = cy (edge cubes hold
+ *         fewer); nQB = nKB = ceil(T/4) ceil(Hh/4) ceil(Ww/4)
+ * Block means, scores, kv_idx and the sparse branch all use the blocks of
+ * the configured geometry; the low-rank branch does not depend on it.
+ */
+typedef enum {
+    ROLA_BLOCK_FLAT = 0,
+    ROLA_BLOCK_CUBE = 1
+} rola_block_geometry_t;
+
 /* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
 rola_status_t rola_config_init(rola_config_t* cfg);
 
-/* ceil(N / block): the number of query blocks nQB, equal to the number of key blocks nKB. */
+/* The number of query blocks nQB, equal to the number of key blocks nKB: ceil(N / block), or
+ * the cube count for ROLA_BLOCK_CUBE; 0 if cfg is invalid. */
 int32_t rola_num_blocks(const rola_config_t* cfg);
 
 /* Kept key blocks per query block, clamp(floor(keep_ratio*nKB + 0.5), 1, nKB); 0 if cfg is invalid. */
@@ -149,7 +170,8 @@ size_t rola_workspace_bytes(const rola_config_t* cfg);
 
 /*
  * Kernel (1): block mask.  Rotates q and k by the full 3D RoPE R(p)
- * (Sec. 3, Eq. shiftinv), mean-pools each 64-token block, scores every
+ * (Sec. 3, Eq. shiftinv), mean-pools each block (of cfg->block_geometry)
+ * over its tokens, scores every
  * (query block, key block) pair as q_bar . k_bar / sqrt(d_h) and keeps the
  * n_keep highest-scoring key blocks of each query block (Alg. 1, "topk
  * ratio"; the pooling / scoring rule is this library's reading of the

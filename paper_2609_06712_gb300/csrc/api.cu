@@ -8,7 +8,18 @@ using namespace rola;
 
 namespace rola {
 
-int num_blocks_of(const rola_config_t& c) { return (int)(((int64_t)c.N + c.block - 1) / c.block); }
+int num_blocks_of(const rola_config_t& c)
+{
+    if (c.block_geometry == ROLA_BLOCK_CUBE)
+        return ((c.T + 3) / 4) * ((c.Hh + 3) / 4) * ((c.Ww + 3) / 4);
+    return (int)(((int64_t)c.N + c.block - 1) / c.block);
+}
+
+// Rows per head of the block-ordered copies q^r, k^r (and v in cube geometry).
+int64_t block_rows_of(const rola_config_t& c)
+{
+    return c.block_geometry == ROLA_BLOCK_CUBE ? (int64_t)num_blocks_of(c) * c.block : c.N;
+}
 
 int num_keep_of(const rola_config_t& c)
 {
@@ -45,11 +56,16 @@ rola_status_t validate(const rola_config_t* c)
     if (c->lowrank_rope < ROLA_LOWRANK_ROPE_OUTSIDE || c->lowrank_rope > ROLA_LOWRANK_ROPE_NONE)
         return ROLA_ERR_INVALID_ARG;
     if (c->lowrank_act < ROLA_LOWRANK_ACT_SILU || c->lowrank_act > ROLA_LOWRANK_ACT_GELU) return ROLA_ERR_INVALID_ARG;
+    if (c->block_geometry != ROLA_BLOCK_FLAT && c->block_geometry != ROLA_BLOCK_CUBE) return ROLA_ERR_INVALID_ARG;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
+    // the top-k kernel holds a row of nB keys per warp in shared memory (8 warps, 227 KB)
+    if (num_blocks_of(*c) > kMaxBlocks) return ROLA_ERR_UNSUPPORTED;
     // the sparse kernel counts a CTA's kept blocks in 32 bits (ring slots and phases)
     if ((int64_t)c->B * c->H * num_blocks_of(*c) * num_keep_of(*c) >= ((int64_t)1 << 31)) return ROLA_ERR_UNSUPPORTED;
     if ((int64_t)c->B * c->H * c->N * c->d_h > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
+    // cube geometry: the padded block-ordered rows of a head stay addressable in int
+    if (block_rows_of(*c) > ((int64_t)1 << 30)) return ROLA_ERR_UNSUPPORTED;
     return ROLA_OK;
 }
 
@@ -59,6 +75,7 @@ Shape make_shape(const rola_config_t& c)
     s.B = c.B; s.H = c.H; s.N = c.N; s.r = c.r;
     s.rp = (c.r + 15) & ~15;
     s.nB = num_blocks_of(c);
+    s.nC = (int)(((int64_t)c.N + kBlock - 1) / kBlock);
     s.n_keep = num_keep_of(c);
     s.T = c.T; s.Hh = c.Hh; s.Ww = c.Ww;
     s.pt = c.rope_split[0] / 2;
@@ -71,6 +88,12 @@ Shape make_shape(const rola_config_t& c)
     s.debug_flags = c.debug_flags;
     s.lr_rope = c.lowrank_rope;
     s.lr_act = c.lowrank_act;
+    s.cube = c.block_geometry == ROLA_BLOCK_CUBE;
+    s.nCh = (c.Hh + 3) / 4;
+    s.nCw = (c.Ww + 3) / 4;
+    s.Np = (int)block_rows_of(c);
+    s.rcp_plane = (float)(1.0 / ((double)s.nCh * s.nCw));
+    s.rcp_nCw = (float)(1.0 / (double)s.nCw);
     return s;
 }
 
@@ -94,8 +117,9 @@ Workspace layout(const rola_config_t& c)
     size_t off = 0;
     w.status = off; off = align_up(off + sizeof(DeviceStatus));
     w.table = off; off = align_up(off + sizeof(float2) * (size_t)(c.T + c.Hh + c.Ww) * kPairs);
-    w.qr = off; off = align_up(off + esz * bh * c.N * kDh);
-    w.kr = off; off = align_up(off + esz * bh * c.N * kDh);
+    w.qr = off; off = align_up(off + esz * bh * s.Np * kDh);
+    w.kr = off; off = align_up(off + esz * bh * s.Np * kDh);
+    w.vp = off; off = align_up(off + (s.cube ? esz * bh * s.Np * kDh : 0));   // v in block order (cube)
     w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.scores = off; off = align_up(off + 4 * bh * s.nB * s.nB);
@@ -104,7 +128,7 @@ Workspace layout(const rola_config_t& c)
     w.z = off; off = align_up(off + 4 * bh * c.r);
     w.Cbf = off; off = align_up(off + 2 * bh * s.rp * kDh);           // zero-padded to rp rows
     // summary partials: fp32 split-N slots, or the bf16 pre-pass's per-(CTA, head) slots
-    const size_t units = bh * s.nB;
+    const size_t units = bh * s.nC;          // the pre-pass works on 64-token chunks
     w.prepass_slots = (units < (size_t)kMaxPrepassCtas ? units : (size_t)kMaxPrepassCtas) + bh - 1;
     const size_t slots = c.dtype == ROLA_BF16 ? w.prepass_slots : bh * w.nsplit;
     w.partials = off; off = align_up(off + 4 * slots * ((size_t)s.rp * kDh + s.rp));
@@ -159,11 +183,24 @@ rola_status_t run_summary(const rola_config_t& c, const Shape& s, const Workspac
     return ROLA_OK;
 }
 
-rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& w, const void* q, const void* k,
-                       int32_t* kv_idx, void* ws, cudaStream_t st)
+// q^r, k^r and the block means; v in block order too when v is given and the geometry is cubes.
+cudaError_t rope_pool(const rola_config_t& c, const Shape& s, const Workspace& w, const void* q, const void* k,
+                      const void* v, void* ws, cudaStream_t st)
 {
-    ROLA_TRY(launch_rope_pool(c, s, q, k, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
-                              at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
+    return launch_rope_pool(c, s, q, k, s.cube ? v : nullptr, at<float2>(ws, w.table), at<void>(ws, w.qr),
+                            at<void>(ws, w.kr), at<void>(ws, w.vp), at<float>(ws, w.qbar), at<float>(ws, w.kbar), st);
+}
+
+// The v rows the sparse kernels read: the caller's v, or its block-ordered copy in cube geometry.
+const void* sparse_v(const Shape& s, const Workspace& w, const void* v, void* ws)
+{
+    return s.cube ? at<void>(ws, w.vp) : v;
+}
+
+rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& w, const void* q, const void* k,
+                       const void* v, int32_t* kv_idx, void* ws, cudaStream_t st)
+{
+    ROLA_TRY(rope_pool(c, s, w, q, k, v, ws, st));
     ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv_idx,
                                st));
     return ROLA_OK;
@@ -220,7 +257,7 @@ rola_status_t rola_block_mask(const rola_config_t* cfg, const void* q, const voi
     Workspace w = layout(*cfg);
     Shape s = make_shape(*cfg);
     ROLA_CHECK(prologue(*cfg, ws, w, st));
-    return run_mask(*cfg, s, w, q, k, kv_idx, ws, st);
+    return run_mask(*cfg, s, w, q, k, nullptr, kv_idx, ws, st);
 }
 
 rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const void* k, const void* v,
@@ -235,11 +272,10 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
     Workspace w = layout(*cfg);
     Shape s = make_shape(*cfg);
     ROLA_CHECK(prologue(*cfg, ws, w, st));
-    // rotated copies (the pooled means are a by-product here)
-    ROLA_TRY(launch_rope_pool(*cfg, s, q, k, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
-                              at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
-    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv_idx, o_s,
-                                at<DeviceStatus>(ws, w.status), st));
+    // rotated copies in block order (the pooled means are a by-product here)
+    ROLA_TRY(rope_pool(*cfg, s, w, q, k, v, ws, st));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), sparse_v(s, w, v, ws), kv_idx,
+                                o_s, at<DeviceStatus>(ws, w.status), st));
     return ROLA_OK;
 }
 
@@ -297,7 +333,21 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
     int32_t* kv = kv_idx_out ? kv_idx_out : at<int32_t>(ws, w.kv_idx);
     ROLA_TRY(mark(0));
     ROLA_CHECK(prologue(*cfg, ws, w, st));
-    if (cfg->dtype == ROLA_BF16) {
+    if (cfg->dtype == ROLA_BF16 && s.cube) {
+        // stage 1: q^r, k^r, v in cube order and the cube means, then the summary
+        // partials (the fused pre-pass pools contiguous chunks only);
+        // stage 2: block scores + top-k, and the summary combine
+        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        ROLA_TRY(rope_pool(*cfg, s, w, q, k, v, ws, st));
+        ROLA_TRY(launch_prepass(s, ctas, nullptr, k, v, P_k, at<float2>(ws, w.table), nullptr, nullptr, nullptr,
+                                nullptr, at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
+        ROLA_TRY(mark(1));
+        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
+                                   st));
+        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
+                                        at<__nv_bfloat16>(ws, w.Cbf), st));
+    } else if (cfg->dtype == ROLA_BF16) {
         // stage 1: one pass over q, k, v -> q^r, k^r, block means, summary partials;
         // stage 2: block scores + top-k, and the summary combine
         const int ctas = prepass_ctas(s, kMaxPrepassCtas);
@@ -312,13 +362,13 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                         at<__nv_bfloat16>(ws, w.Cbf), st));
     } else {
         // stage 1: the block mask; stage 2: the summary
-        ROLA_CHECK(run_mask(*cfg, s, w, q, k, kv, ws, st));
+        ROLA_CHECK(run_mask(*cfg, s, w, q, k, v, kv, ws, st));
         ROLA_TRY(mark(1));
         ROLA_CHECK(run_summary(*cfg, s, w, k, v, P_k, at<float>(ws, w.C), at<float>(ws, w.z),
                                at<__nv_bfloat16>(ws, w.Cbf), ws, st));
     }
     ROLA_TRY(mark(2));
-    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), v, kv, o,
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), sparse_v(s, w, v, ws), kv, o,
                                 at<DeviceStatus>(ws, w.status), st));
     ROLA_TRY(mark(3));
     ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, o,

@@ -31,7 +31,8 @@ struct DeviceStatus {
 
 // Kernel-side view of a validated configuration.
 struct Shape {
-    int B, H, N, nB, n_keep, r;
+    int B, H, N, nB, n_keep, r;   // nB: blocks of the sparse branch (chunks or cubes)
+    int nC;                   // 64-token chunks ceil(N / 64): the units of the low-rank kernels
     int rp;                   // r rounded up to a multiple of 16: the width the bf16 kernels run at
                               // (rows r .. rp-1 of P are read as zero, so those features are zero)
     int T, Hh, Ww;
@@ -43,7 +44,46 @@ struct Shape {
     int debug_flags;          // ROLA_DEBUG_* test hooks
     int lr_rope;              // rola_lowrank_rope_t
     int lr_act;               // rola_lowrank_act_t
+    int cube;                 // block geometry: 0 contiguous 64-token chunks, 1 4x4x4 cubes
+    int nCh, nCw;             // cubes along the row / column axis (cube geometry)
+    int Np;                   // rows per head of the block-ordered copies q^r, k^r (and v):
+                              // N, or nB * 64 in cube geometry (a cube's slots, padded)
+    float rcp_plane, rcp_nCw; // fp32 1 / (nCh * nCw) and 1 / nCw (cube_origin_rcp)
 };
+
+// Most blocks per sequence: the top-k kernel keeps one row of nB 32-bit keys per
+// warp (8 warps) beside 8 KB of scratch in 227 KB of shared memory.
+constexpr int kMaxBlocks = 7008;
+
+// Cube geometry: block b is the cube (ct, cx, cy) = t-major index b over the
+// cube grid; its slot i = 16 dt + 4 dx + dy holds token (4ct+dt, 4cx+dx, 4cy+dy)
+// when that lies inside the grid.
+struct CubeOrigin {
+    int t, x, y;
+};
+__host__ __device__ __forceinline__ CubeOrigin cube_origin(const Shape& s, int b)
+{
+    const int per_t = s.nCh * s.nCw;
+    const int ct = b / per_t, rem = b - ct * per_t, cx = rem / s.nCw;
+    return {4 * ct, 4 * cx, 4 * (rem - cx * s.nCw)};
+}
+// cube_origin with both divisions done as a multiply by the fp32 reciprocal:
+// floor((a + 0.5) * fl(1/d)) equals a / d exactly whenever a < 2^22, because the
+// product's error, below (a + 0.5) / d * 2^-23, stays under the distance 0.5 / d
+// from (a + 0.5) / d to the nearest integer (block ids are below kMaxBlocks).
+__device__ __forceinline__ CubeOrigin cube_origin_rcp(const Shape& s, int b)
+{
+    const int ct = __float2int_rz(__fmul_rn((float)b + 0.5f, s.rcp_plane));
+    const int rem = b - ct * (s.nCh * s.nCw);
+    const int cx = __float2int_rz(__fmul_rn((float)rem + 0.5f, s.rcp_nCw));
+    return {4 * ct, 4 * cx, 4 * (rem - cx * s.nCw)};
+}
+// Flat index of the token in slot i of the cube at o, or -1 outside the grid.
+__host__ __device__ __forceinline__ int cube_token(const Shape& s, CubeOrigin o, int i)
+{
+    const int t = o.t + (i >> 4), x = o.x + ((i >> 2) & 3), y = o.y + (i & 3);
+    return (t < s.T && x < s.Hh && y < s.Ww) ? (t * s.Hh + x) * s.Ww + y : -1;
+}
 
 // Rotation (cos, sin) of pair m for the token at flat index n.
 __device__ __forceinline__ float2 rope_cs(const float2* __restrict__ tab, const Shape& s, int n, int m)
@@ -83,16 +123,18 @@ __device__ __forceinline__ float2 lowrank_pair(float u0, float u1, float2 cs, in
 
 // Workspace carve-up for one configuration.
 struct Workspace {
-    size_t status, table, qr, kr, qbar, kbar, scores, kv_idx, C, z, Cbf, partials, total;
+    size_t status, table, qr, kr, vp, qbar, kbar, scores, kv_idx, C, z, Cbf, partials, total;
     int nsplit;               // fp32 summary splits
     size_t prepass_slots;     // bf16 pre-pass partial slots
 };
 
 // Host launchers, one per kernel family.  All return cudaGetLastError().
 cudaError_t launch_rope_table(const rola_config_t& cfg, float2* tab, cudaStream_t st);
+// q^r, k^r (rows in block order, Np per head) and the block means; in cube
+// geometry also v copied into block order (vp) when v is given.
 cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k,
-                             const float2* tab, void* qr, void* kr, float* qbar, float* kbar,
-                             cudaStream_t st);
+                             const void* v, const float2* tab, void* qr, void* kr, void* vp, float* qbar,
+                             float* kbar, cudaStream_t st);
 cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
                               int32_t* kv_idx, cudaStream_t st);
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr,

@@ -236,7 +236,7 @@ cudaError_t launch_lowrank_apply(rola_dtype_t dt, const Shape& s, const void* q,
                                    kBlock * (s.r + 1));
     cudaError_t e = cudaFuncSetAttribute(apply_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    apply_f32_kernel<<<dim3(s.nB, s.B * s.H), 256, smem, st>>>(s, (const float*)q, (const float*)P_q, C, gate,
+    apply_f32_kernel<<<dim3(s.nC, s.B * s.H), 256, smem, st>>>(s, (const float*)q, (const float*)P_q, C, gate,
                                                               (const float*)o_s, (float*)o, tab);
     return cudaGetLastError();
 }

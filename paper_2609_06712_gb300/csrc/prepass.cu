@@ -94,7 +94,7 @@ struct Params {
     float* kbar;
     float* partials;
     DeviceStatus* status;
-    int units;                    // B * H * nB
+    int units;                    // B * H * nC
 };
 
 __device__ __forceinline__ void record_timeout(const Params& p, int where)
@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     // warps 0, 1, 2 issue the k, v, q boxes; thread 0 also arms the barrier
     const uint32_t bytes = fuse ? 3 * kHalf : 2 * kHalf;
     auto issue = [&](int j) {
-        const int u = u0 + (j >> 1), bh = u / s.nB, row = (u - bh * s.nB) * 64 + (j & 1) * kHalfRows;
+        const int u = u0 + (j >> 1), bh = u / s.nC, row = (u - bh * s.nC) * 64 + (j & 1) * kHalfRows;
         const uint32_t dst = sbase + (j % S) * lay.stage_bytes, bar = full0 + 8 * (j % S);
         if (tid == 0) {
             mbar_expect_tx(bar, bytes);
@@ -270,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     // the start of the range, since consecutive units are consecutive blocks)
     int kt_t, kt_x, kt_y, rt_t, rt_x, rt_y;
     {
-        const int blk0 = u0 - (u0 / s.nB) * s.nB;
+        const int blk0 = u0 - (u0 / s.nC) * s.nC;
         position(blk0 * kBlock + mt * 16 + g, kt_t, kt_x, kt_y);
         position(blk0 * kBlock + rs, rt_t, rt_x, rt_y);
     }
@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     int i = 0;                                      // half-stage index
     for (; i < count; ++i) {
         const int u = u0 + (i >> 1), h = i & 1;
-        const int bh = u / s.nB, blk = u - bh * s.nB;
+        const int bh = u / s.nC, blk = u - bh * s.nC;
         const int st = i % S, buf = i & 1;
         if (h == 0 && bh != hb) {
             if (hb >= 0) {
@@ -421,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
 #pragma unroll
             for (int r = 0; r < 16; ++r) sum += src[r * kDh];
             const int cnt = min(kBlock, s.N - blk * kBlock);
-            (which ? p.kbar : p.qbar)[((size_t)bh * s.nB + blk) * kDh + d] = sum / (float)cnt;
+            (which ? p.kbar : p.qbar)[((size_t)bh * s.nC + blk) * kDh + d] = sum / (float)cnt;
         }
         // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 32 tokens
 #pragma unroll
@@ -458,8 +458,8 @@ __global__ void prepass_combine_kernel(Shape s, int ctas, int units, const float
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= per) return;
     // CTAs whose unit ranges meet head bh: those holding its first and last unit, and all between
-    const int c0 = (int)((((long long)bh * s.nB + 1) * ctas - 1) / units);
-    const int c1 = (int)((((long long)(bh + 1) * s.nB) * ctas - 1) / units);
+    const int c0 = (int)((((long long)bh * s.nC + 1) * ctas - 1) / units);
+    const int c1 = (int)((((long long)(bh + 1) * s.nC) * ctas - 1) / units);
     float x = 0.0f;
     for (int c = c0; c <= c1; ++c) x += partials[(size_t)(c + bh) * per + e];
     // C and z have r rows; the bf16 copy keeps all rp (rows past r are exactly zero)
@@ -499,7 +499,7 @@ int prepass_ctas(const Shape& s, int max_ctas)
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) !=
                                                    cudaSuccess)
         return 0;
-    const long long units = (long long)s.B * s.H * s.nB;
+    const long long units = (long long)s.B * s.H * s.nC;
     long long g = (long long)nsm * (s.rp <= 48 ? 2 : 1);     // CTAs per SM as Cfg<R>::kCtasPerSm
     if (g > max_ctas) g = max_ctas;
     if (g > kMaxPrepassCtas) g = kMaxPrepassCtas;
@@ -511,7 +511,7 @@ cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* 
                            const void* P_k, const float2* tab, void* qr, void* kr, float* qbar, float* kbar,
                            float* partials, DeviceStatus* status, cudaStream_t st)
 {
-    if (ctas <= 0 || ctas > kMaxPrepassCtas || ctas > s.B * s.H * s.nB) return cudaErrorInvalidValue;
+    if (ctas <= 0 || ctas > kMaxPrepassCtas || ctas > s.B * s.H * s.nC) return cudaErrorInvalidValue;
     const bool fuse = q != nullptr;
     CUtensorMap mq, mk, mv;
     if (!make_block_map(&mk, k, s, kHalfRows) || !make_block_map(&mv, v, s, kHalfRows)) return cudaErrorInvalidValue;
@@ -530,7 +530,7 @@ cudaError_t launch_prepass(const Shape& s, int ctas, const void* q, const void* 
     p.kbar = kbar;
     p.partials = partials;
     p.status = status;
-    p.units = s.B * s.H * s.nB;
+    p.units = s.B * s.H * s.nC;
     switch (s.rp) {
         case 16: return launch_r<16>(mq, mk, mv, p, ctas, fuse, st);
         case 32: return launch_r<32>(mq, mk, mv, p, ctas, fuse, st);
@@ -548,7 +548,7 @@ cudaError_t launch_prepass_combine(const Shape& s, int ctas, const float* partia
                                    __nv_bfloat16* Cbf, cudaStream_t st)
 {
     const int per = s.rp * kDh + s.rp;
-    const int units = s.B * s.H * s.nB;
+    const int units = s.B * s.H * s.nC;
     prepass_combine_kernel<<<dim3((per + 255) / 256, s.B * s.H), 256, 0, st>>>(s, ctas, units, partials, C, z, Cbf);
     return cudaGetLastError();
 }

@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(c
     // loads of the j-th unit into stage j % S, by thread 0 (the thread that
     // stores, so that its bulk-group waits order a refill after the store)
     auto issue = [&](int j) {
-        const int u = u0 + j, bh = u / s.nB, blk = u - bh * s.nB, st = j % kStages;
+        const int u = u0 + j, bh = u / s.nC, blk = u - bh * s.nC, st = j % kStages;
         const uint32_t dst = sbase + st * L::stage_bytes, bar = full0 + 8 * st;
         if (tid == 0) {
             mbar_expect_tx(bar, 2 * kBox);
@@ -135,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, Occupancy<R>::ctas) readout_kernel(c
     bool failed = false;
     int i = 0;
     for (int u = u0; u < u1; ++u, ++i) {
-        const int bh = u / s.nB, blk = u - bh * s.nB, b = bh / s.H;
+        const int bh = u / s.nC, blk = u - bh * s.nC, b = bh / s.H;
         const int st = i % kStages;
         if (bh != hb) {
             // P_q of the head and C of (batch, head); every reader of the old ones has passed the last barrier
@@ -352,7 +352,7 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
                            const float* gate, const void* o_s, void* o, const float2* tab, DeviceStatus* status,
                            cudaStream_t st)
 {
-    const int units = s.B * s.H * s.nB;
+    const int units = s.B * s.H * s.nC;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;

@@ -157,18 +157,104 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
     }
 }
 
-cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k,
-                             const float2* tab, void* qr, void* kr, float* qbar, float* kbar, cudaStream_t st)
+// ---------------------------------------------------------------------------
+// The same pass in cube geometry: one CTA per (cube, head, q|k|v).  Thread
+// (rsub, c8) handles slot rsub + 16 dt of the cube for dt = 0..3, i.e. grid
+// position (t0 + dt, x0 + rsub / 4, y0 + rsub % 4).  The rotated rows are
+// written in block order (row 64 b + slot of the head's Np rows, zeros for
+// slots outside the grid, so that the sparse kernels read finite values
+// there); the v slice copies v into the same order without rotating it.
+
+template <typename T>
+__global__ void __launch_bounds__(256) rope_pool_cube_kernel(Shape s, const T* __restrict__ q,
+                                                             const T* __restrict__ k, const T* __restrict__ v,
+                                                             const float2* __restrict__ tab, T* __restrict__ qr,
+                                                             T* __restrict__ kr, T* __restrict__ vp,
+                                                             float* __restrict__ qbar, float* __restrict__ kbar)
 {
-    dim3 grid(s.nB, s.B * s.H, 2);
-    if (cfg.dtype == ROLA_BF16)
-        rope_pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-            s, (const __nv_bfloat16*)q, (const __nv_bfloat16*)k, tab, (__nv_bfloat16*)qr, (__nv_bfloat16*)kr,
-            qbar, kbar);
-    else
-        rope_pool_kernel<float><<<grid, 256, 0, st>>>(s, (const float*)q, (const float*)k, tab, (float*)qr,
-                                                      (float*)kr, qbar, kbar);
+    __shared__ float part[16][kDh];
+    const int blk = blockIdx.x, bh = blockIdx.y, z = blockIdx.z;
+    const T* x = z == 0 ? q : (z == 1 ? k : v);
+    T* xr = z == 0 ? qr : (z == 1 ? kr : vp);
+    const int c8 = threadIdx.x & 15;
+    const int rsub = threadIdx.x >> 4;
+    constexpr int kPasses = kBlock / 16;
+    const CubeOrigin o = cube_origin(s, blk);
+    float v8[kPasses][8];
+#pragma unroll
+    for (int dt = 0; dt < kPasses; ++dt) {
+        const int n = cube_token(s, o, rsub + 16 * dt);
+        if (n >= 0) Vec8<T>::load(x + ((size_t)bh * s.N + n) * kDh + c8 * 8, v8[dt]);
+    }
+    int axis[4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+        const int m = c8 * 4 + p;
+        axis[p] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
+    }
+    const int xx = o.x + (rsub >> 2), yy = o.y + (rsub & 3);
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+    for (int dt = 0; dt < kPasses; ++dt) {
+        const int slot = rsub + 16 * dt;
+        const int n = cube_token(s, o, slot);
+        float out[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (n >= 0) {
+            if (z == 2) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) out[i] = v8[dt][i];
+            } else {
+                const int t = o.t + dt;
+#pragma unroll
+                for (int p = 0; p < 4; ++p) {
+                    const int row = axis[p] == 0 ? t : (axis[p] == 1 ? s.T + xx : s.T + s.Hh + yy);
+                    const float2 cs = __ldg(tab + row * kPairs + c8 * 4 + p);
+                    const float2 y = rope_rotate(v8[dt][2 * p], v8[dt][2 * p + 1], cs);
+                    out[2 * p] = y.x;
+                    out[2 * p + 1] = y.y;
+                }
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] += out[i];
+            }
+        }
+        Vec8<T>::store(xr + ((size_t)bh * s.Np + (size_t)blk * kBlock + slot) * kDh + c8 * 8, out);
+    }
+    if (z == 2) return;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) part[rsub][c8 * 8 + i] = acc[i];
+    __syncthreads();
+    if (threadIdx.x < kDh) {
+        float sum = 0.0f;
+#pragma unroll
+        for (int r = 0; r < 16; ++r) sum += part[r][threadIdx.x];
+        const int cnt = min(4, s.T - o.t) * min(4, s.Hh - o.x) * min(4, s.Ww - o.y);
+        (z == 0 ? qbar : kbar)[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = sum / (float)cnt;
+    }
+}
+
+template <typename T>
+cudaError_t launch_rope_pool_t(const Shape& s, const void* q, const void* k, const void* v, const float2* tab,
+                               void* qr, void* kr, void* vp, float* qbar, float* kbar, cudaStream_t st)
+{
+    if (s.cube) {
+        dim3 grid(s.nB, s.B * s.H, v ? 3 : 2);
+        rope_pool_cube_kernel<T><<<grid, 256, 0, st>>>(s, (const T*)q, (const T*)k, (const T*)v, tab, (T*)qr,
+                                                       (T*)kr, (T*)vp, qbar, kbar);
+    } else {
+        dim3 grid(s.nB, s.B * s.H, 2);
+        rope_pool_kernel<T><<<grid, 256, 0, st>>>(s, (const T*)q, (const T*)k, tab, (T*)qr, (T*)kr, qbar, kbar);
+    }
     return cudaGetLastError();
+}
+
+cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k, const void* v,
+                             const float2* tab, void* qr, void* kr, void* vp, float* qbar, float* kbar,
+                             cudaStream_t st)
+{
+    if (s.cube && v && !vp) return cudaErrorInvalidValue;
+    return cfg.dtype == ROLA_BF16
+               ? launch_rope_pool_t<__nv_bfloat16>(s, q, k, v, tab, qr, kr, vp, qbar, kbar, st)
+               : launch_rope_pool_t<float>(s, q, k, v, tab, qr, kr, vp, qbar, kbar, st);
 }
 
 }  // namespace rola

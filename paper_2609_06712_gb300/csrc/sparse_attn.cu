@@ -13,6 +13,9 @@ namespace rola {
 // ===========================================================================
 // fp32 validation mode: plain SIMT, one CTA per (query block, head), 256
 // threads.  Shared memory: Q, K with padded rows (129 floats), V, S.
+// q^r, k^r and v are read in block order (Np rows per head: the token order
+// itself for contiguous chunks, cube slots for cubes); O^s rows go to their
+// tokens.
 
 constexpr int kF32Threads = 256;
 constexpr int kPad = kDh + 1;
@@ -29,11 +32,11 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
     float* Vs = Ks + kBlock * kPad;        // [64][128]
     float* Ss = Vs + kBlock * kDh;         // [64][65]
     const int qb = blockIdx.x, bh = blockIdx.y, tid = threadIdx.x;
-    const size_t head = (size_t)bh * s.N * kDh;
+    const size_t head = (size_t)bh * s.Np * kDh;
     const int32_t* kept = kv_idx + ((size_t)bh * s.nB + qb) * s.n_keep;
     for (int e = tid; e < kBlock * kDh; e += kF32Threads) {
         int r = e / kDh, d = e % kDh, n = qb * kBlock + r;
-        Qs[r * kPad + d] = n < s.N ? qr[head + (size_t)n * kDh + d] : 0.0f;
+        Qs[r * kPad + d] = n < s.Np ? qr[head + (size_t)n * kDh + d] : 0.0f;
     }
     const int row = tid >> 2, quarter = tid & 3;
     float acc[32];
@@ -46,12 +49,13 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
         __syncthreads();
         for (int e = tid; e < kBlock * kDh; e += kF32Threads) {
             int r = e / kDh, d = e % kDh, n = j * kBlock + r;
-            bool ok = n >= 0 && n < s.N;
+            bool ok = n >= 0 && n < s.Np;
             Ks[r * kPad + d] = ok ? kr[head + (size_t)n * kDh + d] : 0.0f;
             Vs[r * kDh + d] = ok ? v[head + (size_t)n * kDh + d] : 0.0f;
         }
         __syncthreads();
         const int kvalid = s.N - j * kBlock;
+        const CubeOrigin jo = cube_origin(s, j);
         float sv[16];
         float mx = m_run;
 #pragma unroll 1
@@ -59,7 +63,8 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
             int col = quarter * 16 + c;
             float dot = 0.0f;
             for (int d = 0; d < kDh; ++d) dot = fmaf(Qs[row * kPad + d], Ks[col * kPad + d], dot);
-            sv[c] = col < kvalid ? dot * scale : -INFINITY;
+            const bool valid = s.cube ? cube_token(s, jo, col) >= 0 : col < kvalid;
+            sv[c] = valid ? dot * scale : -INFINITY;
             mx = fmaxf(mx, sv[c]);
         }
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
@@ -85,11 +90,12 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
             for (int i = 0; i < 32; ++i) acc[i] = fmaf(p, Vs[c * kDh + quarter + 4 * i], acc[i]);
         }
     }
-    const int n = qb * kBlock + row;
-    if (n < s.N) {
+    const int n = s.cube ? cube_token(s, cube_origin(s, qb), row) : qb * kBlock + row;
+    if (n >= 0 && n < s.N) {
         float inv = 1.0f / l_run;
+        float* on = o + ((size_t)bh * s.N + n) * kDh;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o[head + (size_t)n * kDh + quarter + 4 * i] = acc[i] * inv;
+        for (int i = 0; i < 32; ++i) on[quarter + 4 * i] = acc[i] * inv;
     }
 }
 

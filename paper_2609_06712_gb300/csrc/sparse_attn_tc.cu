@@ -175,6 +175,10 @@ __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[NC])
     for (int c = 1; c < NC / 16; ++c) reg_fence(*reinterpret_cast<float(*)[16]>(&v[c * 16]));
 }
 
+// kCube: blocks are 4x4x4 cubes.  q^r, k^r, v are then read in block order
+// (the maps span the padded Np rows), a key is valid when its cube slot lies
+// inside the grid, and each O^s row goes to the token of its slot.
+template <bool kCube>
 __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                                                                      const __grid_constant__ CUtensorMap map_k,
                                                                      const __grid_constant__ CUtensorMap map_v,
@@ -427,8 +431,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     jb_n = 2 * t + 3 < s.n_keep ? __ldg(kept + 2 * t + 3) : -1;
                 }
                 const int blk = wtid < 64 ? ja : jb;
-                const int key = blk * 64 + (wtid & 63);
-                const bool valid = blk >= 0 && key < s.N;
+                bool valid;
+                if constexpr (kCube) {
+                    valid = blk >= 0 && cube_token(s, cube_origin_rcp(s, blk), wtid & 63) >= 0;
+                } else {
+                    const int key = blk * 64 + (wtid & 63);
+                    valid = blk >= 0 && key < s.N;
+                }
                 if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
                 fence_after_sync();
                 const uint32_t saddr = tmem + lane_off + sb * 64 + col0;
@@ -534,11 +543,21 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
-                __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + wtid;
-                const int rows = min(64, s.N - qb * 64) - col0;     // rows of this warpgroup inside the sequence
+                if constexpr (kCube) {
+                    const CubeOrigin co = cube_origin_rcp(s, qb);
+                    __nv_bfloat16* dst = p.o + (size_t)bh * s.N * kDh + wtid;
 #pragma unroll
-                for (int q = 0; q < kCols; ++q)
-                    if (q < rows) dst[(size_t)q * kDh] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
+                    for (int q = 0; q < kCols; ++q) {
+                        const int n = cube_token(s, co, col0 + q);
+                        if (n >= 0) dst[(size_t)n * kDh] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
+                    }
+                } else {
+                    __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + wtid;
+                    const int rows = min(64, s.N - qb * 64) - col0;     // rows of this warpgroup inside the sequence
+#pragma unroll
+                    for (int q = 0; q < kCols; ++q)
+                        if (q < rows) dst[(size_t)q * kDh] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
+                }
             }
         }
         if (!ok) record_timeout(p, 3);
@@ -600,8 +619,12 @@ bool make_block_map(CUtensorMap* m, const void* ptr, const Shape& s, int rows)
 cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
                                   const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st)
 {
+    // the maps span the block-ordered rows (the token order itself for contiguous chunks)
+    Shape rows = s;
+    rows.N = s.Np;
     CUtensorMap mq, mk, mv;
-    if (!make_block_map(&mq, qr, s) || !make_chunk_map(&mk, kr, s) || !make_block_map(&mv, v, s)) return cudaErrorInvalidValue;
+    if (!make_block_map(&mq, qr, rows) || !make_chunk_map(&mk, kr, rows) || !make_block_map(&mv, v, rows))
+        return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -615,10 +638,11 @@ cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr
     p.total_items = s.B * s.H * s.nB;
     p.tiles = (s.n_keep + 1) / 2;
     const size_t smem = kSmemTiles + sizeof(Smem);
-    e = cudaFuncSetAttribute(sparse_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     const int grid = p.total_items < nsm ? p.total_items : nsm;
-    sparse_attn_tc_kernel<<<grid, kThreads, smem, st>>>(mq, mk, mv, p);
+    auto kernel = s.cube ? sparse_attn_tc_kernel<true> : sparse_attn_tc_kernel<false>;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kernel<<<grid, kThreads, smem, st>>>(mq, mk, mv, p);
     return cudaGetLastError();
 }
 

@@ -38,6 +38,7 @@ class RolaConfig(ctypes.Structure):
         ("debug_flags", ctypes.c_int32),
         ("lowrank_rope", ctypes.c_int32),
         ("lowrank_act", ctypes.c_int32),
+        ("block_geometry", ctypes.c_int32),
     ]
 
 
@@ -49,6 +50,9 @@ ROLA_LOWRANK_ROPE_OUTSIDE, ROLA_LOWRANK_ROPE_INSIDE, ROLA_LOWRANK_ROPE_NONE = 0,
  ROLA_LOWRANK_ACT_GELU) = 0, 1, 2, 3, 4
 LOWRANK_ACTS = {"silu": ROLA_LOWRANK_ACT_SILU, "identity": ROLA_LOWRANK_ACT_IDENTITY,
                 "tanh": ROLA_LOWRANK_ACT_TANH, "relu": ROLA_LOWRANK_ACT_RELU, "gelu": ROLA_LOWRANK_ACT_GELU}
+# rola_block_geometry_t: contiguous 64-token chunks, or 4 x 4 x 4 cubes of the latent grid
+ROLA_BLOCK_FLAT, ROLA_BLOCK_CUBE = 0, 1
+BLOCK_GEOMETRIES = {"flat": ROLA_BLOCK_FLAT, "cube": ROLA_BLOCK_CUBE}
 
 
 class RolaError(RuntimeError):
@@ -116,6 +120,8 @@ def make_config(cfg: dict, dtype: int = ROLA_BF16) -> RolaConfig:
     c.lowrank_rope = int(cfg.get("lowrank_rope", ROLA_LOWRANK_ROPE_OUTSIDE))
     act = cfg.get("lowrank_act", "silu")
     c.lowrank_act = LOWRANK_ACTS[act] if isinstance(act, str) else int(act)
+    geom = cfg.get("block_geometry", "flat")
+    c.block_geometry = BLOCK_GEOMETRIES[geom] if isinstance(geom, str) else int(geom)
     return c
 
 

@@ -69,7 +69,7 @@ def test_defaults_and_sizes(rl):
     assert rl.library().rola_config_init(ctypes.byref(c)) == rl.ROLA_OK
     assert (c.d_h, c.block, list(c.rope_split), c.rope_theta) == (128, 64, [44, 42, 42], 10000.0)
     assert c.gate_bias == pytest.approx(-1.946) and c.eps_lr == pytest.approx(1e-6)
-    assert c.lowrank_act == rl.ROLA_LOWRANK_ACT_SILU
+    assert c.lowrank_act == rl.ROLA_LOWRANK_ACT_SILU and c.block_geometry == rl.ROLA_BLOCK_FLAT
     assert c.lowrank_rope == rl.ROLA_LOWRANK_ROPE_OUTSIDE and c.wait_limit_ms == 0 and c.debug_flags == 0
     from paper_2609_06712_gb300 import configs
     for name, nb, nk in [("tiny", 16, 2), ("wan13b_480p", 512, 51), ("wan14b_720p", 1182, 118),
@@ -114,6 +114,8 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
     ("lowrank_rope", -1, 1),
     ("lowrank_act", 5, 1),
     ("lowrank_act", -1, 1),
+    ("block_geometry", 2, 1),
+    ("block_geometry", -1, 1),
 ])
 def test_invalid_config_is_rejected_before_launch(rl, field, value, code):
     c = cfg_tiny(rl, **{field: value})
@@ -129,6 +131,24 @@ def test_kept_block_count_limit(rl):
     assert rl.workspace_bytes(big) == 0
     half = cfg_tiny(rl, H=64, N=N, T=1, Hh=1, Ww=N, keep_ratio=0.5)
     assert rl.num_keep(half) == 2897 and rl.workspace_bytes(half) > 0
+
+
+def test_cube_geometry_sizes(rl):
+    """Cube geometry: nB is the cube count of the latent grid, n_keep rounds on it, and the
+    workspace grows by the padded cube-ordered copies (q^r, k^r and v)."""
+    from oracle import oracle as O
+    from paper_2609_06712_gb300 import configs
+    for T, Hh, Ww in [(5, 9, 13), (21, 45, 80), (1, 1, 3), (4, 16, 16)]:
+        cfg = dict(configs.get("tiny"), T=T, Hh=Hh, Ww=Ww, N=T * Hh * Ww, keep=0.1)
+        flat = rl.make_config(cfg)
+        cube = rl.make_config(dict(cfg, block_geometry="cube"))
+        nb = -(-T // 4) * -(-Hh // 4) * -(-Ww // 4)
+        assert rl.num_blocks(cube) == nb == O.num_blocks(dict(cfg, block_geometry="cube"))
+        assert rl.num_keep(cube) == O.num_keep(dict(cfg, block_geometry="cube"))
+        assert rl.workspace_bytes(cube) > rl.workspace_bytes(flat) or nb * 64 == T * Hh * Ww
+    # more blocks than the top-k kernel holds
+    big = rl.make_config(dict(configs.get("tiny"), T=1, Hh=1, Ww=7009 * 64, N=7009 * 64, keep=0.01))
+    assert rl.num_blocks(big) == 0 and rl.workspace_bytes(big) == 0
 
 
 def test_rope_split_must_sum_to_head_dim(rl):
