@@ -544,12 +544,20 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
                 if constexpr (kCube) {
+                    // this warpgroup's 32 slots are (dt, dx, dy) = (2 wg + q / 16, q / 4 % 4, q % 4):
+                    // offsets and bounds per row are compile-time against three runtime limits
+                    static_assert(kCols == 32, "a warpgroup owns two 16-slot layers of the cube");
                     const CubeOrigin co = cube_origin_rcp(s, qb);
-                    __nv_bfloat16* dst = p.o + (size_t)bh * s.N * kDh + wtid;
+                    const int t0 = co.t + 2 * wg;
+                    const int lt = s.T - t0, lx = s.Hh - co.x, ly = s.Ww - co.y;
+                    const size_t plane = (size_t)s.Hh * s.Ww * kDh, line = (size_t)s.Ww * kDh;
+                    const size_t row0 = ((size_t)bh * s.N + ((size_t)t0 * s.Hh + co.x) * s.Ww + co.y) * kDh + wtid;
 #pragma unroll
                     for (int q = 0; q < kCols; ++q) {
-                        const int n = cube_token(s, co, col0 + q);
-                        if (n >= 0) dst[(size_t)n * kDh] = __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
+                        const int dt = q >> 4, dx = (q >> 2) & 3, dy = q & 3;
+                        if (dt < lt && dx < lx && dy < ly)
+                            p.o[row0 + dt * plane + dx * line + dy * kDh] =
+                                __float2bfloat16_rn(ov[q] * sm.inv_l[col0 + q]);
                     }
                 } else {
                     __nv_bfloat16* dst = p.o + ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + wtid;
