@@ -76,6 +76,9 @@ def _get():
             lib.orc_pair_angle.restype = ctypes.c_double
             lib.orc_activation.argtypes = [cfgp, ctypes.c_double]
             lib.orc_activation.restype = ctypes.c_double
+            lib.orc_activation_grad.argtypes = [cfgp, ctypes.c_double]
+            lib.orc_activation_grad.restype = ctypes.c_double
+            lib.orc_backward.argtypes = [cfgp] + [P] * 14
             lib.orc_rotate.argtypes = [cfgp, ctypes.c_int, P, P, P, ctypes.c_int]
             lib.orc_lowrank_features.argtypes = [cfgp, P, P, P]
             lib.orc_lowrank_summary.argtypes = [cfgp, P, P, P, P, P]
@@ -126,6 +129,33 @@ def activation(name: str, x: float) -> float:
     c = make_config({"B": 1, "H": 1, "N": 1, "T": 1, "Hh": 1, "Ww": 1, "keep": 1.0, "r": 2,
                      "lowrank_act": name})
     return _get().orc_activation(ctypes.byref(c), float(x))
+
+
+def activation_grad(name: str, x: float) -> float:
+    """phi'(x) of the feature map, one fp64 value (the backward pass's derivative)."""
+    c = make_config({"B": 1, "H": 1, "N": 1, "T": 1, "Hh": 1, "Ww": 1, "keep": 1.0, "r": 2,
+                     "lowrank_act": name})
+    return _get().orc_activation_grad(ctypes.byref(c), float(x))
+
+
+def backward(cfg: dict, q, k, v, Pq, Pk, gate, kv_idx, dO, rope_mode: int = ROPE_OUTSIDE) -> dict:
+    """Gradients of sum(dO * O) through the forward pass under the mask kv_idx: dq, dk, dv
+    [B,H,N,dh], dP_q, dP_k [H,r,dh] (summed over the batch) and dgate [B,N] (summed over heads)."""
+    c = make_config(cfg, rope_mode)
+    q, qp = _f32(q)
+    k, kp = _f32(k)
+    v, vp = _f32(v)
+    Pq, Pqp = _f32(Pq)
+    Pk, Pkp = _f32(Pk)
+    g = None if gate is None else np.ascontiguousarray(gate, dtype=np.float32)
+    idx = np.ascontiguousarray(kv_idx, dtype=np.int32)
+    dO, dOp = _f32(dO)
+    shape = (c.B, c.H, c.N, c.dh)
+    out = {"dq": np.empty(shape), "dk": np.empty(shape), "dv": np.empty(shape),
+           "dP_q": np.empty((c.H, c.r, c.dh)), "dP_k": np.empty((c.H, c.r, c.dh)), "dgate": np.empty((c.B, c.N))}
+    _get().orc_backward(ctypes.byref(c), qp, kp, vp, Pqp, Pkp, _ptr(g), idx.ctypes.data, dOp,
+                        *(out[n].ctypes.data for n in ("dq", "dk", "dv", "dP_q", "dP_k", "dgate")))
+    return out
 
 
 def num_blocks(cfg: dict) -> int:
@@ -317,6 +347,6 @@ def forward(cfg: dict, q, k, v, Pq, Pk, gate=None, mask_override=None, qblocks=N
     _get().orc_forward(ctypes.byref(c), qp, kp, vp, Pqp, Pkp, _ptr(g), _ptr(mo), _ptr(sel),
                        o.ctypes.data, idx.ctypes.data, o_s.ctypes.data, C.ctypes.data, z.ctypes.data)
     if sel is not None:
-        rows = np.repeat(sel.astype(bool), c.block)[: c.N]
+        rows = sel.astype(bool)[block_of(cfg)]
         o_s[:, :, ~rows, :] = np.nan
     return dict(o=o, kv_idx=idx, o_s=o_s, C=C, z=z)

@@ -651,6 +651,244 @@ void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* 
     free(mask);
 }
 
+/* ------------------------------------------------------------------ */
+/* backward pass: the gradients of the single-stage fine-tune         */
+/* (Sec. impl, post-training: q, k, v, P_q, P_k and the gate train)   */
+/* ------------------------------------------------------------------ */
+
+/* phi'(x) of the configured feature map (the derivatives of the maps of
+ * orc_activation; Phi' is the standard normal density). */
+double orc_activation_grad(const orc_cfg* c, double x)
+{
+    switch (c->act) {
+        case 1: return 1.0;
+        case 2: { double t = tanh(x); return 1.0 - t * t; }
+        case 3: return x > 0.0 ? 1.0 : 0.0;
+        case 4: return 0.5 * (1.0 + erf(x / sqrt(2.0))) + x * exp(-0.5 * x * x) / sqrt(2.0 * acos(-1.0));
+        default: { double sg = 1.0 / (1.0 + exp(-x)); return sg * (1.0 + x * (1.0 - sg)); }
+    }
+}
+
+/* R^T on the first npairs pairs (the rotation by the opposite angles). */
+static void rotate_pairs_t(int npairs, const double* cs, const double* in, double* out, int len)
+{
+    for (int m = 0; m < npairs; ++m) {
+        double ca = cs[2 * m], sa = cs[2 * m + 1];
+        double x = in[2 * m], y = in[2 * m + 1];
+        out[2 * m] = x * ca + y * sa;
+        out[2 * m + 1] = -x * sa + y * ca;
+    }
+    for (int i = 2 * npairs; i < len; ++i) out[i] = in[i];
+}
+
+/* Backward of one token's features: given df [r] = dL/d(feature), add
+ * P^T du to dx [dh] and du x^T to dP [r][dh], du = dL/d(P x). */
+static void lowrank_feature_bwd(const orc_cfg* c, const double* cs, const float* x, const float* P,
+                                const double* df, double* dx, double* dP)
+{
+    int r = c->r, dh = c->dh;
+    double* u = (double*)malloc(sizeof(double) * (size_t)r);
+    double* w = (double*)malloc(sizeof(double) * (size_t)r);
+    double* du = (double*)malloc(sizeof(double) * (size_t)r);
+    for (int a = 0; a < r; ++a) {
+        double sum = 0.0;
+        for (int d = 0; d < dh; ++d) sum += (double)P[(size_t)a * dh + d] * (double)x[d];
+        u[a] = sum;
+    }
+    if (c->rope_mode == 0) {            /* f = R_r phi(u):  du = phi'(u) (R_r^T df) */
+        rotate_pairs_t(r / 2, cs, df, w, r);
+        for (int a = 0; a < r; ++a) du[a] = orc_activation_grad(c, u[a]) * w[a];
+    } else if (c->rope_mode == 1) {     /* f = phi(R_r u):  du = R_r^T (phi'(R_r u) df) */
+        rotate_pairs(r / 2, cs, u, w, r);
+        for (int a = 0; a < r; ++a) w[a] = orc_activation_grad(c, w[a]) * df[a];
+        rotate_pairs_t(r / 2, cs, w, du, r);
+    } else {                            /* f = phi(u) */
+        for (int a = 0; a < r; ++a) du[a] = orc_activation_grad(c, u[a]) * df[a];
+    }
+    for (int a = 0; a < r; ++a)
+        for (int d = 0; d < dh; ++d) {
+            dx[d] += (double)P[(size_t)a * dh + d] * du[a];
+            dP[(size_t)a * dh + d] += du[a] * (double)x[d];
+        }
+    free(u);
+    free(w);
+    free(du);
+}
+
+/*
+ * Gradients of L = sum_p dO_p . O_p for the forward pass under the block mask
+ * kv_idx (the top-k selection is piecewise constant in q and k, so nothing
+ * flows through it): dq, dk, dv [B][H][N][dh]; dPq, dPk [H][r][dh] summed over
+ * the batch; dgate [B][N] = dL/dg_p summed over the heads (also when gate is
+ * NULL, for the constant g = sigmoid(gate_bias)).  The steps undo the forward
+ * steps in reverse order: fusion, RMSNorm readout, features of q, summary,
+ * features of k, block-sparse softmax attention, full RoPE.
+ */
+void orc_backward(const orc_cfg* c, const float* q, const float* k, const float* v, const float* Pq,
+                  const float* Pk, const float* gate, const int32_t* kv_idx, const float* dO, double* dq,
+                  double* dk, double* dv, double* dPq, double* dPk, double* dgate)
+{
+    int B = c->B, H = c->H, N = c->N, dh = c->dh, r = c->r, bs = c->block, BH = c->B * c->H;
+    int nB = orc_num_blocks(c), nk = orc_num_keep(c);
+    double isd = 1.0 / sqrt((double)dh);
+    size_t nel = (size_t)BH * N * dh, nrd = (size_t)r * dh;
+    /* forward quantities the chain rule needs */
+    double* qr = (double*)malloc(sizeof(double) * nel);
+    double* kr = (double*)malloc(sizeof(double) * nel);
+    double* os = (double*)calloc(nel, sizeof(double));
+    double* C = (double*)malloc(sizeof(double) * (size_t)BH * nrd);
+    orc_rope_full(c, q, qr);
+    orc_rope_full(c, k, kr);
+    orc_sparse_attn(c, qr, kr, v, kv_idx, nk, NULL, os);
+    orc_lowrank_summary(c, k, v, Pk, C, NULL);
+    double* tcs = token_cs(c);
+    int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
+    int* count = (int*)malloc(sizeof(int) * (size_t)nB);
+    block_members(c, members, count);
+    double* dPq_bh = (double*)calloc((size_t)BH * nrd, sizeof(double));
+    double* dPk_bh = (double*)calloc((size_t)BH * nrd, sizeof(double));
+    double* dg_bh = (double*)calloc((size_t)BH * N, sizeof(double));
+    memset(dq, 0, sizeof(double) * nel);
+    memset(dk, 0, sizeof(double) * nel);
+    memset(dv, 0, sizeof(double) * nel);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        int b = bh / H, h = bh % H;
+        size_t head = (size_t)bh * N * dh;
+        const double* Cb = C + (size_t)bh * nrd;
+        double* dOs = (double*)calloc((size_t)N * dh, sizeof(double));
+        double* dqr = (double*)calloc((size_t)N * dh, sizeof(double));
+        double* dkr = (double*)calloc((size_t)N * dh, sizeof(double));
+        double* dC = (double*)calloc(nrd, sizeof(double));
+        double* olr = (double*)malloc(sizeof(double) * (size_t)dh);
+        double* y = (double*)malloc(sizeof(double) * (size_t)dh);
+        double* dy = (double*)malloc(sizeof(double) * (size_t)dh);
+        double* ft = (double*)malloc(sizeof(double) * (size_t)r);
+        double* dft = (double*)malloc(sizeof(double) * (size_t)r);
+        /* fusion O = (O^s / r_p + g O^lr) r_p and readout O^lr = y / rho, y = q~^T C */
+        for (int p = 0; p < N; ++p) {
+            const double* osp = os + head + (size_t)p * dh;
+            const float* dop = dO + head + (size_t)p * dh;
+            double g = gate_value(c, gate, b, p);
+            lowrank_readout(c, tcs, bh, p, q, Pq, C, olr, y);
+            double ss = 0.0, yy = 0.0, a = 0.0;
+            for (int d = 0; d < dh; ++d) {
+                ss += osp[d] * osp[d];
+                yy += y[d] * y[d];
+                a += olr[d] * (double)dop[d];
+            }
+            double rp = sqrt(ss / (double)dh + c->eps_f);
+            double rho = sqrt(yy / (double)dh + c->eps_lr);
+            double dr = g * a;                          /* dL/dr_p */
+            dg_bh[(size_t)bh * N + p] = rp * a;         /* dL/dg_p from this head */
+            double od = 0.0;                            /* O^lr . dL/dO^lr */
+            for (int d = 0; d < dh; ++d) {
+                dOs[(size_t)p * dh + d] = (double)dop[d] + dr * osp[d] / ((double)dh * rp);
+                od += olr[d] * g * rp * (double)dop[d];
+            }
+            for (int d = 0; d < dh; ++d) dy[d] = (g * rp * (double)dop[d] - olr[d] * od / (double)dh) / rho;
+            lowrank_feature(c, tcs + (size_t)p * dh, q + head + (size_t)p * dh, Pq + (size_t)h * nrd, ft);
+            for (int aa = 0; aa < r; ++aa) {
+                double sum = 0.0;
+                for (int d = 0; d < dh; ++d) {
+                    sum += Cb[(size_t)aa * dh + d] * dy[d];
+                    dC[(size_t)aa * dh + d] += ft[aa] * dy[d];
+                }
+                dft[aa] = sum;
+            }
+            lowrank_feature_bwd(c, tcs + (size_t)p * dh, q + head + (size_t)p * dh, Pq + (size_t)h * nrd, dft,
+                                dq + head + (size_t)p * dh, dPq_bh + (size_t)bh * nrd);
+        }
+        /* summary C = sum_j k~_j v_j^T */
+        for (int j = 0; j < N; ++j) {
+            const float* vj = v + head + (size_t)j * dh;
+            lowrank_feature(c, tcs + (size_t)j * dh, k + head + (size_t)j * dh, Pk + (size_t)h * nrd, ft);
+            for (int aa = 0; aa < r; ++aa) {
+                double sum = 0.0;
+                for (int d = 0; d < dh; ++d) {
+                    sum += dC[(size_t)aa * dh + d] * (double)vj[d];
+                    dv[head + (size_t)j * dh + d] += ft[aa] * dC[(size_t)aa * dh + d];
+                }
+                dft[aa] = sum;
+            }
+            lowrank_feature_bwd(c, tcs + (size_t)j * dh, k + head + (size_t)j * dh, Pk + (size_t)h * nrd, dft,
+                                dk + head + (size_t)j * dh, dPk_bh + (size_t)bh * nrd);
+        }
+        /* block-sparse softmax attention: s = q^r k^r / sqrt(d_h), P = softmax(s), O^s = P v */
+        for (int i = 0; i < nB; ++i) {
+            const int32_t* kept = kv_idx + ((size_t)bh * nB + i) * nk;
+            int nkeys = 0;
+            for (int t = 0; t < nk; ++t) nkeys += count[kept[t]];
+            int* keys = (int*)malloc(sizeof(int) * (size_t)nkeys);
+            double* pr = (double*)malloc(sizeof(double) * (size_t)nkeys);
+            double* dpr = (double*)malloc(sizeof(double) * (size_t)nkeys);
+            int kk = 0;
+            for (int t = 0; t < nk; ++t)
+                for (int m = 0; m < count[kept[t]]; ++m) keys[kk++] = members[(size_t)kept[t] * bs + m];
+            for (int mi = 0; mi < count[i]; ++mi) {
+                int p = members[(size_t)i * bs + mi];
+                const double* qp = qr + head + (size_t)p * dh;
+                const double* dop = dOs + (size_t)p * dh;
+                double mx = -INFINITY;
+                for (int t = 0; t < nkeys; ++t) {
+                    const double* kq = kr + head + (size_t)keys[t] * dh;
+                    double acc = 0.0;
+                    for (int d = 0; d < dh; ++d) acc += qp[d] * kq[d];
+                    pr[t] = acc * isd;
+                    if (pr[t] > mx) mx = pr[t];
+                }
+                double den = 0.0;
+                for (int t = 0; t < nkeys; ++t) { pr[t] = exp(pr[t] - mx); den += pr[t]; }
+                double Dp = 0.0;                        /* sum_t P_t dP_t */
+                for (int t = 0; t < nkeys; ++t) {
+                    pr[t] /= den;
+                    const float* vq = v + head + (size_t)keys[t] * dh;
+                    double acc = 0.0;
+                    for (int d = 0; d < dh; ++d) acc += dop[d] * (double)vq[d];
+                    dpr[t] = acc;
+                    Dp += pr[t] * acc;
+                }
+                for (int t = 0; t < nkeys; ++t) {
+                    int j = keys[t];
+                    double dsv = pr[t] * (dpr[t] - Dp) * isd;     /* dL/d(q^r . k^r) */
+                    const double* kq = kr + head + (size_t)j * dh;
+                    for (int d = 0; d < dh; ++d) {
+                        dqr[(size_t)p * dh + d] += dsv * kq[d];
+                        dkr[(size_t)j * dh + d] += dsv * qp[d];
+                        dv[head + (size_t)j * dh + d] += pr[t] * dop[d];
+                    }
+                }
+            }
+            free(keys);
+            free(pr);
+            free(dpr);
+        }
+        /* full RoPE: dq += R(p)^T dq^r, dk += R(p)^T dk^r */
+        for (int n = 0; n < N; ++n) {
+            rotate_pairs_t(dh / 2, tcs + (size_t)n * dh, dqr + (size_t)n * dh, dy, dh);
+            for (int d = 0; d < dh; ++d) dq[head + (size_t)n * dh + d] += dy[d];
+            rotate_pairs_t(dh / 2, tcs + (size_t)n * dh, dkr + (size_t)n * dh, dy, dh);
+            for (int d = 0; d < dh; ++d) dk[head + (size_t)n * dh + d] += dy[d];
+        }
+        free(dOs); free(dqr); free(dkr); free(dC); free(olr); free(y); free(dy); free(ft); free(dft);
+    }
+    memset(dPq, 0, sizeof(double) * (size_t)H * nrd);
+    memset(dPk, 0, sizeof(double) * (size_t)H * nrd);
+    for (int bh = 0; bh < BH; ++bh)
+        for (size_t e = 0; e < nrd; ++e) {
+            dPq[(size_t)(bh % H) * nrd + e] += dPq_bh[(size_t)bh * nrd + e];
+            dPk[(size_t)(bh % H) * nrd + e] += dPk_bh[(size_t)bh * nrd + e];
+        }
+    for (int b = 0; b < B; ++b)
+        for (int p = 0; p < N; ++p) {
+            double sum = 0.0;
+            for (int h = 0; h < H; ++h) sum += dg_bh[((size_t)b * H + h) * N + p];
+            dgate[(size_t)b * N + p] = sum;
+        }
+    free(qr); free(kr); free(os); free(C); free(tcs); free(members); free(count);
+    free(dPq_bh); free(dPk_bh); free(dg_bh);
+}
+
 /* Token gate of the gated fusion (Sec. fusion, Alg. 1 "token-wise scalar
  * gate"): g_p = sigmoid(x_p . w_g + b_g), one scalar per token from the
  * attention block's input hidden state x_p (d_model wide).  X is [B][N][D],

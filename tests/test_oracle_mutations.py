@@ -47,6 +47,16 @@ MUTATIONS = {
     "relu_leaky": ("case 3: return x > 0.0 ? x : 0.0;", "case 3: return x > 0.0 ? x : 0.01 * x;"),
     "activation_before_rotation_only": ("for (int a = 0; a < r; ++a) u[a] = orc_activation(c, u[a]);",
                                         "for (int a = 0; a < r; ++a) u[a] = silu(u[a]);"),
+    "bwd_softmax_no_centering": ("double dsv = pr[t] * (dpr[t] - Dp) * isd;", "double dsv = pr[t] * dpr[t] * isd;"),
+    "bwd_rope_not_transposed": ("out[2 * m] = x * ca + y * sa;\n        out[2 * m + 1] = -x * sa + y * ca;",
+                                "out[2 * m] = x * ca - y * sa;\n        out[2 * m + 1] = x * sa + y * ca;"),
+    "bwd_fusion_rms_term": ("dOs[(size_t)p * dh + d] = (double)dop[d] + dr * osp[d] / ((double)dh * rp);",
+                            "dOs[(size_t)p * dh + d] = (double)dop[d];"),
+    "bwd_rmsnorm_projection": ("dy[d] = (g * rp * (double)dop[d] - olr[d] * od / (double)dh) / rho;",
+                               "dy[d] = g * rp * (double)dop[d] / rho;"),
+    "bwd_silu_derivative": ("return sg * (1.0 + x * (1.0 - sg));", "return sg;"),
+    "bwd_summary_value_grad": ("dv[head + (size_t)j * dh + d] += ft[aa] * dC[(size_t)aa * dh + d];",
+                               "dv[head + (size_t)j * dh + d] += ft[aa] * dC[(size_t)aa * dh + (d + 1) % dh];"),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 
@@ -63,6 +73,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
                            str(mutated), "-lm"])
     env = dict(os.environ, ORACLE_LIB=str(lib), OMP_NUM_THREADS="4")
     res = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                          os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                          os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+                          os.path.join(ROOT, "tests", "test_oracle_backward_pins.py")],
                          cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert res.returncode != 0, f"mutation {name} survived the pins:\n{res.stdout[-2000:]}"
