@@ -242,6 +242,68 @@ def run_reference(args, cfg, ws, rank):
     print(json.dumps(line), flush=True)
 
 
+# fp32 FMA peak of the SIMT backward kernels: 152 SMs x 128 fp32 lanes x 2 flops x 2.07 GHz
+FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def run_backward(args, cfg, c, x, stream, ws, rank):
+    """Times rola_forward_train and rola_backward (one training step of the module) on the layer."""
+    import torch
+    from paper_2609_06712_gb300 import rola
+    dev = x["q"].device
+    B, H, N, r = cfg["B"], cfg["H"], cfg["N"], cfg["r"]
+    wsb = rola.workspace(c, dev)
+    bws = rola.backward_workspace(c, dev)
+    o, o_s = torch.empty_like(x["q"]), torch.empty_like(x["q"])
+    kv = torch.empty((B, H, rola.num_blocks(c), rola.num_keep(c)), dtype=torch.int32, device=dev)
+    lse = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+    C = torch.empty((B, H, r, 128), dtype=torch.float32, device=dev)
+    dO = torch.randn(x["q"].shape, generator=torch.Generator(device=dev).manual_seed(5), device=dev,
+                     dtype=torch.float32).to(x["q"].dtype)
+    g = {n: torch.empty_like(x[n[1:]]) for n in ("dq", "dk", "dv")}
+    dPq = torch.empty(x["P_q"].shape, dtype=torch.float32, device=dev)
+    dPk = torch.empty(x["P_k"].shape, dtype=torch.float32, device=dev)
+    dgate = torch.empty((B, N), dtype=torch.float32, device=dev) if x["gate"] is not None else None
+    fw = lambda: rola.forward_train(c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kv, o_s, lse, C,
+                                    wsb)
+    bw = lambda: rola.backward(c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], kv, o_s, lse, C, dO,
+                               g["dq"], g["dk"], g["dv"], dPq, dPk, dgate, bws)
+    for _ in range(args.warmup):
+        fw()
+        bw()
+    torch.cuda.synchronize()
+    barrier(ws)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    t_fw = t_bw = 0.0
+    for _ in range(args.steps):
+        ev[0].record(stream)
+        fw()
+        ev[1].record(stream)
+        bw()
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        t_fw += ev[0].elapsed_time(ev[1])
+        t_bw += ev[1].elapsed_time(ev[2])
+    ms_fw = reduce_max(t_fw / args.steps, ws)
+    ms_bw = reduce_max(t_bw / args.steps, ws)
+    assert rola.get_device_status(wsb) == rola.ROLA_OK and rola.get_device_status(bws) == rola.ROLA_OK
+    if rank == 0:
+        sparse_fw = sparse_flops_from_mask(kv, block_sizes(cfg))
+        # algorithmic: recompute S, dP = dO^s V^T, dQ, dK, dV (5 products of the sparse pattern), and the
+        # low-rank backward's six N x r x d_h products (u, y, dq~, dq, dC, dP_q on the query side; u, dk~,
+        # dv, dk, dP_k on the key side: 11 products of 2 N d_h r flops)
+        flops = 2.5 * sparse_fw + 11 * 2.0 * B * H * N * 128 * r
+        print(json.dumps({"entry": "rola_backward", "ms_forward_train": ms_fw, "ms_backward": ms_bw,
+                          "train_step_tokens_per_s": job_throughput(B * N, ms_fw + ms_bw, ws),
+                          "backward_flops": flops, "achieved_tflops": flops / (ms_bw * 1e-3) / 1e12,
+                          "bound": "alu", "peak_tflops": FP32_SIMT_PEAK_TFLOPS,
+                          "frac": flops / (ms_bw * 1e-3) / 1e12 / FP32_SIMT_PEAK_TFLOPS,
+                          "peak_source": "fp32 FMA lanes x clock (152 SMs x 128 x 2 x 2.07 GHz), derived",
+                          "steps": args.steps, "warmup": args.warmup,
+                          "config": {"workload": cfg["name"], "B": B, "H": H, "N": N, "r": r, "keep": cfg["keep"],
+                                     "dtype": "bf16 storage, fp32 arithmetic"}}), flush=True)
+
+
 def run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank):
     """Times one per-stage entry point of the C ABI on the layer (inputs resident in HBM)."""
     import torch
@@ -299,7 +361,8 @@ def main():
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--entry", default="forward", choices=["forward", "mask", "summary", "sparse", "apply"],
+    ap.add_argument("--entry", default="forward", choices=["forward", "mask", "summary", "sparse", "apply",
+                                                           "backward"],
                     help="time one per-stage entry point alone instead of the layer")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -343,6 +406,9 @@ def main():
         for e in row:
             e.record(stream)
     args_fw = (c, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kv, wsb)
+    if args.entry == "backward":
+        run_backward(args, cfg, c, x, stream, ws, rank)
+        return
     if args.entry != "forward":
         run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank)
         return

@@ -241,6 +241,48 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
                            int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * rola_forward for training: the same computation, keeping what rola_backward
+ * reads.  kv_idx_out is required here.
+ *   o_s : out, [B][H][N][d_h] sparse-branch output O^s, dtype (must not alias o)
+ *   lse : out, fp32 [B][H][N], log sum_j exp(<q^r_p, k^r_j> / sqrt(d_h)) over the
+ *         kept keys of each query row (natural log)
+ *   C   : out, fp32 [B][H][r][d_h], the low-rank summary
+ */
+rola_status_t rola_forward_train(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                                 const void* P_q, const void* P_k, const float* gate, void* o,
+                                 int32_t* kv_idx_out, void* o_s, float* lse, float* C, void* ws,
+                                 size_t ws_bytes, void* stream);
+
+/* Bytes of workspace rola_backward needs (256-byte aligned); 0 if cfg is
+ * invalid or not supported by the backward pass (block_geometry CUBE). */
+size_t rola_backward_workspace_bytes(const rola_config_t* cfg);
+
+/*
+ * Backward pass: the gradients of L = sum_p dO_p . O_p through the forward
+ * pass under the block mask kv_idx (the top-k selection is piecewise constant,
+ * so no gradient flows through it), for the single-stage fine-tune that trains
+ * q, k, v (the backbone's projections), P_q, P_k and the gate (Sec. impl).
+ * Undoes the fusion (Eq. gate), the RMSNorm readout and the summary (Eq. ctx),
+ * the low-rank features (Eq. qklr, with the configured placement and map), the
+ * block-sparse softmax attention and the full RoPE (Sec. 3), in that order.
+ *   q, k, v, P_q, P_k, gate : the forward inputs
+ *   kv_idx, o_s, lse, C     : what rola_forward_train returned for them
+ *   dO      : [B][H][N][d_h], dtype
+ *   dq, dk, dv : out, [B][H][N][d_h], dtype
+ *   dP_q, dP_k : out, fp32 [H][r][d_h], summed over the batch
+ *   dgate   : out, fp32 [B][N], dL/dg_p summed over the heads (for gate == NULL:
+ *             the gradient at the constant sigmoid(gate_bias)), or NULL
+ * Arithmetic is fp32 throughout (SIMT), accumulation of dq, dk, dv in fp32;
+ * results are bitwise reproducible (fixed-order reductions).  Contiguous
+ * 64-token blocks only (ROLA_BLOCK_CUBE returns ROLA_ERR_UNSUPPORTED).
+ */
+rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                            const void* P_q, const void* P_k, const float* gate, const int32_t* kv_idx,
+                            const void* o_s, const float* lse, const float* C, const void* dO, void* dq,
+                            void* dk, void* dv, float* dP_q, float* dP_k, float* dgate, void* ws,
+                            size_t ws_bytes, void* stream);
+
+/*
  * rola_forward with stage timing: identical computation and launches, plus
  * cudaEventRecord(stage_events[i], stream) at five stage boundaries --
  *   [0] start  [1] after the block mask (fp32) or the fused pass over

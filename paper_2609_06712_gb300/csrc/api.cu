@@ -206,6 +206,117 @@ rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& 
     return ROLA_OK;
 }
 
+// Backward workspace: the status word and RoPE table as in the forward
+// workspace, the rotated copies, fp32 gradient rows and partials.
+struct BwdWorkspace {
+    size_t status, table, qr, kr, qbar, kbar, dOs, Dv, dq, dk, dv, dg, partC, partPq, partPk, dC, tr_off, tr_list,
+        total;
+};
+
+BwdWorkspace bwd_layout(const rola_config_t& c)
+{
+    const Shape s = make_shape(c);
+    const size_t esz = c.dtype == ROLA_BF16 ? 2 : 4;
+    const size_t bh = (size_t)c.B * c.H, rows = bh * c.N;
+    const size_t part = 4 * bh * s.nC * (size_t)c.r * kDh;
+    BwdWorkspace w;
+    size_t off = 0;
+    w.status = off; off = align_up(off + sizeof(DeviceStatus));
+    w.table = off; off = align_up(off + sizeof(float2) * (size_t)(c.T + c.Hh + c.Ww) * kPairs);
+    w.qr = off; off = align_up(off + esz * rows * kDh);
+    w.kr = off; off = align_up(off + esz * rows * kDh);
+    w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
+    w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
+    w.dOs = off; off = align_up(off + 4 * rows * kDh);
+    w.Dv = off; off = align_up(off + 4 * rows);
+    w.dq = off; off = align_up(off + 4 * rows * kDh);
+    w.dk = off; off = align_up(off + 4 * rows * kDh);
+    w.dv = off; off = align_up(off + 4 * rows * kDh);
+    w.dg = off; off = align_up(off + 4 * rows);
+    w.partC = off; off = align_up(off + part);
+    w.partPq = off; off = align_up(off + part);
+    w.partPk = off; off = align_up(off + part);
+    w.dC = off; off = align_up(off + 4 * bh * (size_t)c.r * kDh);
+    w.tr_off = off; off = align_up(off + 4 * bh * (s.nB + 1));
+    w.tr_list = off; off = align_up(off + 4 * bh * (size_t)s.nB * s.n_keep);
+    w.total = off;
+    return w;
+}
+
+// The forward pass.  With o_s_out the sparse output is kept there (and O written
+// to o), with lse_out the log-sum-exp of every query row, with C_out the summary:
+// what the backward pass reads.
+rola_status_t forward_impl(const rola_config_t* cfg, const void* q, const void* k, const void* v, const void* P_q,
+                           const void* P_k, const float* gate, void* o, int32_t* kv_idx_out, void* o_s_out,
+                           float* lse_out, float* C_out, void* ws, size_t ws_bytes, void* stream,
+                           void* const* stage_events)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!q || !k || !v || !P_q || !P_k || !o) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(P_q) || !aligned16(P_k) || !aligned16(o) ||
+        (kv_idx_out && !aligned16(kv_idx_out)) || (gate && (reinterpret_cast<uintptr_t>(gate) & 3u)) ||
+        (o_s_out && (!aligned16(o_s_out) || o_s_out == o)) || (lse_out && !aligned16(lse_out)) ||
+        (C_out && !aligned16(C_out)))
+        return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    auto mark = [&](int i) -> cudaError_t {
+        return stage_events ? cudaEventRecord(static_cast<cudaEvent_t>(stage_events[i]), st) : cudaSuccess;
+    };
+    Workspace w = layout(*cfg);
+    Shape s = make_shape(*cfg);
+    int32_t* kv = kv_idx_out ? kv_idx_out : at<int32_t>(ws, w.kv_idx);
+    ROLA_TRY(mark(0));
+    ROLA_CHECK(prologue(*cfg, ws, w, st));
+    if (cfg->dtype == ROLA_BF16 && s.cube) {
+        // stage 1: q^r, k^r, v in cube order and the cube means, then the summary
+        // partials (the fused pre-pass pools contiguous chunks only);
+        // stage 2: block scores + top-k, and the summary combine
+        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        ROLA_TRY(rope_pool(*cfg, s, w, q, k, v, ws, st));
+        ROLA_TRY(launch_prepass(s, ctas, nullptr, k, v, P_k, at<float2>(ws, w.table), nullptr, nullptr, nullptr,
+                                nullptr, at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
+        ROLA_TRY(mark(1));
+        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
+                                   st));
+        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
+                                        at<__nv_bfloat16>(ws, w.Cbf), st));
+    } else if (cfg->dtype == ROLA_BF16) {
+        // stage 1: one pass over q, k, v -> q^r, k^r, block means, summary partials;
+        // stage 2: block scores + top-k, and the summary combine
+        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
+        if (ctas <= 0) return ROLA_ERR_CUDA;
+        ROLA_TRY(launch_prepass(s, ctas, q, k, v, P_k, at<float2>(ws, w.table), at<void>(ws, w.qr),
+                                at<void>(ws, w.kr), at<float>(ws, w.qbar), at<float>(ws, w.kbar),
+                                at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
+        ROLA_TRY(mark(1));
+        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
+                                   st));
+        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
+                                        at<__nv_bfloat16>(ws, w.Cbf), st));
+    } else {
+        // stage 1: the block mask; stage 2: the summary
+        ROLA_CHECK(run_mask(*cfg, s, w, q, k, v, kv, ws, st));
+        ROLA_TRY(mark(1));
+        ROLA_CHECK(run_summary(*cfg, s, w, k, v, P_k, at<float>(ws, w.C), at<float>(ws, w.z),
+                               at<__nv_bfloat16>(ws, w.Cbf), ws, st));
+    }
+    if (C_out)
+        ROLA_TRY(cudaMemcpyAsync(C_out, at<float>(ws, w.C), sizeof(float) * (size_t)s.B * s.H * s.r * kDh,
+                                 cudaMemcpyDeviceToDevice, st));
+    void* os = o_s_out ? o_s_out : o;
+    ROLA_TRY(mark(2));
+    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), sparse_v(s, w, v, ws), kv, os,
+                                lse_out, at<DeviceStatus>(ws, w.status), st));
+    ROLA_TRY(mark(3));
+    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, os,
+                                  o, at<float2>(ws, w.table), at<DeviceStatus>(ws, w.status), st));
+    ROLA_TRY(mark(4));
+    return ROLA_OK;
+}
+
+
 }  // namespace
 
 extern "C" {
@@ -275,7 +386,7 @@ rola_status_t rola_sparse_attn(const rola_config_t* cfg, const void* q, const vo
     // rotated copies in block order (the pooled means are a by-product here)
     ROLA_TRY(rope_pool(*cfg, s, w, q, k, v, ws, st));
     ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), sparse_v(s, w, v, ws), kv_idx,
-                                o_s, at<DeviceStatus>(ws, w.status), st));
+                                o_s, nullptr, at<DeviceStatus>(ws, w.status), st));
     return ROLA_OK;
 }
 
@@ -318,63 +429,16 @@ rola_status_t rola_forward_timed(const rola_config_t* cfg, const void* q, const 
                                  const void* P_q, const void* P_k, const float* gate, void* o, int32_t* kv_idx_out,
                                  void* ws, size_t ws_bytes, void* stream, void* const* stage_events)
 {
-    ROLA_CHECK(validate(cfg));
-    if (!q || !k || !v || !P_q || !P_k || !o) return ROLA_ERR_INVALID_ARG;
-    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(P_q) || !aligned16(P_k) || !aligned16(o) ||
-        (kv_idx_out && !aligned16(kv_idx_out)) || (gate && (reinterpret_cast<uintptr_t>(gate) & 3u)))
-        return ROLA_ERR_INVALID_ARG;
-    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    auto mark = [&](int i) -> cudaError_t {
-        return stage_events ? cudaEventRecord(static_cast<cudaEvent_t>(stage_events[i]), st) : cudaSuccess;
-    };
-    Workspace w = layout(*cfg);
-    Shape s = make_shape(*cfg);
-    int32_t* kv = kv_idx_out ? kv_idx_out : at<int32_t>(ws, w.kv_idx);
-    ROLA_TRY(mark(0));
-    ROLA_CHECK(prologue(*cfg, ws, w, st));
-    if (cfg->dtype == ROLA_BF16 && s.cube) {
-        // stage 1: q^r, k^r, v in cube order and the cube means, then the summary
-        // partials (the fused pre-pass pools contiguous chunks only);
-        // stage 2: block scores + top-k, and the summary combine
-        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
-        if (ctas <= 0) return ROLA_ERR_CUDA;
-        ROLA_TRY(rope_pool(*cfg, s, w, q, k, v, ws, st));
-        ROLA_TRY(launch_prepass(s, ctas, nullptr, k, v, P_k, at<float2>(ws, w.table), nullptr, nullptr, nullptr,
-                                nullptr, at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
-        ROLA_TRY(mark(1));
-        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
-                                   st));
-        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
-                                        at<__nv_bfloat16>(ws, w.Cbf), st));
-    } else if (cfg->dtype == ROLA_BF16) {
-        // stage 1: one pass over q, k, v -> q^r, k^r, block means, summary partials;
-        // stage 2: block scores + top-k, and the summary combine
-        const int ctas = prepass_ctas(s, kMaxPrepassCtas);
-        if (ctas <= 0) return ROLA_ERR_CUDA;
-        ROLA_TRY(launch_prepass(s, ctas, q, k, v, P_k, at<float2>(ws, w.table), at<void>(ws, w.qr),
-                                at<void>(ws, w.kr), at<float>(ws, w.qbar), at<float>(ws, w.kbar),
-                                at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
-        ROLA_TRY(mark(1));
-        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
-                                   st));
-        ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
-                                        at<__nv_bfloat16>(ws, w.Cbf), st));
-    } else {
-        // stage 1: the block mask; stage 2: the summary
-        ROLA_CHECK(run_mask(*cfg, s, w, q, k, v, kv, ws, st));
-        ROLA_TRY(mark(1));
-        ROLA_CHECK(run_summary(*cfg, s, w, k, v, P_k, at<float>(ws, w.C), at<float>(ws, w.z),
-                               at<__nv_bfloat16>(ws, w.Cbf), ws, st));
-    }
-    ROLA_TRY(mark(2));
-    ROLA_TRY(launch_sparse_attn(cfg->dtype, s, at<void>(ws, w.qr), at<void>(ws, w.kr), sparse_v(s, w, v, ws), kv, o,
-                                at<DeviceStatus>(ws, w.status), st));
-    ROLA_TRY(mark(3));
-    ROLA_TRY(launch_lowrank_apply(cfg->dtype, s, q, P_q, at<float>(ws, w.C), at<__nv_bfloat16>(ws, w.Cbf), gate, o,
-                                  o, at<float2>(ws, w.table), at<DeviceStatus>(ws, w.status), st));
-    ROLA_TRY(mark(4));
-    return ROLA_OK;
+    return forward_impl(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, nullptr, nullptr, nullptr, ws, ws_bytes, stream,
+                        stage_events);
+}
+
+rola_status_t rola_forward_train(const rola_config_t* cfg, const void* q, const void* k, const void* v,
+                                 const void* P_q, const void* P_k, const float* gate, void* o, int32_t* kv_idx_out,
+                                 void* o_s, float* lse, float* C, void* ws, size_t ws_bytes, void* stream)
+{
+    if (!kv_idx_out || !o_s || !lse || !C) return validate(cfg) == ROLA_OK ? ROLA_ERR_INVALID_ARG : validate(cfg);
+    return forward_impl(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, o_s, lse, C, ws, ws_bytes, stream, nullptr);
 }
 
 rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* k, const void* v, const void* P_q,
@@ -382,6 +446,48 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
                            size_t ws_bytes, void* stream)
 {
     return rola_forward_timed(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, ws_bytes, stream, nullptr);
+}
+
+size_t rola_backward_workspace_bytes(const rola_config_t* cfg)
+{
+    if (validate(cfg) != ROLA_OK || cfg->block_geometry != ROLA_BLOCK_FLAT) return 0;
+    return bwd_layout(*cfg).total;
+}
+
+rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void* k, const void* v, const void* P_q,
+                            const void* P_k, const float* gate, const int32_t* kv_idx, const void* o_s,
+                            const float* lse, const float* C, const void* dO, void* dq, void* dk, void* dv,
+                            float* dP_q, float* dP_k, float* dgate, void* ws, size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (cfg->block_geometry != ROLA_BLOCK_FLAT) return ROLA_ERR_UNSUPPORTED;
+    const void* in[] = {q, k, v, P_q, P_k, kv_idx, o_s, lse, C, dO, dq, dk, dv, dP_q, dP_k};
+    for (const void* p : in)
+        if (!p || !aligned16(p)) return ROLA_ERR_INVALID_ARG;
+    if ((gate && (reinterpret_cast<uintptr_t>(gate) & 3u)) || (dgate && (reinterpret_cast<uintptr_t>(dgate) & 3u)))
+        return ROLA_ERR_INVALID_ARG;
+    const BwdWorkspace w = bwd_layout(*cfg);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) || ws_bytes < w.total) return ROLA_ERR_WORKSPACE;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Shape s = make_shape(*cfg);
+    ROLA_TRY(cudaMemsetAsync(at<uint8_t>(ws, w.status), 0, sizeof(DeviceStatus), st));
+    ROLA_TRY(launch_rope_table(*cfg, at<float2>(ws, w.table), st));
+    ROLA_TRY(launch_rope_pool(*cfg, s, q, k, nullptr, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
+                              nullptr, at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
+    BackwardArgs a;
+    a.q = q; a.k = k; a.v = v; a.P_q = P_q; a.P_k = P_k; a.o_s = o_s; a.dO = dO;
+    a.C = C; a.gate = gate; a.lse = lse; a.kv_idx = kv_idx;
+    a.tab = at<float2>(ws, w.table);
+    a.qr = at<void>(ws, w.qr); a.kr = at<void>(ws, w.kr);
+    a.dOs = at<float>(ws, w.dOs); a.Dv = at<float>(ws, w.Dv);
+    a.dq_acc = at<float>(ws, w.dq); a.dk_acc = at<float>(ws, w.dk); a.dv_acc = at<float>(ws, w.dv);
+    a.dg_h = at<float>(ws, w.dg);
+    a.partC = at<float>(ws, w.partC); a.partPq = at<float>(ws, w.partPq); a.partPk = at<float>(ws, w.partPk);
+    a.dC = at<float>(ws, w.dC);
+    a.tr_off = at<int32_t>(ws, w.tr_off); a.tr_list = at<int32_t>(ws, w.tr_list);
+    a.dq = dq; a.dk = dk; a.dv = dv; a.dP_q = dP_q; a.dP_k = dP_k; a.dgate = dgate;
+    ROLA_TRY(launch_backward(cfg->dtype, s, a, st));
+    return ROLA_OK;
 }
 
 rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g, float b_g, int32_t d_model,

@@ -137,11 +137,13 @@ cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const voi
                              float* kbar, cudaStream_t st);
 cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
                               int32_t* kv_idx, cudaStream_t st);
+// lse (nullable): fp32 [B][H][N], log sum_j exp(s_pj) of each query row (natural log).
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr,
-                               const void* v, const int32_t* kv_idx, void* o_s, DeviceStatus* status,
+                               const void* v, const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status,
                                cudaStream_t st);
 cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
-                                  const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st);
+                                  const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status,
+                                  cudaStream_t st);
 cudaError_t launch_lowrank_summary(rola_dtype_t dt, const Shape& s, int nsplit, const void* k,
                                    const void* v, const void* P_k, const float2* tab, float* partials,
                                    float* C, float* z, __nv_bfloat16* Cbf, cudaStream_t st);
@@ -156,6 +158,22 @@ cudaError_t launch_readout(const Shape& s, const void* q, const void* P_q, const
                            cudaStream_t st);
 
 // Token gate g = sigmoid(X w_g + b) over `rows` rows of D features (gate.cu).
+// Everything the backward pass reads and writes (device pointers; the fp32
+// scratch rows live in the backward workspace).
+struct BackwardArgs {
+    const void *q, *k, *v, *P_q, *P_k, *o_s, *dO;     // storage dtype
+    const float *C, *gate, *lse;
+    const int32_t* kv_idx;
+    const float2* tab;
+    const void *qr, *kr;                                // rotated copies
+    float *dOs, *Dv, *dq_acc, *dk_acc, *dv_acc, *dg_h;  // fp32 scratch
+    float *partC, *partPq, *partPk, *dC;                // per-chunk partials, reduced dC
+    int32_t *tr_off, *tr_list;                          // transposed mask
+    void *dq, *dk, *dv;                                 // outputs, storage dtype
+    float *dP_q, *dP_k, *dgate;                         // outputs, fp32 (dgate nullable)
+};
+cudaError_t launch_backward(rola_dtype_t dt, const Shape& s, const BackwardArgs& a, cudaStream_t st);
+
 cudaError_t launch_gate(rola_dtype_t dt, long long rows, int D, const void* X, const void* w, float b, float* g,
                         cudaStream_t st);
 

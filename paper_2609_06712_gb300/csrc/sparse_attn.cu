@@ -24,7 +24,7 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
                                                                       const float* __restrict__ kr,
                                                                       const float* __restrict__ v,
                                                                       const int32_t* __restrict__ kv_idx,
-                                                                      float* __restrict__ o)
+                                                                      float* __restrict__ o, float* __restrict__ lse)
 {
     extern __shared__ float fsm[];
     float* Qs = fsm;                       // [64][129]
@@ -93,6 +93,7 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
     const int n = s.cube ? cube_token(s, cube_origin(s, qb), row) : qb * kBlock + row;
     if (n >= 0 && n < s.N) {
         float inv = 1.0f / l_run;
+        if (lse && quarter == 0) lse[(size_t)bh * s.N + n] = m_run + logf(l_run);
         float* on = o + ((size_t)bh * s.N + n) * kDh;
 #pragma unroll
         for (int i = 0; i < 32; ++i) on[quarter + 4 * i] = acc[i] * inv;
@@ -100,16 +101,16 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
 }
 
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr, const void* v,
-                               const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st)
+                               const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status, cudaStream_t st)
 {
-    if (dt == ROLA_BF16) return launch_sparse_attn_tc(s, qr, kr, v, kv_idx, o_s, status, st);
+    if (dt == ROLA_BF16) return launch_sparse_attn_tc(s, qr, kr, v, kv_idx, o_s, lse, status, st);
     dim3 grid(s.nB, s.B * s.H);
     size_t smem = sizeof(float) * (2 * kBlock * kPad + kBlock * kDh + kBlock * 65);
     cudaError_t e = cudaFuncSetAttribute(sparse_attn_f32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
     sparse_attn_f32_kernel<<<grid, kF32Threads, smem, st>>>(s, (const float*)qr, (const float*)kr, (const float*)v,
-                                                            kv_idx, (float*)o_s);
+                                                            kv_idx, (float*)o_s, lse);
     return cudaGetLastError();
 }
 

@@ -98,6 +98,7 @@ struct Params {
     Shape s;
     const int32_t* kv_idx;
     __nv_bfloat16* o;
+    float* lse;           // nullable: log-sum-exp per query row (natural log)
     DeviceStatus* status;
     int total_items;      // B*H*nB
     int tiles;            // ceil(n_keep / 2)
@@ -533,7 +534,17 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
             // reduction overlaps the last P V; then thread wtid writes d = wtid of
             // this warpgroup's 32 query rows, so each warp store is one 64-byte segment
             column_reduce<false>(l, sm, wg, wtid, sm.inv_l + col0);
-            if (wtid < kCols) sm.inv_l[col0 + wtid] = 1.0f / sm.inv_l[col0 + wtid];
+            if (wtid < kCols) {
+                const float lsum = sm.inv_l[col0 + wtid];
+                if (p.lse) {
+                    // sum_j exp(s_j / sqrt d) = 2^(m_q) l_q, with -m_q stored in sm.m (log2 units)
+                    int n;
+                    if constexpr (kCube) n = cube_token(s, cube_origin_rcp(s, qb), col0 + wtid);
+                    else n = qb * 64 + col0 + wtid < s.N ? qb * 64 + col0 + wtid : -1;
+                    if (n >= 0) p.lse[(size_t)bh * s.N + n] = (log2f(lsum) - sm.m[col0 + wtid]) * 0.6931471805599453f;
+                }
+                sm.inv_l[col0 + wtid] = 1.0f / lsum;
+            }
             bar_sync(1 + wg, kWGThreads);
             if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
@@ -625,7 +636,8 @@ bool make_block_map(CUtensorMap* m, const void* ptr, const Shape& s, int rows)
 }
 
 cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr, const void* v,
-                                  const int32_t* kv_idx, void* o_s, DeviceStatus* status, cudaStream_t st)
+                                  const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status,
+                                  cudaStream_t st)
 {
     // the maps span the block-ordered rows (the token order itself for contiguous chunks)
     Shape rows = s;
@@ -642,6 +654,7 @@ cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr
     p.s = s;
     p.kv_idx = kv_idx;
     p.o = static_cast<__nv_bfloat16*>(o_s);
+    p.lse = lse;
     p.status = status;
     p.total_items = s.B * s.H * s.nB;
     p.tiles = (s.n_keep + 1) / 2;

@@ -81,6 +81,9 @@ def _load():
         "rola_lowrank_apply": (st, [cfgp, P, P, P, P, P, P, P, S, P]),
         "rola_forward": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P]),
         "rola_forward_timed": (st, [cfgp, P, P, P, P, P, P, P, P, P, S, P, P]),
+        "rola_forward_train": (st, [cfgp, P, P, P, P, P, P, P, P, P, P, P, P, S, P]),
+        "rola_backward_workspace_bytes": (S, [cfgp]),
+        "rola_backward": (st, [cfgp] + [P] * 18 + [S, P]),
         "rola_gate": (st, [cfgp, P, P, ctypes.c_float, ctypes.c_int32, P, P]),
         "rola_get_device_status": (st, [P, P]),
         "rola_status_string": (ctypes.c_char_p, [st]),
@@ -194,6 +197,26 @@ def forward(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, stream=None):
                              _p(kv_idx_out), _p(ws), ws.numel(), _stream(stream)), "rola_forward")
 
 
+def forward_train(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, o_s, lse, C, ws, stream=None):
+    """rola_forward keeping O^s, the per-row log-sum-exp and C for backward()."""
+    _check(_lib.rola_forward_train(ctypes.byref(c), _p(q), _p(k), _p(v), _p(P_q), _p(P_k), _p(gate), _p(o),
+                                   _p(kv_idx_out), _p(o_s), _p(lse), _p(C), _p(ws), ws.numel(), _stream(stream)),
+           "rola_forward_train")
+
+
+def backward_workspace(c: RolaConfig, device="cuda") -> torch.Tensor:
+    n = _lib.rola_backward_workspace_bytes(ctypes.byref(c))
+    if n == 0:
+        raise RolaError(ROLA_ERR_UNSUPPORTED, "rola_backward_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def backward(c, q, k, v, P_q, P_k, gate, kv_idx, o_s, lse, C, dO, dq, dk, dv, dP_q, dP_k, dgate, ws, stream=None):
+    _check(_lib.rola_backward(ctypes.byref(c), _p(q), _p(k), _p(v), _p(P_q), _p(P_k), _p(gate), _p(kv_idx),
+                              _p(o_s), _p(lse), _p(C), _p(dO), _p(dq), _p(dk), _p(dv), _p(dP_q), _p(dP_k),
+                              _p(dgate), _p(ws), ws.numel(), _stream(stream)), "rola_backward")
+
+
 def gate(c, X, w_g, b_g: float, gate_out, stream=None):
     """Token gate g = sigmoid(X w_g + b_g) into gate_out (fp32 [B][N]); X [B][N][d_model]."""
     _check(_lib.rola_gate(ctypes.byref(c), _p(X), _p(w_g), float(b_g), int(X.shape[-1]), _p(gate_out),
@@ -231,3 +254,43 @@ class RoLAAttention:
             kv_idx = torch.empty((c.B, c.H, self.nB, self.n_keep), dtype=torch.int32, device=q.device)
         forward(c, q, k, v, P_q, P_k, gate, out, kv_idx, self.ws, stream)
         return out, kv_idx
+
+
+class RoLAFunction(torch.autograd.Function):
+    """The module as a differentiable torch op on this library's kernels:
+    rola_forward_train in forward, rola_backward in backward (torch allocates the
+    buffers and casts the fp32 P gradients to P's dtype; it computes nothing else).
+
+    ``RoLAFunction.apply(c, q, k, v, P_q, P_k, gate)`` returns O; ``gate`` may be None."""
+
+    @staticmethod
+    def forward(ctx, c, q, k, v, P_q, P_k, gate):
+        B, H, N = c.B, c.H, c.N
+        dev = q.device
+        ws = workspace(c, dev)
+        o = torch.empty_like(q)
+        o_s = torch.empty_like(q)
+        kv = torch.empty((B, H, num_blocks(c), num_keep(c)), dtype=torch.int32, device=dev)
+        lse = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+        C = torch.empty((B, H, c.r, 128), dtype=torch.float32, device=dev)
+        forward_train(c, q, k, v, P_q, P_k, gate, o, kv, o_s, lse, C, ws)
+        ctx.c = c
+        ctx.has_gate = gate is not None
+        ctx.save_for_backward(q, k, v, P_q, P_k, gate if gate is not None else torch.empty(0, device=dev),
+                              kv, o_s, lse, C)
+        return o
+
+    @staticmethod
+    def backward(ctx, dO):
+        q, k, v, P_q, P_k, gate, kv, o_s, lse, C = ctx.saved_tensors
+        c = ctx.c
+        gate = gate if ctx.has_gate else None
+        dO = dO.contiguous()
+        dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+        dP_q = torch.empty(P_q.shape, dtype=torch.float32, device=q.device)
+        dP_k = torch.empty(P_k.shape, dtype=torch.float32, device=q.device)
+        dgate = torch.empty((c.B, c.N), dtype=torch.float32, device=q.device) if ctx.has_gate else None
+        ws = backward_workspace(c, q.device)
+        backward(c, q, k, v, P_q, P_k, gate, kv, o_s, lse, C, dO, dq, dk, dv, dP_q, dP_k, dgate, ws)
+        return None, dq, dk, dv, dP_q.to(P_q.dtype), dP_k.to(P_k.dtype), dgate
+

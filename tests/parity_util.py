@@ -36,6 +36,27 @@ def assert_close(got, want, dtype_is_bf16, what, unit_rms=False):
     return rl, ma
 
 
+# Gradients (backward pass) in bf16: rel-L2 as for the outputs, max-abs in units
+# of the reference's largest magnitude -- gradient entries spread to ~10x their
+# RMS, and one bf16 rounding of the largest is 2^-9 of it; the bar allows about
+# five roundings' worth along the chain (rotated copies, O^s, the gradient).
+BF16_GRAD_MAX_REL = 1e-2
+
+
+def assert_close_grad(got, want, dtype_is_bf16, what):
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    assert got.shape == want.shape, (what, got.shape, want.shape)
+    assert np.isfinite(got).all(), f"{what}: non-finite values"
+    rl = rel_l2(got, want)
+    if dtype_is_bf16:
+        ma = float(np.abs(got - want).max()) / max(float(np.abs(want).max()), 1e-300)
+        assert rl <= BF16_REL_L2 and ma <= BF16_GRAD_MAX_REL, f"{what}: rel-L2 {rl:.3e}, max-abs/max {ma:.3e}"
+    else:
+        assert rl <= F32_REL_L2, f"{what}: rel-L2 {rl:.3e}"
+    return rl
+
+
 def check_mask(gpu_idx, orc_idx, scores, gap, tau, nB):
     """Mask parity.  Rows whose oracle gap (n_keep-th minus (n_keep+1)-th score)
     exceeds the fp32 error bound tau must match bit for bit.  On the remaining

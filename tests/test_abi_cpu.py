@@ -180,6 +180,40 @@ def test_status_strings(rl):
     assert b"unknown" in L.rola_status_string(42)
 
 
+def test_training_entry_points_are_checked_before_launch(rl):
+    """rola_forward_train and rola_backward reject bad arguments before any launch: an invalid
+    config, missing saved tensors, a cube-geometry backward, a short or misaligned workspace."""
+    L = rl.library()
+    P = ctypes.c_void_p
+    p, w = P(0x10000), P(0x100000)
+    c = cfg_tiny(rl)
+    bad = cfg_tiny(rl, r=15)
+    cube = cfg_tiny(rl, block_geometry=rl.ROLA_BLOCK_CUBE)
+    need = L.rola_backward_workspace_bytes(ctypes.byref(c))
+    assert need > rl.workspace_bytes(c) and L.rola_backward_workspace_bytes(ctypes.byref(cube)) == 0
+    assert L.rola_backward_workspace_bytes(ctypes.byref(bad)) == 0
+
+    def bwd(cfg, ptr=p, ws=w, ws_bytes=1 << 40):
+        return L.rola_backward(ctypes.byref(cfg), *([ptr] * 17), ws, ws_bytes, None)
+
+    assert bwd(bad) == rl.ROLA_ERR_INVALID_ARG
+    assert bwd(cube) == rl.ROLA_ERR_UNSUPPORTED
+    assert bwd(c, ptr=P(0)) == rl.ROLA_ERR_INVALID_ARG
+    assert bwd(c, ptr=P(0x10008)) == rl.ROLA_ERR_INVALID_ARG
+    assert bwd(c, ws_bytes=need - 1) == rl.ROLA_ERR_WORKSPACE
+    assert bwd(c, ws=P(0x100080)) == rl.ROLA_ERR_WORKSPACE
+
+    def fwd(cfg, o_s=p, lse=p, C=p, kv=p, ws_bytes=1 << 40):
+        return L.rola_forward_train(ctypes.byref(cfg), p, p, p, p, p, None, P(0x20000), kv, o_s, lse, C, w,
+                                    ws_bytes, None)
+
+    assert fwd(bad) == rl.ROLA_ERR_INVALID_ARG
+    for missing in ({"o_s": None}, {"lse": None}, {"C": None}, {"kv": None}):
+        assert fwd(c, **missing) == rl.ROLA_ERR_INVALID_ARG
+    assert fwd(c, o_s=P(0x20000)) == rl.ROLA_ERR_INVALID_ARG           # o_s may not alias o
+    assert fwd(c, ws_bytes=rl.workspace_bytes(c) - 1) == rl.ROLA_ERR_WORKSPACE
+
+
 def test_gate_arguments_are_checked_before_launch(rl):
     """Every call here is rejected by validation, so no kernel is launched on the dummy pointers."""
     L = rl.library()
