@@ -293,15 +293,22 @@ def run_backward(args, cfg, c, x, stream, ws, rank):
         # low-rank backward's six N x r x d_h products (u, y, dq~, dq, dC, dP_q on the query side; u, dk~,
         # dv, dk, dP_k on the key side: 11 products of 2 N d_h r flops)
         flops = 2.5 * sparse_fw + 11 * 2.0 * B * H * N * 128 * r
+        if c.dtype == rola.ROLA_BF16:
+            # the sparse products run on the tensor cores (bf16 mma.sync, fp32 accumulation)
+            peaks, src = load_peaks()
+            peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+            bound, peak_src = "tensor", f"{src} bf16_tflops_sustained"
+        else:
+            peak, bound = FP32_SIMT_PEAK_TFLOPS, "alu"
+            peak_src = "fp32 FMA lanes x clock (152 SMs x 128 x 2 x 2.07 GHz), derived"
         print(json.dumps({"entry": "rola_backward", "ms_forward_train": ms_fw, "ms_backward": ms_bw,
                           "train_step_tokens_per_s": job_throughput(B * N, ms_fw + ms_bw, ws),
                           "backward_flops": flops, "achieved_tflops": flops / (ms_bw * 1e-3) / 1e12,
-                          "bound": "alu", "peak_tflops": FP32_SIMT_PEAK_TFLOPS,
-                          "frac": flops / (ms_bw * 1e-3) / 1e12 / FP32_SIMT_PEAK_TFLOPS,
-                          "peak_source": "fp32 FMA lanes x clock (152 SMs x 128 x 2 x 2.07 GHz), derived",
+                          "bound": bound, "peak_tflops": peak,
+                          "frac": flops / (ms_bw * 1e-3) / 1e12 / peak, "peak_source": peak_src,
                           "steps": args.steps, "warmup": args.warmup,
                           "config": {"workload": cfg["name"], "B": B, "H": H, "N": N, "r": r, "keep": cfg["keep"],
-                                     "dtype": "bf16 storage, fp32 arithmetic"}}), flush=True)
+                                     "dtype": "bf16"}}), flush=True)
 
 
 def run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank):

@@ -227,7 +227,7 @@ BwdWorkspace bwd_layout(const rola_config_t& c)
     w.kr = off; off = align_up(off + esz * rows * kDh);
     w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
-    w.dOs = off; off = align_up(off + 4 * rows * kDh);
+    w.dOs = off; off = align_up(off + esz * rows * kDh);
     w.Dv = off; off = align_up(off + 4 * rows);
     w.dq = off; off = align_up(off + 4 * rows * kDh);
     w.dk = off; off = align_up(off + 4 * rows * kDh);
@@ -479,7 +479,7 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
     a.C = C; a.gate = gate; a.lse = lse; a.kv_idx = kv_idx;
     a.tab = at<float2>(ws, w.table);
     a.qr = at<void>(ws, w.qr); a.kr = at<void>(ws, w.kr);
-    a.dOs = at<float>(ws, w.dOs); a.Dv = at<float>(ws, w.Dv);
+    a.dOs = at<void>(ws, w.dOs); a.Dv = at<float>(ws, w.Dv);
     a.dq_acc = at<float>(ws, w.dq); a.dk_acc = at<float>(ws, w.dk); a.dv_acc = at<float>(ws, w.dv);
     a.dg_h = at<float>(ws, w.dg);
     a.partC = at<float>(ws, w.partC); a.partPq = at<float>(ws, w.partPq); a.partPk = at<float>(ws, w.partPk);

@@ -166,7 +166,8 @@ struct BackwardArgs {
     const int32_t* kv_idx;
     const float2* tab;
     const void *qr, *kr;                                // rotated copies
-    float *dOs, *Dv, *dq_acc, *dk_acc, *dv_acc, *dg_h;  // fp32 scratch
+    void* dOs;                                          // dL/dO^s, storage dtype
+    float *Dv, *dq_acc, *dk_acc, *dv_acc, *dg_h;        // fp32 scratch
     float *partC, *partPq, *partPk, *dC;                // per-chunk partials, reduced dC
     int32_t *tr_off, *tr_list;                          // transposed mask
     void *dq, *dk, *dv;                                 // outputs, storage dtype
