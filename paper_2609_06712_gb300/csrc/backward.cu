@@ -702,6 +702,416 @@ __device__ __forceinline__ void store_rows(const Shape& s, const float2* tab, co
     }
 }
 
+// ---------------------------------------------------------------------------
+// bf16 low-rank backward on the tensor cores: one CTA (4 warps, 16 tokens
+// each) per (64-token chunk, head), R = r rounded up to 16 (rows r .. R-1 of
+// P read as zero, so those features and their gradients are zero).  A
+// thread's accumulator columns 8 nt + 2 tig, +1 are one feature pair (the
+// layout the forward's readout uses), so the rotation, phi and phi' are
+// thread-local.  Token-contracting products (dC = F^T dY, dP = dU^T X) read
+// the bf16 copies the warps leave in shared memory, A through ldmatrix.trans.
+
+// A = (a 16-row slice of a [k][m] tile)^T: ldmatrix.trans lane address for
+// m rows from m0 (chunks m0/8, m0/8 + 1) and k rows from k0.
+__device__ __forceinline__ uint32_t at_addr(uint32_t t, int k0, int m0, int lane)
+{
+    return t + sw128(k0 + (lane & 7) + (lane >> 4) * 8, (m0 >> 3) + ((lane >> 3) & 1));
+}
+
+// C-fragment pairs (rows g, g + 8) to A fragments over k = 16 ks.. (see mma_frag_x_tile).
+template <int NT>
+__device__ __forceinline__ void frag_a(const float (&w)[NT][4], int ks, uint32_t& a0, uint32_t& a1, uint32_t& a2,
+                                       uint32_t& a3)
+{
+    a0 = pack_bf16(w[2 * ks][0], w[2 * ks][1]);
+    a1 = pack_bf16(w[2 * ks][2], w[2 * ks][3]);
+    a2 = pack_bf16(w[2 * ks + 1][0], w[2 * ks + 1][1]);
+    a3 = pack_bf16(w[2 * ks + 1][2], w[2 * ks + 1][3]);
+}
+
+// rows [0, rows) of a [rows][128] array (bf16 or fp32) into a swizzled bf16 tile;
+// rows [rows, R) zero.
+template <typename T>
+__device__ void weight_tile(uint8_t* base, uint32_t off, const T* src, int rows, int R)
+{
+    for (int e = threadIdx.x; e < R * 64; e += kMT) {
+        const int a = e >> 6, d = (e & 63) * 2;
+        const float x0 = a < rows ? to_f(src[(size_t)a * kDh + d]) : 0.0f;
+        const float x1 = a < rows ? to_f(src[(size_t)a * kDh + d + 1]) : 0.0f;
+        *reinterpret_cast<uint32_t*>(base + off + sw128(a, d >> 3) + (d & 7) * 2) = pack_bf16(x0, x1);
+    }
+}
+
+__device__ __forceinline__ void put_pair(uint8_t* base, uint32_t off, int row, int col, float x0, float x1)
+{
+    *reinterpret_cast<uint32_t*>(base + off + sw128(row, col >> 3) + (col & 7) * 2) = pack_bf16(x0, x1);
+}
+
+// acc[R/8][4] = A(16 x 128: rows r0 of tile ta) * (R rows of tile tb)^T
+template <int R>
+__device__ __forceinline__ void mma_rows_x_w(float (&acc)[R / 8][4], uint32_t ta, int r0, uint32_t tb, int lane)
+{
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(a_addr(ta, r0, kk, lane), a0, a1, a2, a3);
+#pragma unroll
+        for (int np = 0; np < R / 16; ++np) {
+            uint32_t b0, b1, b2, b3;
+            ldsm_x4(bn_addr(tb, 16 * np, kk, lane), b0, b1, b2, b3);
+            mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
+            mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+        }
+    }
+}
+
+// acc[16][4] = A(16 x R from fragments w) * (R rows x 128 of tile tb)
+template <int R>
+__device__ __forceinline__ void mma_wfrag_x_w(float (&acc)[16][4], const float (&w)[R / 8][4], uint32_t tb, int lane)
+{
+#pragma unroll
+    for (int ks = 0; ks < R / 16; ++ks) {
+        uint32_t a0, a1, a2, a3;
+        frag_a(w, ks, a0, a1, a2, a3);
+#pragma unroll
+        for (int np = 0; np < 8; ++np) {
+            uint32_t b0, b1, b2, b3;
+            ldsm_x4_t(bt_addr(tb, 16 * ks, 2 * np, lane), b0, b1, b2, b3);
+            mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
+            mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+        }
+    }
+}
+
+// acc[R/8][4] = A(16 x 128 from fragments w[16][4]) * (R rows of tile tb)^T
+template <int R>
+__device__ __forceinline__ void mma_dfrag_x_wt(float (&acc)[R / 8][4], const float (&w)[16][4], uint32_t tb, int lane)
+{
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+        uint32_t a0, a1, a2, a3;
+        frag_a(w, kk, a0, a1, a2, a3);
+#pragma unroll
+        for (int np = 0; np < R / 16; ++np) {
+            uint32_t b0, b1, b2, b3;
+            ldsm_x4(bn_addr(tb, 16 * np, kk, lane), b0, b1, b2, b3);
+            mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
+            mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+        }
+    }
+}
+
+// part[a][d] (R x 128, fp32, first r rows stored) = sum over the chunk's 64 tokens of
+// A[t][a] B[t][d], A and B swizzled bf16 tiles; warp w takes the 16 x 32 output tiles w, w + 4, ...
+template <int R>
+__device__ void mma_outer(uint32_t tA, uint32_t tB, int r, float* part, int warp, int lane)
+{
+    const int g = lane >> 2, tig = lane & 3;
+    for (int tile = warp; tile < (R / 16) * 4; tile += 4) {
+        const int a0 = (tile >> 2) * 16, d0 = (tile & 3) * 32;
+        float acc[4][4] = {};
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            uint32_t x0, x1, x2, x3;
+            ldsm_x4_t(at_addr(tA, 16 * ks, a0, lane), x0, x1, x2, x3);
+#pragma unroll
+            for (int np = 0; np < 2; ++np) {
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_t(bt_addr(tB, 16 * ks, (d0 >> 3) + 2 * np, lane), b0, b1, b2, b3);
+                mma_bf16(acc[2 * np], x0, x1, x2, x3, b0, b1);
+                mma_bf16(acc[2 * np + 1], x0, x1, x2, x3, b2, b3);
+            }
+        }
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt) {
+            const int d = d0 + 8 * nt + 2 * tig;
+            if (a0 + g < r) *reinterpret_cast<float2*>(part + (size_t)(a0 + g) * kDh + d) = make_float2(acc[nt][0], acc[nt][1]);
+            if (a0 + g + 8 < r)
+                *reinterpret_cast<float2*>(part + (size_t)(a0 + g + 8) * kDh + d) = make_float2(acc[nt][2], acc[nt][3]);
+        }
+    }
+}
+
+// u (fragments) -> features (fragments) for rows t0, t0 + 8 of the chunk, tokens n0 + t.
+template <int R>
+__device__ __forceinline__ void frag_features(const Shape& s, const float2* tab, const float (&u)[R / 8][4],
+                                              float (&f)[R / 8][4], int n0, int t0, int tig, ActBwd act)
+{
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int n = n0 + t0 + 8 * h;
+#pragma unroll
+        for (int nt = 0; nt < R / 8; ++nt) {
+            const int a = 8 * nt + 2 * tig;
+            float2 y = make_float2(0.0f, 0.0f);
+            if (n < s.N && a < s.r) y = lowrank_pair(u[nt][2 * h], u[nt][2 * h + 1], rope_cs(tab, s, n, a >> 1), s.lr_rope, act);
+            f[nt][2 * h] = y.x;
+            f[nt][2 * h + 1] = y.y;
+        }
+    }
+}
+
+// dL/du (fragments, over df) for rows t0, t0 + 8.
+template <int R>
+__device__ __forceinline__ void frag_features_bwd(const Shape& s, const float2* tab, const float (&u)[R / 8][4],
+                                                  float (&df)[R / 8][4], int n0, int t0, int tig, ActBwd act)
+{
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int n = n0 + t0 + 8 * h;
+#pragma unroll
+        for (int nt = 0; nt < R / 8; ++nt) {
+            const int a = 8 * nt + 2 * tig;
+            float2 d = make_float2(0.0f, 0.0f);
+            if (n < s.N && a < s.r)
+                d = lowrank_pair_bwd(u[nt][2 * h], u[nt][2 * h + 1], df[nt][2 * h], df[nt][2 * h + 1],
+                                     rope_cs(tab, s, n, a >> 1), s.lr_rope, act);
+            df[nt][2 * h] = d.x;
+            df[nt][2 * h + 1] = d.y;
+        }
+    }
+}
+
+template <int R>
+__global__ void __launch_bounds__(kMT) lr_bwd_q_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
+                                                           const __nv_bfloat16* __restrict__ Pq,
+                                                           const float* __restrict__ C,
+                                                           const float* __restrict__ gate,
+                                                           const __nv_bfloat16* __restrict__ o_s,
+                                                           const __nv_bfloat16* __restrict__ dO,
+                                                           const float2* __restrict__ tab,
+                                                           __nv_bfloat16* __restrict__ dOs, float* __restrict__ Dv,
+                                                           float* __restrict__ dq_acc, float* __restrict__ dg_h,
+                                                           float* __restrict__ partC, float* __restrict__ partPq)
+{
+    extern __shared__ __align__(128) uint8_t msm[];
+    const uint32_t b0 = smem_u32(msm);
+    // layout: X [64] | P [R rows] | C [R rows] | F [64] | dY [64] | dU [64] (rows of 256 B)
+    const uint32_t sX = b0, sP = b0 + kTile, sC = b0 + kTile + R * 256, sF = sC + R * 256, sY = sF + kTile,
+                   sU = sY + kTile;
+    const int chunk = blockIdx.x, bh = blockIdx.y, h = bh % s.H, b = bh / s.H;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tig = lane & 3;
+    const int n0 = chunk * 64, t0 = 16 * warp + g;
+    const size_t head = (size_t)bh * s.N * kDh;
+    const ActBwd act{s.lr_act};
+    tile_async(sX, q + head, n0, s.N);
+    cp_async_commit();
+    weight_tile(msm, sP - b0, Pq + (size_t)h * s.r * kDh, s.r, R);
+    weight_tile(msm, sC - b0, C + (size_t)bh * s.r * kDh, s.r, R);
+    cp_async_wait<0>();
+    __syncthreads();
+    // u = P_q q, features
+    float u[R / 8][4] = {}, f[R / 8][4];
+    mma_rows_x_w<R>(u, sX, 16 * warp, sP, lane);
+    frag_features<R>(s, tab, u, f, n0, t0, tig, act);
+#pragma unroll
+    for (int nt = 0; nt < R / 8; ++nt) {
+        put_pair(msm, sF - b0, t0, 8 * nt + 2 * tig, f[nt][0], f[nt][1]);
+        put_pair(msm, sF - b0, t0 + 8, 8 * nt + 2 * tig, f[nt][2], f[nt][3]);
+    }
+    // y = q~^T C
+    float y[16][4] = {};
+    mma_wfrag_x_w<R>(y, f, sC, lane);
+    // fusion and RMSNorm backward, rows t0 and t0 + 8 (the quad of a row holds its 128 columns)
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+        const int n = n0 + t0 + 8 * hh;
+        const bool valid = n < s.N;
+        float os[32], go[32];
+        float syy = 0.0f, sos = 0.0f;
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt) {
+            const int d = 8 * nt + 2 * tig;
+            float2 ov = make_float2(0.0f, 0.0f), gv = make_float2(0.0f, 0.0f);
+            if (valid) {
+                ov = unpack_bf16(*reinterpret_cast<const uint32_t*>(o_s + head + (size_t)n * kDh + d));
+                gv = unpack_bf16(*reinterpret_cast<const uint32_t*>(dO + head + (size_t)n * kDh + d));
+            }
+            os[2 * nt] = ov.x; os[2 * nt + 1] = ov.y;
+            go[2 * nt] = gv.x; go[2 * nt + 1] = gv.y;
+            syy = fmaf(y[nt][2 * hh], y[nt][2 * hh], fmaf(y[nt][2 * hh + 1], y[nt][2 * hh + 1], syy));
+            sos = fmaf(ov.x, ov.x, fmaf(ov.y, ov.y, sos));
+        }
+        syy += __shfl_xor_sync(0xffffffffu, syy, 1);
+        syy += __shfl_xor_sync(0xffffffffu, syy, 2);
+        sos += __shfl_xor_sync(0xffffffffu, sos, 1);
+        sos += __shfl_xor_sync(0xffffffffu, sos, 2);
+        const float irho = 1.0f / sqrtf(syy / (float)kDh + s.eps_lr);
+        const float rp = sqrtf(sos / (float)kDh + s.eps_fuse);
+        const float gt = valid ? (gate ? gate[(size_t)b * s.N + n] : s.default_gate) : 0.0f;
+        float a_dot = 0.0f;
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt)
+            a_dot = fmaf(y[nt][2 * hh] * irho, go[2 * nt], fmaf(y[nt][2 * hh + 1] * irho, go[2 * nt + 1], a_dot));
+        a_dot += __shfl_xor_sync(0xffffffffu, a_dot, 1);
+        a_dot += __shfl_xor_sync(0xffffffffu, a_dot, 2);
+        const float coef = gt * a_dot / ((float)kDh * rp);
+        float dsum = 0.0f, od = 0.0f;
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt) {
+            const int d = 8 * nt + 2 * tig;
+            const float gs0 = fmaf(coef, os[2 * nt], go[2 * nt]), gs1 = fmaf(coef, os[2 * nt + 1], go[2 * nt + 1]);
+            if (valid) *reinterpret_cast<uint32_t*>(dOs + head + (size_t)n * kDh + d) = pack_bf16(gs0, gs1);
+            dsum = fmaf(gs0, os[2 * nt], fmaf(gs1, os[2 * nt + 1], dsum));
+            od = fmaf(y[nt][2 * hh] * irho, gt * rp * go[2 * nt], fmaf(y[nt][2 * hh + 1] * irho, gt * rp * go[2 * nt + 1], od));
+        }
+        dsum += __shfl_xor_sync(0xffffffffu, dsum, 1);
+        dsum += __shfl_xor_sync(0xffffffffu, dsum, 2);
+        od += __shfl_xor_sync(0xffffffffu, od, 1);
+        od += __shfl_xor_sync(0xffffffffu, od, 2);
+        if (tig == 0 && valid) {
+            Dv[(size_t)bh * s.N + n] = dsum;
+            dg_h[(size_t)bh * s.N + n] = rp * a_dot;
+        }
+        // y <- dy (rows of invalid tokens zero)
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt) {
+            const float dy0 = valid ? (gt * rp * go[2 * nt] - y[nt][2 * hh] * irho * od / (float)kDh) * irho : 0.0f;
+            const float dy1 = valid ? (gt * rp * go[2 * nt + 1] - y[nt][2 * hh + 1] * irho * od / (float)kDh) * irho : 0.0f;
+            y[nt][2 * hh] = dy0;
+            y[nt][2 * hh + 1] = dy1;
+            put_pair(msm, sY - b0, t0 + 8 * hh, 8 * nt + 2 * tig, dy0, dy1);
+        }
+    }
+    // dq~ = C dy, then du
+    float df[R / 8][4] = {};
+    mma_dfrag_x_wt<R>(df, y, sC, lane);
+    frag_features_bwd<R>(s, tab, u, df, n0, t0, tig, act);
+#pragma unroll
+    for (int nt = 0; nt < R / 8; ++nt) {
+        put_pair(msm, sU - b0, t0, 8 * nt + 2 * tig, df[nt][0], df[nt][1]);
+        put_pair(msm, sU - b0, t0 + 8, 8 * nt + 2 * tig, df[nt][2], df[nt][3]);
+    }
+    // dq (low-rank part) = P_q^T du, fp32 rows
+    {
+        float dq[16][4] = {};
+        mma_wfrag_x_w<R>(dq, df, sP, lane);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int n = n0 + t0 + 8 * hh;
+            if (n >= s.N) continue;
+#pragma unroll
+            for (int nt = 0; nt < 16; ++nt)
+                *reinterpret_cast<float2*>(dq_acc + head + (size_t)n * kDh + 8 * nt + 2 * tig) =
+                    make_float2(dq[nt][2 * hh], dq[nt][2 * hh + 1]);
+        }
+    }
+    __syncthreads();
+    const size_t slot = ((size_t)bh * s.nC + chunk) * s.r * kDh;
+    mma_outer<R>(sF, sY, s.r, partC + slot, warp, lane);
+    mma_outer<R>(sU, sX, s.r, partPq + slot, warp, lane);
+}
+
+template <int R>
+__global__ void __launch_bounds__(kMT) lr_bwd_k_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ k,
+                                                           const __nv_bfloat16* __restrict__ v,
+                                                           const __nv_bfloat16* __restrict__ Pk,
+                                                           const float* __restrict__ dC,
+                                                           const float2* __restrict__ tab,
+                                                           float* __restrict__ dk_acc, float* __restrict__ dv_acc,
+                                                           float* __restrict__ partPk)
+{
+    extern __shared__ __align__(128) uint8_t msm[];
+    const uint32_t b0 = smem_u32(msm);
+    // layout: X (k) [64] | V [64] | P [R rows] | dC [R rows] | dU [64]
+    const uint32_t sX = b0, sV = b0 + kTile, sP = b0 + 2 * kTile, sC = sP + R * 256, sU = sC + R * 256;
+    const int chunk = blockIdx.x, bh = blockIdx.y, h = bh % s.H;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tig = lane & 3;
+    const int n0 = chunk * 64, t0 = 16 * warp + g;
+    const size_t head = (size_t)bh * s.N * kDh;
+    const ActBwd act{s.lr_act};
+    tile_async(sX, k + head, n0, s.N);
+    tile_async(sV, v + head, n0, s.N);
+    cp_async_commit();
+    weight_tile(msm, sP - b0, Pk + (size_t)h * s.r * kDh, s.r, R);
+    weight_tile(msm, sC - b0, dC + (size_t)bh * s.r * kDh, s.r, R);
+    cp_async_wait<0>();
+    __syncthreads();
+    float u[R / 8][4] = {}, f[R / 8][4];
+    mma_rows_x_w<R>(u, sX, 16 * warp, sP, lane);
+    frag_features<R>(s, tab, u, f, n0, t0, tig, act);
+    // dv (low-rank part) = dC^T k~ : rows of F times dC
+    {
+        float dv[16][4] = {};
+        mma_wfrag_x_w<R>(dv, f, sC, lane);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int n = n0 + t0 + 8 * hh;
+            if (n >= s.N) continue;
+#pragma unroll
+            for (int nt = 0; nt < 16; ++nt)
+                *reinterpret_cast<float2*>(dv_acc + head + (size_t)n * kDh + 8 * nt + 2 * tig) =
+                    make_float2(dv[nt][2 * hh], dv[nt][2 * hh + 1]);
+        }
+    }
+    // dk~ = dC v, then du
+    float df[R / 8][4] = {};
+    mma_rows_x_w<R>(df, sV, 16 * warp, sC, lane);
+    frag_features_bwd<R>(s, tab, u, df, n0, t0, tig, act);
+#pragma unroll
+    for (int nt = 0; nt < R / 8; ++nt) {
+        put_pair(msm, sU - b0, t0, 8 * nt + 2 * tig, df[nt][0], df[nt][1]);
+        put_pair(msm, sU - b0, t0 + 8, 8 * nt + 2 * tig, df[nt][2], df[nt][3]);
+    }
+    {
+        float dk[16][4] = {};
+        mma_wfrag_x_w<R>(dk, df, sP, lane);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int n = n0 + t0 + 8 * hh;
+            if (n >= s.N) continue;
+#pragma unroll
+            for (int nt = 0; nt < 16; ++nt)
+                *reinterpret_cast<float2*>(dk_acc + head + (size_t)n * kDh + 8 * nt + 2 * tig) =
+                    make_float2(dk[nt][2 * hh], dk[nt][2 * hh + 1]);
+        }
+    }
+    __syncthreads();
+    mma_outer<R>(sU, sX, s.r, partPk + ((size_t)bh * s.nC + chunk) * s.r * kDh, warp, lane);
+}
+
+template <int R>
+size_t lr_mma_smem() { return 4 * (size_t)kTile + 2 * (size_t)R * 256; }
+
+template <int R>
+cudaError_t launch_lr_mma_r(const Shape& s, const BackwardArgs& a, bool key_side, cudaStream_t st)
+{
+    const dim3 chunks(s.nC, s.B * s.H);
+    const size_t smem = lr_mma_smem<R>();
+    using bf = __nv_bfloat16;
+    if (!key_side) {
+        cudaError_t e = cudaFuncSetAttribute(lr_bwd_q_mma_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        lr_bwd_q_mma_kernel<R><<<chunks, kMT, smem, st>>>(
+            s, static_cast<const bf*>(a.q), static_cast<const bf*>(a.P_q), a.C, a.gate, static_cast<const bf*>(a.o_s),
+            static_cast<const bf*>(a.dO), a.tab, static_cast<bf*>(a.dOs), a.Dv, a.dq_acc, a.dg_h, a.partC, a.partPq);
+    } else {
+        cudaError_t e = cudaFuncSetAttribute(lr_bwd_k_mma_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        lr_bwd_k_mma_kernel<R><<<chunks, kMT, smem, st>>>(s, static_cast<const bf*>(a.k), static_cast<const bf*>(a.v),
+                                                          static_cast<const bf*>(a.P_k), a.dC, a.tab, a.dk_acc,
+                                                          a.dv_acc, a.partPk);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lr_mma(const Shape& s, const BackwardArgs& a, bool key_side, cudaStream_t st)
+{
+    switch (s.rp) {
+        case 16: return launch_lr_mma_r<16>(s, a, key_side, st);
+        case 32: return launch_lr_mma_r<32>(s, a, key_side, st);
+        case 48: return launch_lr_mma_r<48>(s, a, key_side, st);
+        case 64: return launch_lr_mma_r<64>(s, a, key_side, st);
+        case 80: return launch_lr_mma_r<80>(s, a, key_side, st);
+        case 96: return launch_lr_mma_r<96>(s, a, key_side, st);
+        case 112: return launch_lr_mma_r<112>(s, a, key_side, st);
+        case 128: return launch_lr_mma_r<128>(s, a, key_side, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
 constexpr size_t kMmaSmemBytes = 6 * kTile + 4 * 64 * sizeof(float);
 
 __global__ void __launch_bounds__(kMT) sparse_bwd_dq_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ qr,
@@ -898,18 +1308,28 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
     const T* v = static_cast<const T*>(a.v);
     const T* qr = static_cast<const T*>(a.qr);
     const T* kr = static_cast<const T*>(a.kr);
-    lr_bwd_q_kernel<T><<<chunks, kBT, lsm, st>>>(s, q, static_cast<const T*>(a.P_q), a.C, a.gate,
-                                                 static_cast<const T*>(a.o_s), static_cast<const T*>(a.dO), a.tab,
-                                                 static_cast<T*>(a.dOs), a.Dv, a.dq_acc, a.dg_h, a.partC, a.partPq);
-    e = cudaGetLastError();
+    constexpr bool kMma = std::is_same<T, __nv_bfloat16>::value;
+    if constexpr (kMma) {
+        e = launch_lr_mma(s, a, false, st);
+    } else {
+        lr_bwd_q_kernel<T><<<chunks, kBT, lsm, st>>>(s, q, static_cast<const T*>(a.P_q), a.C, a.gate,
+                                                     static_cast<const T*>(a.o_s), static_cast<const T*>(a.dO), a.tab,
+                                                     static_cast<T*>(a.dOs), a.Dv, a.dq_acc, a.dg_h, a.partC,
+                                                     a.partPq);
+        e = cudaGetLastError();
+    }
     if (e != cudaSuccess) return e;
     const dim3 red((s.r * kDh + 255) / 256, s.B * s.H), red_h((s.r * kDh + 255) / 256, s.H);
     reduce_chunks_kernel<<<red, 256, 0, st>>>(s, a.partC, a.dC, false);
     reduce_chunks_kernel<<<red_h, 256, 0, st>>>(s, a.partPq, a.dP_q, true);
-    lr_bwd_k_kernel<T><<<chunks, kBT, lsm, st>>>(s, k, v, static_cast<const T*>(a.P_k), a.dC, a.tab, a.dk_acc,
-                                                 a.dv_acc, a.partPk);
+    if constexpr (kMma) {
+        e = launch_lr_mma(s, a, true, st);
+        if (e != cudaSuccess) return e;
+    } else {
+        lr_bwd_k_kernel<T><<<chunks, kBT, lsm, st>>>(s, k, v, static_cast<const T*>(a.P_k), a.dC, a.tab, a.dk_acc,
+                                                     a.dv_acc, a.partPk);
+    }
     reduce_chunks_kernel<<<red_h, 256, 0, st>>>(s, a.partPk, a.dP_k, true);
-    constexpr bool kMma = std::is_same<T, __nv_bfloat16>::value;
     if constexpr (kMma) {
         e = cudaFuncSetAttribute(sparse_bwd_dq_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kMmaSmemBytes);

@@ -37,6 +37,8 @@ CASES = {
                              lowrank_act="gelu", lowrank_rope=1),
     "tanh_none_b2": layer(T=3, Hh=6, Ww=8, B=2, H=2, r=32, keep=0.5, seed=74, dist="normal_gate",
                           lowrank_act="tanh", lowrank_rope=2),
+    # a rank that is not a multiple of 16 (the bf16 kernels run at 32 with zero rows of P)
+    "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=76, dist="normal_gate"),
     # latent frames of the 480p layers: 74 blocks (the last of 8 tokens), 15 kept
     "frames_3x30x52": layer(T=3, Hh=30, Ww=52, H=2, r=32, keep=0.2, seed=75, dist="normal_gate"),
 }
