@@ -38,7 +38,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # kernel from one ncu capture of the 480p layer (12 heads x 32760 tokens), scaled
 # to a launch by heads x tokens (the traffic is the streaming q^r, k^r, v reads and
 # the O^s write, which grow in proportion).  Set to None whenever the kernel changes.
-SPARSE_TRAFFIC_PER_HEAD_TOKEN = (303.404288e6 + 86.913792e6) / (12 * 32760)
+SPARSE_TRAFFIC_PER_HEAD_TOKEN = (303.265280e6 + 86.776064e6) / (12 * 32760)
 
 
 def load_peaks():
