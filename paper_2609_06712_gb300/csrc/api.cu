@@ -486,6 +486,7 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
     a.dC = at<float>(ws, w.dC);
     a.tr_off = at<int32_t>(ws, w.tr_off); a.tr_list = at<int32_t>(ws, w.tr_list);
     a.dq = dq; a.dk = dk; a.dv = dv; a.dP_q = dP_q; a.dP_k = dP_k; a.dgate = dgate;
+    a.status = at<DeviceStatus>(ws, w.status);
     ROLA_TRY(launch_backward(cfg->dtype, s, a, st));
     return ROLA_OK;
 }

@@ -598,17 +598,16 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
 }
 
 // ---------------------------------------------------------------------------
-// bf16 sparse backward on the tensor cores (mma.sync m16n8k16, fp32
-// accumulation), FlashAttention-2 style: 4 warps per CTA, each owning 16 rows
-// of the CTA's 64-row block; tiles of 64 rows x 128 bf16 in shared memory with
+// bf16 key-side sparse backward on the tensor cores (mma.sync m16n8k16, fp32
+// accumulation), FlashAttention-2 style: 4 warps per CTA, each owning 16 keys
+// of the CTA's key block; tiles of 64 rows x 128 bf16 in shared memory with
 // 256-byte rows whose 16-byte chunks are XOR-swizzled by the row (sw128),
-// filled by cp.async and double-buffered over the other side's blocks.
-//   dq kernel  (query block):  S = Q K^T, dP = dO V^T, dS = P (dP - D),  dQ += dS K
-//   dkdv kernel (key block):   S^T = K Q^T, dP^T = V dO^T, dS^T = P^T (dP^T - D),
-//                              dV += P^T dO,  dK += dS^T Q
-// The epilogues add the low-rank part (fp32 rows written by the low-rank
-// kernels), rotate dq^r / dk^r back by R^T (a thread's accumulator columns
-// 2 tig, 2 tig + 1 are one RoPE pair) and store the gradients in bf16.
+// filled by cp.async and double-buffered over the query blocks that kept it:
+//   S^T = K Q^T, dP^T = V dO^T, dS^T = P^T (dP^T - D),  dV += P^T dO,  dK += dS^T Q
+// The epilogue adds the low-rank part (fp32 rows written by the low-rank
+// kernels), rotates dk^r back by R^T (a thread's accumulator columns 2 tig,
+// 2 tig + 1 are one RoPE pair) and stores the gradients in bf16.  The
+// query-side gradient runs on tcgen05 (sparse_bwd_tc.cu).
 
 constexpr int kMT = 128;                          // threads of the mma kernels
 constexpr uint32_t kTile = 64 * 256;              // one 64 x 128 bf16 tile
@@ -1114,81 +1113,6 @@ cudaError_t launch_lr_mma(const Shape& s, const BackwardArgs& a, bool key_side, 
 
 constexpr size_t kMmaSmemBytes = 6 * kTile + 4 * 64 * sizeof(float);
 
-__global__ void __launch_bounds__(kMT) sparse_bwd_dq_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ qr,
-                                                                const __nv_bfloat16* __restrict__ kr,
-                                                                const __nv_bfloat16* __restrict__ v,
-                                                                const int32_t* __restrict__ kv_idx,
-                                                                const float* __restrict__ lse,
-                                                                const float* __restrict__ Dv,
-                                                                const __nv_bfloat16* __restrict__ dOs,
-                                                                const float2* __restrict__ tab,
-                                                                const float* __restrict__ dq_lr,
-                                                                __nv_bfloat16* __restrict__ dq)
-{
-    extern __shared__ __align__(128) uint8_t msm[];
-    const uint32_t sQ = smem_u32(msm), sO = sQ + kTile, sKV = sQ + 2 * kTile;     // stage st: K, V at sKV + 2 st kTile
-    float* s_lse = reinterpret_cast<float*>(msm + 6 * kTile);
-    float* s_D = s_lse + 64;
-    const int qb = blockIdx.x, bh = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = lane >> 2, tig = lane & 3;
-    const size_t head = (size_t)bh * s.N * kDh;
-    const int n0 = qb * 64;
-    const int32_t* kept = kv_idx + ((size_t)bh * s.nB + qb) * s.n_keep;
-    tile_async(sQ, qr + head, n0, s.N);
-    tile_async(sO, dOs + head, n0, s.N);
-    if (threadIdx.x < 64) {
-        const int n = n0 + threadIdx.x;
-        s_lse[threadIdx.x] = n < s.N ? lse[(size_t)bh * s.N + n] * 1.4426950408889634f : 0.0f;
-        s_D[threadIdx.x] = n < s.N ? Dv[(size_t)bh * s.N + n] : 0.0f;
-    }
-    int j0 = __ldg(kept);
-    j0 = j0 >= 0 && j0 < s.nB ? j0 : 0;
-    tile_async(sKV, kr + head, j0 * 64, s.N);
-    tile_async(sKV + kTile, v + head, j0 * 64, s.N);
-    cp_async_commit();
-    const float sl2 = 0.08838834764831845f * 1.4426950408889634f;      // log2(e) / sqrt(128)
-    float acc[16][4] = {};
-    for (int it = 0; it < s.n_keep; ++it) {
-        const int j = __ldg(kept + it);
-        if (it + 1 < s.n_keep) {
-            int jn = __ldg(kept + it + 1);
-            jn = jn >= 0 && jn < s.nB ? jn : 0;
-            const uint32_t st = sKV + ((it + 1) & 1) * 2 * kTile;
-            tile_async(st, kr + head, jn * 64, s.N);
-            tile_async(st + kTile, v + head, jn * 64, s.N);
-        }
-        cp_async_commit();
-        cp_async_wait<1>();
-        __syncthreads();
-        const uint32_t sK = sKV + (it & 1) * 2 * kTile, sV = sK + kTile;
-        if (j >= 0 && j < s.nB) {
-            float sc[8][4] = {}, dp[8][4] = {};
-            mma_rows_x_rows(sc, sQ, 16 * warp, sK, lane);
-            mma_rows_x_rows(dp, sO, 16 * warp, sV, lane);
-            const int r0 = 16 * warp + g;
-            const bool v0 = n0 + r0 < s.N, v1 = n0 + r0 + 8 < s.N;
-            const float l0 = s_lse[r0], l1 = s_lse[r0 + 8], D0 = s_D[r0], D1 = s_D[r0 + 8];
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                const int key = j * 64 + 8 * nt + 2 * tig;
-                const bool k0 = key < s.N, k1 = key + 1 < s.N;
-                const float p00 = v0 && k0 ? exp2f(fmaf(sc[nt][0], sl2, -l0)) : 0.0f;
-                const float p01 = v0 && k1 ? exp2f(fmaf(sc[nt][1], sl2, -l0)) : 0.0f;
-                const float p10 = v1 && k0 ? exp2f(fmaf(sc[nt][2], sl2, -l1)) : 0.0f;
-                const float p11 = v1 && k1 ? exp2f(fmaf(sc[nt][3], sl2, -l1)) : 0.0f;
-                sc[nt][0] = p00 * (dp[nt][0] - D0);
-                sc[nt][1] = p01 * (dp[nt][1] - D0);
-                sc[nt][2] = p10 * (dp[nt][2] - D1);
-                sc[nt][3] = p11 * (dp[nt][3] - D1);
-            }
-            mma_frag_x_tile(acc, sc, sK, lane);
-        }
-        __syncthreads();
-    }
-    cp_async_wait<0>();
-    store_rows(s, tab, acc, n0 + 16 * warp, lane, 0.08838834764831845f, true, dq_lr + head, dq + head);
-}
-
 __global__ void __launch_bounds__(kMT) sparse_bwd_dkdv_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ qr,
                                                                   const __nv_bfloat16* __restrict__ kr,
                                                                   const __nv_bfloat16* __restrict__ v,
@@ -1331,15 +1255,11 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
     }
     reduce_chunks_kernel<<<red_h, 256, 0, st>>>(s, a.partPk, a.dP_k, true);
     if constexpr (kMma) {
-        e = cudaFuncSetAttribute(sparse_bwd_dq_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kMmaSmemBytes);
-        if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(sparse_bwd_dkdv_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kMmaSmemBytes);
         if (e != cudaSuccess) return e;
-        sparse_bwd_dq_mma_kernel<<<blocks, kMT, kMmaSmemBytes, st>>>(s, qr, kr, v, a.kv_idx, a.lse, a.Dv,
-                                                                     static_cast<const T*>(a.dOs), a.tab, a.dq_acc,
-                                                                     static_cast<T*>(a.dq));
+        e = launch_sparse_bwd_dq_tc(s, qr, kr, v, a.dOs, a.kv_idx, a.lse, a.Dv, a.tab, a.dq_acc, a.dq, a.status, st);
+        if (e != cudaSuccess) return e;
     } else {
         sparse_bwd_dq_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, v, a.kv_idx, a.lse, a.Dv,
                                                                   static_cast<const T*>(a.dOs), a.tab, a.dq_acc);

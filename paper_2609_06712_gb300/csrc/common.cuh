@@ -172,8 +172,13 @@ struct BackwardArgs {
     int32_t *tr_off, *tr_list;                          // transposed mask
     void *dq, *dk, *dv;                                 // outputs, storage dtype
     float *dP_q, *dP_k, *dgate;                         // outputs, fp32 (dgate nullable)
+    DeviceStatus* status;                               // the backward workspace's status word
 };
 cudaError_t launch_backward(rola_dtype_t dt, const Shape& s, const BackwardArgs& a, cudaStream_t st);
+// The bf16 query-side sparse gradient on tcgen05: dq = dq_lr + R^T (dS K / sqrt d), bf16.
+cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
+                                    const int32_t* kv_idx, const float* lse, const float* Dv, const float2* tab,
+                                    const float* dq_lr, void* dq, DeviceStatus* status, cudaStream_t st);
 
 cudaError_t launch_gate(rola_dtype_t dt, long long rows, int D, const void* X, const void* w, float b, float* g,
                         cudaStream_t st);

@@ -1,0 +1,411 @@
+// Backward pass of the block-sparse softmax attention, query side, on the
+// 5th-generation tensor cores (bf16, fp32 accumulation in TMEM):
+//
+//   P = exp(q^r k^r / sqrt d - lse),  dP = dO^s v^T,  dS = P (dP - D),  dq^r = dS k^r / sqrt d
+//
+// over the kept key blocks of each query block (Sec. 3 softmax form, its
+// gradient).  As in the forward kernel the problem is transposed so that every
+// MMA has M = 128: for a query block (N = 64 queries) and a pair of kept key
+// blocks (M = 128 keys)
+//   S^T  = K_pair  Q^T       A = K pair (K-major),   B = Q (K-major)       TMEM
+//   dP^T = V_pair  dO^T      A = V pair (K-major),   B = dO (K-major)      TMEM
+//   dS^T = P^T (dP^T - D)    by the dS warps (thread = key), bf16 into shared memory
+//   dQ^T += K_pair^T dS^T    A = the same K pair read MN-major (M = d), B = dS^T (MN-major)
+// The log-sum-exp of each query is known, so no running maximum is needed.
+//
+// Roles (384 threads, one persistent CTA per SM):
+//   warps 0-7  dS and epilogue: two warpgroups of 32 query columns; thread
+//              wtid owns TMEM lane wtid (a key of S^T / dP^T, a d of dQ^T)
+//   warp  8    TMA: Q and dO (per query block) and the K pairs
+//   warp  9    TMA: the V pairs
+//   warp 10    S^T and dP^T issuer, TMEM owner
+//   warp 11    dQ^T issuer
+// Rings: K pairs 3 deep (held until the tile's dQ^T MMA), V pairs 2 deep,
+// S^T / dP^T / dS^T double-buffered, dQ^T double-buffered across query blocks.
+// Every mbarrier wait is bounded; a wait that gives up records ROLA_ERR_TIMEOUT
+// and the CTA drains what it issued and frees TMEM.
+#include <stddef.h>
+
+#include "common.cuh"
+#include "tcgen05.cuh"
+#include "tensor_map.cuh"
+
+namespace rola {
+namespace {
+
+using namespace tc;
+
+constexpr int kDsWarps = 8;
+constexpr int kCols = 32;                      // query columns per dS warpgroup
+constexpr int kProdKWarp = 8, kProdVWarp = 9, kSWarp = 10, kQWarp = 11;
+constexpr int kThreads = 32 * 12;
+constexpr int kWGThreads = 128;
+constexpr uint32_t kBlockBytes = 64 * 128 * 2;   // one query block (Q or dO), [chunk][row][64]
+constexpr uint32_t kPairBytes = 128 * 128 * 2;   // a pair of key blocks, [chunk][block][row]
+constexpr uint32_t kDsBytes = 128 * 64 * 2;      // dS^T tile [key][64 q]
+constexpr int KS = 3, VS = 2;
+constexpr uint32_t kSmemQ = 0, kSmemO = kBlockBytes, kSmemK = 2 * kBlockBytes;
+constexpr uint32_t kSmemV = kSmemK + KS * kPairBytes;
+constexpr uint32_t kSmemDs = kSmemV + VS * kPairBytes;
+constexpr uint32_t kSmemTiles = kSmemDs + 2 * kDsBytes;   // 224 KB
+constexpr uint32_t kTmemCols = 512;              // S^T x2, dP^T x2, dQ^T x2 (64 columns each)
+
+enum Bar { Q_FULL = 0, Q_EMPTY = 1, K_FULL = 2, K_EMPTY = K_FULL + KS, V_FULL = K_EMPTY + KS, V_EMPTY = V_FULL + VS,
+           S_FULL = V_EMPTY + VS, S_EMPTY = S_FULL + 2, DS_FULL = S_EMPTY + 2, DS_EMPTY = DS_FULL + 2,
+           O_FULL = DS_EMPTY + 2, O_EMPTY = O_FULL + 2, DRAIN = O_EMPTY + 2, NUM_BARS = DRAIN + 2 };
+
+struct Smem {
+    alignas(16) float lse2[64];     // lse of the block's queries, log2 units
+    alignas(16) float D[64];        // dO^s . O^s of the block's queries
+    uint64_t bar[NUM_BARS];
+    uint32_t tmem_base;
+    int abort;
+};
+static_assert(kSmemTiles % 1024 == 0, "the control block starts aligned");
+
+struct Params {
+    Shape s;
+    const int32_t* kv_idx;
+    const float* lse;
+    const float* Dv;
+    const float* dq_lr;                 // fp32 low-rank part of dq
+    const float2* tab;
+    __nv_bfloat16* dq;
+    DeviceStatus* status;
+    int total_items;
+    int tiles;
+};
+
+__device__ __forceinline__ void record_timeout(const Params& p, int where)
+{
+    if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = 16 + where;
+}
+
+template <int NC>
+__device__ __forceinline__ void ld_cols(uint32_t taddr, float (&v)[NC])
+{
+#pragma unroll
+    for (int c = 0; c < NC / 16; ++c) tmem_ld16(taddr + c * 16, *reinterpret_cast<float(*)[16]>(&v[c * 16]));
+    tmem_ld_wait(*reinterpret_cast<float(*)[16]>(&v[0]));
+#pragma unroll
+    for (int c = 1; c < NC / 16; ++c) reg_fence(*reinterpret_cast<float(*)[16]>(&v[c * 16]));
+}
+
+__global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap map_q,
+                                                                       const __grid_constant__ CUtensorMap map_o,
+                                                                       const __grid_constant__ CUtensorMap map_k,
+                                                                       const __grid_constant__ CUtensorMap map_v,
+                                                                       const Params p)
+{
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    if (smem_u32(smem_raw) & 1023u) {
+        if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
+        return;
+    }
+    Smem& sm = *reinterpret_cast<Smem*>(smem_raw + kSmemTiles);
+    const uint32_t sbase = smem_u32(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
+    const Shape& s = p.s;
+    const int T = p.tiles, nB = s.nB;
+
+    if (tid == 0) {
+        sm.abort = 0;
+        mbar_init(bar(Q_FULL), 1);
+        mbar_init(bar(Q_EMPTY), 1);
+        for (int i = 0; i < KS; ++i) {
+            mbar_init(bar(K_FULL + i), 1);
+            mbar_init(bar(K_EMPTY + i), 1);
+        }
+        for (int i = 0; i < VS; ++i) {
+            mbar_init(bar(V_FULL + i), 1);
+            mbar_init(bar(V_EMPTY + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(S_FULL + i), 1);
+            mbar_init(bar(S_EMPTY + i), kDsWarps);
+            mbar_init(bar(DS_FULL + i), kDsWarps);
+            mbar_init(bar(DS_EMPTY + i), 1);
+            mbar_init(bar(O_FULL + i), 1);
+            mbar_init(bar(O_EMPTY + i), kDsWarps);
+        }
+        mbar_init(bar(DRAIN), 1);
+        mbar_init(bar(DRAIN + 1), 1);
+        fence_mbar_init();
+    }
+    if (warp == kSWarp) {
+        tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    if ((warp == kProdKWarp || warp == kProdVWarp) && lane == 0) {
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_o);
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tmem = sm.tmem_base;
+    volatile int* abort = &sm.abort;
+
+    if (warp == kProdKWarp || warp == kProdVWarp) {
+        // ------------------------------------------------------------ TMA producers
+        // lane 2h + c loads d-chunk c of block h of the pair (8 KB boxes) into
+        // the [chunk][block][row] layout; the K warp also loads Q and dO.
+        const bool is_v = warp == kProdVWarp;
+        const int h = lane >> 1, kc = lane & 1;
+        const int NS = is_v ? VS : KS;
+        const uint32_t ring = is_v ? kSmemV : kSmemK;
+        const int full0 = is_v ? V_FULL : K_FULL, empty0 = is_v ? V_EMPTY : K_EMPTY;
+        const CUtensorMap* map = is_v ? &map_v : &map_k;
+        int k = 0, issued_q = 0, issued = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
+            const int bh = item / nB, qb = item - bh * nB;
+            const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
+            if (!is_v) {
+                if (k >= 1) ok = mbar_wait(bar(Q_EMPTY), (k - 1) & 1, abort, s.wait_limit_ns);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                if (lane == 0) {
+                    mbar_expect_tx(bar(Q_FULL), 2 * kBlockBytes);
+                    tma_load_4d(sbase + kSmemQ, &map_q, bar(Q_FULL), 0, qb * 64, 0, bh);
+                    tma_load_4d(sbase + kSmemO, &map_o, bar(Q_FULL), 0, qb * 64, 0, bh);
+                }
+                ++issued_q;
+            }
+            for (int t = 0; t < T; ++t) {
+                const int g = k * T + t, st = g % NS;
+                const int ja = __ldg(kept + 2 * t);
+                const int jb = 2 * t + 1 < s.n_keep ? __ldg(kept + 2 * t + 1) : -1;
+                const int nblk = jb >= 0 ? 2 : 1;
+                if (g >= NS) ok = mbar_wait(bar(empty0 + st), ((g / NS) - 1) & 1, abort, s.wait_limit_ns);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                if (lane == 0) mbar_expect_tx(bar(full0 + st), nblk * 16384u);
+                __syncwarp();
+                if (lane < 4 && h < nblk)
+                    tma_load_3d(sbase + ring + st * kPairBytes + kc * 16384 + h * 8192, map, bar(full0 + st), kc * 64,
+                                (h ? jb : ja) * 64, bh);
+                ++issued;
+            }
+        }
+        if (!ok && lane == 0) record_timeout(p, is_v ? 4 : 1);
+        if (lane == 0) {
+            int never = 0;
+            if (issued_q > 0) mbar_wait(bar(Q_FULL), (issued_q - 1) & 1, &never, s.wait_limit_ns);
+            for (int u = issued > NS ? issued - NS : 0; u < issued; ++u)
+                mbar_wait(bar(full0 + u % NS), (u / NS) & 1, &never, s.wait_limit_ns);
+        }
+    } else if (warp == kSWarp || warp == kQWarp) {
+        // ------------------------------------------------------------ MMA issuers
+        if (lane == 0) {
+            const bool qw = warp == kQWarp;
+            const uint32_t id_s = idesc_bf16(128, 64, false, false);
+            const uint32_t id_q = idesc_bf16(128, 64, true, true);
+            const uint64_t dq_ = smem_desc(sbase + kSmemQ, 16, 1024);      // Q: B of S^T (K-major)
+            const uint64_t do_ = smem_desc(sbase + kSmemO, 16, 1024);      // dO: B of dP^T (K-major)
+            const uint64_t dk = smem_desc(sbase + kSmemK, 16, 1024);       // K pairs: A of S^T (K-major)
+            const uint64_t dv = smem_desc(sbase + kSmemV, 16, 1024);       // V pairs: A of dP^T (K-major)
+            const uint64_t dkt = smem_desc(sbase + kSmemK, 16384, 1024);   // K pairs: A of dQ^T (MN-major, M = d)
+            const uint64_t dds = smem_desc(sbase + kSmemDs, 8192, 1024);   // dS^T: B of dQ^T (MN-major)
+            const uint32_t q_lo = (uint32_t)dq_, q_hi = (uint32_t)(dq_ >> 32);
+            const uint32_t o_lo = (uint32_t)do_, o_hi = (uint32_t)(do_ >> 32);
+            const uint32_t k_lo = (uint32_t)dk, k_hi = (uint32_t)(dk >> 32);
+            const uint32_t v_lo = (uint32_t)dv, v_hi = (uint32_t)(dv >> 32);
+            const uint32_t kt_lo = (uint32_t)dkt, kt_hi = (uint32_t)(dkt >> 32);
+            const uint32_t ds_lo = (uint32_t)dds, ds_hi = (uint32_t)(dds >> 32);
+            bool ok = true;
+            int k = 0;
+            for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
+                const int ob = k & 1;
+                if (!qw) {
+                    if (!(ok = mbar_wait(bar(Q_FULL), k & 1, abort, s.wait_limit_ns))) break;
+                    for (int t = 0; t < T; ++t) {
+                        const int g = k * T + t, sb = g & 1, ks = g % KS, vs = g % VS;
+                        if (!(ok = mbar_wait(bar(K_FULL + ks), (g / KS) & 1, abort, s.wait_limit_ns))) break;
+                        if (!(ok = mbar_wait(bar(V_FULL + vs), (g / VS) & 1, abort, s.wait_limit_ns))) break;
+                        if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t a = k_lo + ks * (kPairBytes >> 4), av = v_lo + vs * (kPairBytes >> 4);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t ko = (kk >> 2) * 1024 + (kk & 3) * 2, qo = (kk >> 2) * 512 + (kk & 3) * 2;
+                            mma_ss_split(tmem + sb * 64, a + ko, k_hi, q_lo + qo, q_hi, id_s, kk > 0 ? 1u : 0u);
+                        }
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t ko = (kk >> 2) * 1024 + (kk & 3) * 2, qo = (kk >> 2) * 512 + (kk & 3) * 2;
+                            mma_ss_split(tmem + 128 + sb * 64, av + ko, v_hi, o_lo + qo, o_hi, id_s, kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(bar(S_FULL + sb));
+                        mma_commit(bar(V_EMPTY + vs));
+                        if (t == T - 1) mma_commit(bar(Q_EMPTY));
+                    }
+                } else {
+                    for (int t = 0; t < T; ++t) {
+                        const int g = k * T + t, sb = g & 1, ks = g % KS;
+                        const bool half = 2 * t + 1 >= s.n_keep;
+                        if (!(ok = mbar_wait(bar(DS_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
+                        if (t == 0 && k >= 2 &&
+                            !(ok = mbar_wait(bar(O_EMPTY + ob), ((k >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t a = kt_lo + ks * (kPairBytes >> 4), b = ds_lo + sb * (kDsBytes >> 4);
+                        const uint32_t d = tmem + 256 + ob * 64;
+                        const int nk = half ? 4 : 8;          // K steps of 16 keys (a half tile has 64)
+                        for (int kk = 0; kk < nk; ++kk)
+                            mma_ss_split(d, a + kk * 128, kt_hi, b + kk * 128, ds_hi, id_q, (t > 0 || kk > 0) ? 1u : 0u);
+                        mma_commit(bar(DS_EMPTY + sb));
+                        mma_commit(bar(K_EMPTY + ks));
+                    }
+                    if (!ok) break;
+                    mma_commit(bar(O_FULL + ob));
+                }
+            }
+            if (!ok) record_timeout(p, qw ? 5 : 2);
+            int never = 0;
+            const uint32_t drain = bar(qw ? DRAIN + 1 : DRAIN);
+            mma_commit(drain);
+            mbar_wait(drain, 0, &never, s.wait_limit_ns);
+        }
+    } else {
+        // ------------------------------------------------------------ dS + epilogue
+        const int wg = warp >> 2, wtid = tid & 127;
+        const int col0 = wg * kCols;
+        const float c_log2 = s.sm_scale_log2;
+        const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
+        bool ok = true;
+        int k = 0;
+        for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
+            const int bh = item / nB, qb = item - bh * nB;
+            const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
+            const int ob = k & 1;
+            const int rows = min(64, s.N - qb * 64) - col0;     // query columns of this warpgroup inside the sequence
+            bar_sync(1 + wg, kWGThreads);                         // the previous block's columns are consumed
+            if (wtid < kCols) {
+                const int n = qb * 64 + col0 + wtid;
+                sm.lse2[col0 + wtid] = wtid < rows ? p.lse[(size_t)bh * s.N + n] * 1.4426950408889634f : 0.0f;
+                sm.D[col0 + wtid] = wtid < rows ? p.Dv[(size_t)bh * s.N + n] : 0.0f;
+            }
+            bar_sync(1 + wg, kWGThreads);
+            int ja_n = __ldg(kept);
+            int jb_n = s.n_keep > 1 ? __ldg(kept + 1) : -1;
+            for (int t = 0; t < T; ++t) {
+                const int g = k * T + t, sb = g & 1;
+                const int ja = ja_n, jb = jb_n;
+                if (t + 1 < T) {
+                    ja_n = __ldg(kept + 2 * t + 2);
+                    jb_n = 2 * t + 3 < s.n_keep ? __ldg(kept + 2 * t + 3) : -1;
+                }
+                const int blk = wtid < 64 ? ja : jb;
+                const bool valid = blk >= 0 && blk * 64 + (wtid & 63) < s.N;
+                if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
+                fence_after_sync();
+                float x[kCols], y[kCols];
+                ld_cols<kCols>(tmem + lane_off + sb * 64 + col0, x);
+                ld_cols<kCols>(tmem + lane_off + 128 + sb * 64 + col0, y);
+                fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));
+                uint32_t pk[kCols / 2];
+#pragma unroll
+                for (int q = 0; q < kCols; q += 2) {
+                    float d0 = 0.0f, d1 = 0.0f;
+                    if (valid) {
+                        const float2 l2 = *reinterpret_cast<const float2*>(&sm.lse2[col0 + q]);
+                        const float2 dd = *reinterpret_cast<const float2*>(&sm.D[col0 + q]);
+                        const float p0 = q < rows ? exp2f(fmaf(x[q], c_log2, -l2.x)) : 0.0f;
+                        const float p1 = q + 1 < rows ? exp2f(fmaf(x[q + 1], c_log2, -l2.y)) : 0.0f;
+                        d0 = p0 * (y[q] - dd.x);
+                        d1 = p1 * (y[q + 1] - dd.y);
+                    }
+                    pk[q >> 1] = pack_bf16(d0, d1);
+                }
+                if (g >= 2 && !(ok = mbar_wait(bar(DS_EMPTY + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                    break;
+                const uint32_t prow = sbase + kSmemDs + sb * kDsBytes + (wtid >> 3) * 1024 + (wtid & 7) * 128;
+#pragma unroll
+                for (int c = 0; c < kCols / 8; ++c) {
+                    const int chunk = wg * (kCols / 8) + c;
+                    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + ((chunk ^ (wtid & 7)) << 4)),
+                                 "r"(pk[4 * c]), "r"(pk[4 * c + 1]), "r"(pk[4 * c + 2]), "r"(pk[4 * c + 3])
+                                 : "memory");
+                }
+                fence_proxy_async_smem();
+                fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(DS_FULL + sb));
+            }
+            if (!ok) break;
+            // ---- epilogue: dq = low-rank rows + R(p)^T (dQ^T / sqrt d); thread wtid holds
+            // d = wtid of this warpgroup's 32 query rows; the pair partner d ^ 1 is lane ^ 1
+            if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
+            fence_after_sync();
+            float ov[kCols];
+            ld_cols<kCols>(tmem + lane_off + 256 + ob * 64 + col0, ov);
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
+            const int d = wtid, m = d >> 1;
+            const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;
+#pragma unroll
+            for (int q = 0; q < kCols; ++q) {
+                const float xv = ov[q] * 0.08838834764831845f;
+                const float other = __shfl_xor_sync(0xffffffffu, xv, 1);
+                if (q < rows) {
+                    const int n = qb * 64 + col0 + q;
+                    const float2 cs = rope_cs(p.tab, s, n, m);
+                    const float x0 = (d & 1) ? other : xv, x1 = (d & 1) ? xv : other;
+                    // R^T: (x0 c + x1 s, x1 c - x0 s)
+                    const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
+                                            : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
+                    p.dq[base + (size_t)q * kDh] = __float2bfloat16_rn(p.dq_lr[base + (size_t)q * kDh] + r);
+                }
+            }
+        }
+        if (!ok) record_timeout(p, 3);
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    if (warp == kSWarp) tmem_dealloc(tmem, kTmemCols);
+}
+
+}  // namespace
+
+cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
+                                    const int32_t* kv_idx, const float* lse, const float* Dv, const float2* tab,
+                                    const float* dq_lr, void* dq, DeviceStatus* status, cudaStream_t st)
+{
+    CUtensorMap mq, mo, mk, mv;
+    if (!make_block_map(&mq, qr, s) || !make_block_map(&mo, dOs, s) || !make_chunk_map(&mk, kr, s) ||
+        !make_chunk_map(&mv, v, s))
+        return cudaErrorInvalidValue;
+    int dev = 0, nsm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    Params p;
+    p.s = s;
+    p.kv_idx = kv_idx;
+    p.lse = lse;
+    p.Dv = Dv;
+    p.dq_lr = dq_lr;
+    p.tab = tab;
+    p.dq = static_cast<__nv_bfloat16*>(dq);
+    p.status = status;
+    p.total_items = s.B * s.H * s.nB;
+    p.tiles = (s.n_keep + 1) / 2;
+    const size_t smem = kSmemTiles + sizeof(Smem);
+    e = cudaFuncSetAttribute(sparse_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int grid = p.total_items < nsm ? p.total_items : nsm;
+    sparse_bwd_dq_tc_kernel<<<grid, kThreads, smem, st>>>(mq, mo, mk, mv, p);
+    return cudaGetLastError();
+}
+
+}  // namespace rola
