@@ -598,16 +598,11 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
 }
 
 // ---------------------------------------------------------------------------
-// bf16 key-side sparse backward on the tensor cores (mma.sync m16n8k16, fp32
-// accumulation), FlashAttention-2 style: 4 warps per CTA, each owning 16 keys
-// of the CTA's key block; tiles of 64 rows x 128 bf16 in shared memory with
-// 256-byte rows whose 16-byte chunks are XOR-swizzled by the row (sw128),
-// filled by cp.async and double-buffered over the query blocks that kept it:
-//   S^T = K Q^T, dP^T = V dO^T, dS^T = P^T (dP^T - D),  dV += P^T dO,  dK += dS^T Q
-// The epilogue adds the low-rank part (fp32 rows written by the low-rank
-// kernels), rotates dk^r back by R^T (a thread's accumulator columns 2 tig,
-// 2 tig + 1 are one RoPE pair) and stores the gradients in bf16.  The
-// query-side gradient runs on tcgen05 (sparse_bwd_tc.cu).
+// Shared helpers of the bf16 mma.sync kernels below: tiles of 64 rows x 128
+// bf16 in shared memory with 256-byte rows whose 16-byte chunks are
+// XOR-swizzled by the row (sw128), filled by cp.async; m16n8k16 fragments
+// through ldmatrix.  (The bf16 sparse gradients run on tcgen05, in
+// sparse_bwd_tc.cu.)
 
 constexpr int kMT = 128;                          // threads of the mma kernels
 constexpr uint32_t kTile = 64 * 256;              // one 64 x 128 bf16 tile
@@ -640,67 +635,6 @@ __device__ __forceinline__ uint32_t bt_addr(uint32_t t, int k0, int c0, int lane
     return t + sw128(k0 + (lane & 7) + ((lane >> 3) & 1) * 8, c0 + (lane >> 4));
 }
 
-// acc[8][4] += A(16 x 128, rows r0 of tile ta) * B^T with B the 64 rows of tile tb.
-__device__ __forceinline__ void mma_rows_x_rows(float (&acc)[8][4], uint32_t ta, int r0, uint32_t tb, int lane)
-{
-#pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4(a_addr(ta, r0, kk, lane), a0, a1, a2, a3);
-#pragma unroll
-        for (int np = 0; np < 4; ++np) {
-            uint32_t b0, b1, b2, b3;
-            ldsm_x4(bn_addr(tb, 16 * np, kk, lane), b0, b1, b2, b3);
-            mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
-            mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
-        }
-    }
-}
-
-// acc[16][4] += A(16 x 64, the C fragments w[8][4] as bf16) * (64 rows x 128 of tile tb).
-__device__ __forceinline__ void mma_frag_x_tile(float (&acc)[16][4], const float (&w)[8][4], uint32_t tb, int lane)
-{
-#pragma unroll
-    for (int ks = 0; ks < 4; ++ks) {
-        const uint32_t a0 = pack_bf16(w[2 * ks][0], w[2 * ks][1]), a1 = pack_bf16(w[2 * ks][2], w[2 * ks][3]);
-        const uint32_t a2 = pack_bf16(w[2 * ks + 1][0], w[2 * ks + 1][1]);
-        const uint32_t a3 = pack_bf16(w[2 * ks + 1][2], w[2 * ks + 1][3]);
-#pragma unroll
-        for (int np = 0; np < 8; ++np) {
-            uint32_t b0, b1, b2, b3;
-            ldsm_x4_t(bt_addr(tb, 16 * ks, 2 * np, lane), b0, b1, b2, b3);
-            mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
-            mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
-        }
-    }
-}
-
-// Final gradient rows: out = bf16(low-rank fp32 row + R^T (scale acc)) (rotate = true), or
-// out = bf16(low-rank + acc).  Accumulator rows g and g + 8 of the warp's 16, columns
-// 8 nt + 2 tig (+1).
-__device__ __forceinline__ void store_rows(const Shape& s, const float2* tab, const float (&acc)[16][4], int row0,
-                                           int lane, float scale, bool rotate, const float* lr, __nv_bfloat16* out)
-{
-    const int g = lane >> 2, tig = lane & 3;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        const int n = row0 + g + 8 * h;
-        if (n >= s.N) continue;
-#pragma unroll
-        for (int nt = 0; nt < 16; ++nt) {
-            const int d = 8 * nt + 2 * tig;
-            float x0 = acc[nt][2 * h] * scale, x1 = acc[nt][2 * h + 1] * scale;
-            if (rotate) {
-                const float2 r = rope_rotate_t(x0, x1, rope_cs(tab, s, n, d >> 1));
-                x0 = r.x;
-                x1 = r.y;
-            }
-            const float2 base = *reinterpret_cast<const float2*>(lr + (size_t)n * kDh + d);
-            *reinterpret_cast<uint32_t*>(out + (size_t)n * kDh + d) = pack_bf16(base.x + x0, base.y + x1);
-        }
-    }
-}
-
 // ---------------------------------------------------------------------------
 // bf16 low-rank backward on the tensor cores: one CTA (4 warps, 16 tokens
 // each) per (64-token chunk, head), R = r rounded up to 16 (rows r .. R-1 of
@@ -717,7 +651,8 @@ __device__ __forceinline__ uint32_t at_addr(uint32_t t, int k0, int m0, int lane
     return t + sw128(k0 + (lane & 7) + (lane >> 4) * 8, (m0 >> 3) + ((lane >> 3) & 1));
 }
 
-// C-fragment pairs (rows g, g + 8) to A fragments over k = 16 ks.. (see mma_frag_x_tile).
+// C-fragment pairs (rows g, g + 8) to A fragments over k = 16 ks .. 16 ks + 15: n-tiles 2 ks and
+// 2 ks + 1 of the C layout are the two k halves of the A layout.
 template <int NT>
 __device__ __forceinline__ void frag_a(const float (&w)[NT][4], int ks, uint32_t& a0, uint32_t& a1, uint32_t& a2,
                                        uint32_t& a3)
@@ -1111,91 +1046,6 @@ cudaError_t launch_lr_mma(const Shape& s, const BackwardArgs& a, bool key_side, 
     }
 }
 
-constexpr size_t kMmaSmemBytes = 6 * kTile + 4 * 64 * sizeof(float);
-
-__global__ void __launch_bounds__(kMT) sparse_bwd_dkdv_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ qr,
-                                                                  const __nv_bfloat16* __restrict__ kr,
-                                                                  const __nv_bfloat16* __restrict__ v,
-                                                                  const int32_t* __restrict__ off,
-                                                                  const int32_t* __restrict__ list,
-                                                                  const float* __restrict__ lse,
-                                                                  const float* __restrict__ Dv,
-                                                                  const __nv_bfloat16* __restrict__ dOs,
-                                                                  const float2* __restrict__ tab,
-                                                                  const float* __restrict__ dk_lr,
-                                                                  const float* __restrict__ dv_lr,
-                                                                  __nv_bfloat16* __restrict__ dk,
-                                                                  __nv_bfloat16* __restrict__ dv)
-{
-    extern __shared__ __align__(128) uint8_t msm[];
-    const uint32_t sK = smem_u32(msm), sV = sK + kTile, sQO = sK + 2 * kTile;     // stage st: Q, dO at sQO + 2 st kTile
-    float* s_lse = reinterpret_cast<float*>(msm + 6 * kTile);                      // [2][64]
-    float* s_D = s_lse + 128;                                                       // [2][64]
-    const int kb = blockIdx.x, bh = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = lane >> 2, tig = lane & 3;
-    const size_t head = (size_t)bh * s.N * kDh;
-    const int32_t* o = off + (size_t)bh * (s.nB + 1);
-    const int32_t* l = list + (size_t)bh * s.nB * s.n_keep;
-    const int e0 = o[kb], e1 = o[kb + 1];
-    tile_async(sK, kr + head, kb * 64, s.N);
-    tile_async(sV, v + head, kb * 64, s.N);
-    auto issue = [&](int e, int st) {
-        const int qb = l[e];
-        tile_async(sQO + st * 2 * kTile, qr + head, qb * 64, s.N);
-        tile_async(sQO + st * 2 * kTile + kTile, dOs + head, qb * 64, s.N);
-        if (threadIdx.x < 64) {
-            const int n = qb * 64 + threadIdx.x;
-            s_lse[st * 64 + threadIdx.x] = n < s.N ? lse[(size_t)bh * s.N + n] * 1.4426950408889634f : 0.0f;
-            s_D[st * 64 + threadIdx.x] = n < s.N ? Dv[(size_t)bh * s.N + n] : 0.0f;
-        }
-    };
-    if (e0 < e1) issue(e0, 0);
-    cp_async_commit();
-    const float sl2 = 0.08838834764831845f * 1.4426950408889634f;
-    float ak[16][4] = {}, av[16][4] = {};
-    const int krow = kb * 64 + 16 * warp + g;
-    const bool kv0 = krow < s.N, kv1 = krow + 8 < s.N;
-    for (int e = e0; e < e1; ++e) {
-        const int st = (e - e0) & 1;
-        if (e + 1 < e1) issue(e + 1, st ^ 1);
-        cp_async_commit();
-        cp_async_wait<1>();
-        __syncthreads();
-        const int qb = l[e];
-        const uint32_t sQ = sQO + st * 2 * kTile, sO = sQ + kTile;
-        float sc[8][4] = {}, dp[8][4] = {};
-        mma_rows_x_rows(sc, sK, 16 * warp, sQ, lane);
-        mma_rows_x_rows(dp, sV, 16 * warp, sO, lane);
-        const float* L = s_lse + st * 64;
-        const float* D = s_D + st * 64;
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            const int c = 8 * nt + 2 * tig;                   // query column of the block
-            const bool q0 = qb * 64 + c < s.N, q1 = qb * 64 + c + 1 < s.N;
-            const float p00 = kv0 && q0 ? exp2f(fmaf(sc[nt][0], sl2, -L[c])) : 0.0f;
-            const float p01 = kv0 && q1 ? exp2f(fmaf(sc[nt][1], sl2, -L[c + 1])) : 0.0f;
-            const float p10 = kv1 && q0 ? exp2f(fmaf(sc[nt][2], sl2, -L[c])) : 0.0f;
-            const float p11 = kv1 && q1 ? exp2f(fmaf(sc[nt][3], sl2, -L[c + 1])) : 0.0f;
-            sc[nt][0] = p00;
-            sc[nt][1] = p01;
-            sc[nt][2] = p10;
-            sc[nt][3] = p11;
-            dp[nt][0] = p00 * (dp[nt][0] - D[c]);
-            dp[nt][1] = p01 * (dp[nt][1] - D[c + 1]);
-            dp[nt][2] = p10 * (dp[nt][2] - D[c]);
-            dp[nt][3] = p11 * (dp[nt][3] - D[c + 1]);
-        }
-        mma_frag_x_tile(av, sc, sO, lane);
-        mma_frag_x_tile(ak, dp, sQ, lane);
-        __syncthreads();
-    }
-    cp_async_wait<0>();
-    __syncthreads();
-    const int row0 = kb * 64 + 16 * warp;
-    store_rows(s, tab, ak, row0, lane, 0.08838834764831845f, true, dk_lr + head, dk + head);
-    store_rows(s, tab, av, row0, lane, 1.0f, false, dv_lr + head, dv + head);
-}
-
 template <typename T>
 __global__ void store_grad_kernel(size_t n, const float* __restrict__ acc, T* __restrict__ out)
 {
@@ -1255,9 +1105,6 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
     }
     reduce_chunks_kernel<<<red_h, 256, 0, st>>>(s, a.partPk, a.dP_k, true);
     if constexpr (kMma) {
-        e = cudaFuncSetAttribute(sparse_bwd_dkdv_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kMmaSmemBytes);
-        if (e != cudaSuccess) return e;
         e = launch_sparse_bwd_dq_tc(s, qr, kr, v, a.dOs, a.kv_idx, a.lse, a.Dv, a.tab, a.dq_acc, a.dq, a.status, st);
         if (e != cudaSuccess) return e;
     } else {
@@ -1271,9 +1118,9 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
     }
     mask_transpose_kernel<<<s.B * s.H, 1024, tsm, st>>>(s, a.kv_idx, a.tr_off, a.tr_list);
     if constexpr (kMma) {
-        sparse_bwd_dkdv_mma_kernel<<<blocks, kMT, kMmaSmemBytes, st>>>(
-            s, qr, kr, v, a.tr_off, a.tr_list, a.lse, a.Dv, static_cast<const T*>(a.dOs), a.tab, a.dk_acc, a.dv_acc,
-            static_cast<T*>(a.dk), static_cast<T*>(a.dv));
+        e = launch_sparse_bwd_dkdv_tc(s, qr, kr, v, a.dOs, a.tr_off, a.tr_list, a.lse, a.Dv, a.tab, a.dk_acc, a.dv_acc,
+                                      a.dk, a.dv, a.status, st);
+        if (e != cudaSuccess) return e;
     } else {
         sparse_bwd_dkdv_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, v, a.tr_off, a.tr_list, a.lse, a.Dv,
                                                                     static_cast<const T*>(a.dOs), a.tab, a.dk_acc,

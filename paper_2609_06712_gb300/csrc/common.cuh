@@ -179,6 +179,12 @@ cudaError_t launch_backward(rola_dtype_t dt, const Shape& s, const BackwardArgs&
 cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
                                     const int32_t* kv_idx, const float* lse, const float* Dv, const float2* tab,
                                     const float* dq_lr, void* dq, DeviceStatus* status, cudaStream_t st);
+// The bf16 key-side sparse gradients on tcgen05 over the transposed mask (off, list):
+// dk = dk_lr + R^T (dS^T Q / sqrt d), dv = dv_lr + P^T dO^s, bf16.
+cudaError_t launch_sparse_bwd_dkdv_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
+                                      const int32_t* off, const int32_t* list, const float* lse, const float* Dv,
+                                      const float2* tab, const float* dk_lr, const float* dv_lr, void* dk, void* dv,
+                                      DeviceStatus* status, cudaStream_t st);
 
 cudaError_t launch_gate(rola_dtype_t dt, long long rows, int D, const void* X, const void* w, float b, float* g,
                         cudaStream_t st);

@@ -50,6 +50,8 @@ constexpr uint32_t kSmemDs = kSmemV + VS * kPairBytes;
 constexpr uint32_t kSmemTiles = kSmemDs + 2 * kDsBytes;   // 224 KB
 constexpr uint32_t kTmemCols = 512;              // S^T x2, dP^T x2, dQ^T x2 (64 columns each)
 
+namespace dq {
+
 enum Bar { Q_FULL = 0, Q_EMPTY = 1, K_FULL = 2, K_EMPTY = K_FULL + KS, V_FULL = K_EMPTY + KS, V_EMPTY = V_FULL + VS,
            S_FULL = V_EMPTY + VS, S_EMPTY = S_FULL + 2, DS_FULL = S_EMPTY + 2, DS_EMPTY = DS_FULL + 2,
            O_FULL = DS_EMPTY + 2, O_EMPTY = O_FULL + 2, DRAIN = O_EMPTY + 2, NUM_BARS = DRAIN + 2 };
@@ -81,6 +83,8 @@ __device__ __forceinline__ void record_timeout(const Params& p, int where)
     if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = 16 + where;
 }
 
+}  // namespace dq
+
 template <int NC>
 __device__ __forceinline__ void ld_cols(uint32_t taddr, float (&v)[NC])
 {
@@ -95,8 +99,9 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                                                                        const __grid_constant__ CUtensorMap map_o,
                                                                        const __grid_constant__ CUtensorMap map_k,
                                                                        const __grid_constant__ CUtensorMap map_v,
-                                                                       const Params p)
+                                                                       const dq::Params p)
 {
+    using namespace dq;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     if (smem_u32(smem_raw) & 1023u) {
         if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
@@ -374,6 +379,358 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
     if (warp == kSWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
+// ===========================================================================
+// Key side: dK and dV.  An item is a key block (N = 64 keys) of a head; the
+// query blocks that kept it (the transposed mask, ascending) are taken in
+// pairs (M = 128 queries):
+//   S  = Q_pair K^T        A = Q pair (K-major),   B = K block (K-major)   TMEM
+//   dP = dO_pair V^T       A = dO pair (K-major),  B = V block (K-major)   TMEM
+//   P, dS = P (dP - D)     by the dS warps (thread = query row), bf16 into shared memory
+//   dV^T += dO_pair^T P    A = the dO pair read MN-major (M = d), B = P (MN-major)
+//   dK^T += Q_pair^T dS    A = the Q pair read MN-major,          B = dS (MN-major)
+// Roles as in the query-side kernel (warp 9 idles): warp 8 loads K, V (per
+// item) and the Q / dO pairs (2-deep ring), warp 10 issues S and dP, warp 11
+// issues dV^T and dK^T.  A key block no query block kept gets its low-rank
+// rows only.
+
+namespace kv {
+
+constexpr int QS = 2;
+constexpr uint32_t kQOBytes = 2 * kPairBytes;                     // Q pair + dO pair
+constexpr uint32_t kSmK = 0, kSmV = kBlockBytes, kSmQO = 2 * kBlockBytes;
+constexpr uint32_t kSmP = kSmQO + QS * kQOBytes, kSmDs = kSmP + 2 * kDsBytes;
+constexpr uint32_t kTiles = kSmDs + 2 * kDsBytes;                 // 224 KB
+
+enum Bar { KV_FULL = 0, KV_EMPTY = 1, QO_FULL = 2, QO_EMPTY = QO_FULL + QS, S_FULL = QO_EMPTY + QS,
+           S_EMPTY = S_FULL + 2, DS_FULL = S_EMPTY + 2, DS_EMPTY = DS_FULL + 2, O_FULL = DS_EMPTY + 2,
+           O_EMPTY = O_FULL + 2, DRAIN = O_EMPTY + 2, NUM_BARS = DRAIN + 2 };
+
+struct Smem {
+    uint64_t bar[NUM_BARS];
+    uint32_t tmem_base;
+    int abort;
+};
+static_assert(kTiles % 1024 == 0, "the control block starts aligned");
+
+struct Params {
+    Shape s;
+    const int32_t* off;                 // [BH][nB + 1]
+    const int32_t* list;                // [BH][nB * n_keep]
+    const float* lse;
+    const float* Dv;
+    const float* dk_lr;
+    const float* dv_lr;
+    const float2* tab;
+    __nv_bfloat16* dk;
+    __nv_bfloat16* dv;
+    DeviceStatus* status;
+    int total_items;
+};
+
+__device__ __forceinline__ void timeout(const Params& p, int where)
+{
+    if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = 32 + where;
+}
+
+}  // namespace kv
+
+__global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap map_k,
+                                                                         const __grid_constant__ CUtensorMap map_v,
+                                                                         const __grid_constant__ CUtensorMap map_q,
+                                                                         const __grid_constant__ CUtensorMap map_o,
+                                                                         const kv::Params p)
+{
+    using namespace kv;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    if (smem_u32(smem_raw) & 1023u) {
+        if (threadIdx.x == 0) atomicCAS(&p.status->code, 0, (int)ROLA_ERR_UNSUPPORTED);
+        return;
+    }
+    kv::Smem& sm = *reinterpret_cast<kv::Smem*>(smem_raw + kTiles);
+    const uint32_t sbase = smem_u32(smem_raw);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
+    const Shape& s = p.s;
+    const int nB = s.nB;
+    // the query blocks that kept key block kb of head bh: l[e0 .. e1)
+    auto range = [&](int item, int& bh, int& kb, int& e0, int& len) {
+        bh = item / nB;
+        kb = item - bh * nB;
+        const int32_t* o = p.off + (size_t)bh * (nB + 1);
+        e0 = __ldg(o + kb);
+        len = __ldg(o + kb + 1) - e0;
+    };
+
+    if (tid == 0) {
+        sm.abort = 0;
+        mbar_init(bar(KV_FULL), 1);
+        mbar_init(bar(KV_EMPTY), 1);
+        for (int i = 0; i < QS; ++i) {
+            mbar_init(bar(QO_FULL + i), 1);
+            mbar_init(bar(QO_EMPTY + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(S_FULL + i), 1);
+            mbar_init(bar(S_EMPTY + i), kDsWarps);
+            mbar_init(bar(DS_FULL + i), kDsWarps);
+            mbar_init(bar(DS_EMPTY + i), 1);
+            mbar_init(bar(O_FULL + i), 1);
+            mbar_init(bar(O_EMPTY + i), kDsWarps);
+        }
+        mbar_init(bar(DRAIN), 1);
+        mbar_init(bar(DRAIN + 1), 1);
+        fence_mbar_init();
+    }
+    if (warp == kSWarp) {
+        tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    if (warp == kProdKWarp && lane == 0) {
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_o);
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tmem = sm.tmem_base;
+    volatile int* abort = &sm.abort;
+
+    if (warp == kProdKWarp) {
+        // ------------------------------------------------------------ TMA producer
+        // lanes 0-3: d-chunk (lane & 1) of Q block (lane >> 1) of the pair,
+        // lanes 4-7: the same of dO; the [chunk][block][row] layout.
+        const int h = (lane >> 1) & 1, kc = lane & 1;
+        const bool is_o = lane >= 4;
+        int ko = 0, g = 0, issued_kv = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x) {
+            int bh, kb, e0, len;
+            range(item, bh, kb, e0, len);
+            if (len == 0) continue;
+            if (ko >= 1) ok = mbar_wait(bar(KV_EMPTY), (ko - 1) & 1, abort, s.wait_limit_ns);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            if (lane == 0) {
+                mbar_expect_tx(bar(KV_FULL), 2 * kBlockBytes);
+                tma_load_4d(sbase + kSmK, &map_k, bar(KV_FULL), 0, kb * 64, 0, bh);
+                tma_load_4d(sbase + kSmV, &map_v, bar(KV_FULL), 0, kb * 64, 0, bh);
+            }
+            ++issued_kv;
+            const int32_t* l = p.list + (size_t)bh * nB * s.n_keep + e0;
+            const int T = (len + 1) / 2;
+            for (int t = 0; t < T && ok; ++t, ++g) {
+                const int slot = g % QS;
+                const int qa = __ldg(l + 2 * t), qb2 = 2 * t + 1 < len ? __ldg(l + 2 * t + 1) : -1;
+                const int nblk = qb2 >= 0 ? 2 : 1;
+                if (g >= QS) ok = mbar_wait(bar(QO_EMPTY + slot), ((g / QS) - 1) & 1, abort, s.wait_limit_ns);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                if (lane == 0) mbar_expect_tx(bar(QO_FULL + slot), nblk * 2 * 16384u);
+                __syncwarp();
+                if (lane < 8 && h < nblk)
+                    tma_load_3d(sbase + kSmQO + slot * kQOBytes + (is_o ? kPairBytes : 0) + kc * 16384 + h * 8192,
+                                is_o ? &map_o : &map_q, bar(QO_FULL + slot), kc * 64, (h ? qb2 : qa) * 64, bh);
+            }
+            ++ko;
+        }
+        if (!ok && lane == 0) timeout(p, 1);
+        if (lane == 0) {
+            int never = 0;
+            if (issued_kv > 0) mbar_wait(bar(KV_FULL), (issued_kv - 1) & 1, &never, s.wait_limit_ns);
+            for (int u = g > QS ? g - QS : 0; u < g; ++u)
+                mbar_wait(bar(QO_FULL + u % QS), (u / QS) & 1, &never, s.wait_limit_ns);
+        }
+    } else if (warp == kSWarp || warp == kQWarp) {
+        // ------------------------------------------------------------ MMA issuers
+        if (lane == 0) {
+            const bool gw = warp == kQWarp;
+            const uint32_t id_s = idesc_bf16(128, 64, false, false);
+            const uint32_t id_g = idesc_bf16(128, 64, true, true);
+            const uint64_t dk = smem_desc(sbase + kSmK, 16, 1024);             // K: B of S (K-major)
+            const uint64_t dvb = smem_desc(sbase + kSmV, 16, 1024);            // V: B of dP (K-major)
+            const uint64_t dqa = smem_desc(sbase + kSmQO, 16, 1024);           // Q pair: A of S (K-major)
+            const uint64_t dqm = smem_desc(sbase + kSmQO, 16384, 1024);        // Q pair: A of dK^T (MN-major)
+            const uint64_t dpb = smem_desc(sbase + kSmP, 8192, 1024);          // P: B of dV^T (MN-major)
+            const uint64_t dsb = smem_desc(sbase + kSmDs, 8192, 1024);         // dS: B of dK^T (MN-major)
+            const uint32_t k_lo = (uint32_t)dk, k_hi = (uint32_t)(dk >> 32);
+            const uint32_t v_lo = (uint32_t)dvb, v_hi = (uint32_t)(dvb >> 32);
+            const uint32_t qa_lo = (uint32_t)dqa, qa_hi = (uint32_t)(dqa >> 32);
+            const uint32_t qm_lo = (uint32_t)dqm, qm_hi = (uint32_t)(dqm >> 32);
+            const uint32_t p_lo = (uint32_t)dpb, p_hi = (uint32_t)(dpb >> 32);
+            const uint32_t ds_lo = (uint32_t)dsb, ds_hi = (uint32_t)(dsb >> 32);
+            constexpr uint32_t kO = kPairBytes >> 4;                          // dO pair after the Q pair
+            bool ok = true;
+            int ko = 0, g = 0;
+            for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x) {
+                int bh, kb, e0, len;
+                range(item, bh, kb, e0, len);
+                if (len == 0) continue;
+                const int T = (len + 1) / 2, ob = ko & 1;
+                if (!gw) {
+                    if (!(ok = mbar_wait(bar(KV_FULL), ko & 1, abort, s.wait_limit_ns))) break;
+                    for (int t = 0; t < T; ++t, ++g) {
+                        const int sb = g & 1, slot = g % QS;
+                        if (!(ok = mbar_wait(bar(QO_FULL + slot), (g / QS) & 1, abort, s.wait_limit_ns))) break;
+                        if (g >= 2 && !(ok = mbar_wait(bar(S_EMPTY + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t a = qa_lo + slot * (kQOBytes >> 4);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t ao = (kk >> 2) * 1024 + (kk & 3) * 2, bo = (kk >> 2) * 512 + (kk & 3) * 2;
+                            mma_ss_split(tmem + sb * 64, a + ao, qa_hi, k_lo + bo, k_hi, id_s, kk > 0 ? 1u : 0u);
+                        }
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t ao = (kk >> 2) * 1024 + (kk & 3) * 2, bo = (kk >> 2) * 512 + (kk & 3) * 2;
+                            mma_ss_split(tmem + 128 + sb * 64, a + kO + ao, qa_hi, v_lo + bo, v_hi, id_s,
+                                         kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(bar(S_FULL + sb));
+                        if (t == T - 1) mma_commit(bar(KV_EMPTY));
+                    }
+                } else {
+                    for (int t = 0; t < T; ++t, ++g) {
+                        const int sb = g & 1, slot = g % QS;
+                        const bool half = 2 * t + 1 >= len;
+                        if (!(ok = mbar_wait(bar(DS_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
+                        if (t == 0 && ko >= 2 &&
+                            !(ok = mbar_wait(bar(O_EMPTY + ob), ((ko >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                            break;
+                        fence_after_sync();
+                        const uint32_t aq = qm_lo + slot * (kQOBytes >> 4);
+                        const uint32_t bp = p_lo + sb * (kDsBytes >> 4), bs = ds_lo + sb * (kDsBytes >> 4);
+                        const int nk = half ? 4 : 8;          // K steps of 16 queries
+                        for (int kk = 0; kk < nk; ++kk)
+                            mma_ss_split(tmem + 256 + ob * 64, aq + kO + kk * 128, qm_hi, bp + kk * 128, p_hi, id_g,
+                                         (t > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < nk; ++kk)
+                            mma_ss_split(tmem + 384 + ob * 64, aq + kk * 128, qm_hi, bs + kk * 128, ds_hi, id_g,
+                                         (t > 0 || kk > 0) ? 1u : 0u);
+                        mma_commit(bar(DS_EMPTY + sb));
+                        mma_commit(bar(QO_EMPTY + slot));
+                    }
+                    if (!ok) break;
+                    mma_commit(bar(O_FULL + ob));
+                }
+                ++ko;
+            }
+            if (!ok) timeout(p, gw ? 5 : 2);
+            int never = 0;
+            const uint32_t drain = bar(gw ? DRAIN + 1 : DRAIN);
+            mma_commit(drain);
+            mbar_wait(drain, 0, &never, s.wait_limit_ns);
+        }
+    } else if (warp < kDsWarps) {
+        // ------------------------------------------------------------ dS + epilogue
+        // thread wtid: TMEM lane wtid = query row wtid of the pair (block wtid / 64)
+        // for S and dP, d = wtid for dV^T and dK^T; warpgroup wg: key columns
+        // [32 wg, 32 wg + 32)
+        const int wg = warp >> 2, wtid = tid & 127;
+        const int col0 = wg * kCols;
+        const float c_log2 = s.sm_scale_log2;
+        const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
+        bool ok = true;
+        int ko = 0, g = 0;
+        for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x) {
+            int bh, kb, e0, len;
+            range(item, bh, kb, e0, len);
+            const int keys = min(64, s.N - kb * 64) - col0;      // key columns of this warpgroup inside the sequence
+            const int d = wtid;
+            const size_t base = ((size_t)bh * s.N + (size_t)kb * 64 + col0) * kDh + d;
+            if (len == 0) {
+                // no query block kept this key block: the low-rank part alone
+                for (int j = 0; j < kCols; ++j)
+                    if (j < keys) {
+                        p.dk[base + (size_t)j * kDh] = __float2bfloat16_rn(p.dk_lr[base + (size_t)j * kDh]);
+                        p.dv[base + (size_t)j * kDh] = __float2bfloat16_rn(p.dv_lr[base + (size_t)j * kDh]);
+                    }
+                continue;
+            }
+            const int32_t* l = p.list + (size_t)bh * nB * s.n_keep + e0;
+            const int T = (len + 1) / 2, ob = ko & 1;
+            for (int t = 0; t < T; ++t, ++g) {
+                const int sb = g & 1;
+                const int qa = __ldg(l + 2 * t), qb2 = 2 * t + 1 < len ? __ldg(l + 2 * t + 1) : -1;
+                const int qblk = wtid < 64 ? qa : qb2;
+                const int n = qblk * 64 + (wtid & 63);
+                const bool vq = qblk >= 0 && n < s.N;
+                const float l2 = vq ? __ldg(p.lse + (size_t)bh * s.N + n) * 1.4426950408889634f : 0.0f;
+                const float Dq = vq ? __ldg(p.Dv + (size_t)bh * s.N + n) : 0.0f;
+                if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
+                fence_after_sync();
+                float x[kCols], y[kCols];
+                ld_cols<kCols>(tmem + lane_off + sb * 64 + col0, x);
+                ld_cols<kCols>(tmem + lane_off + 128 + sb * 64 + col0, y);
+                fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));
+                uint32_t pp[kCols / 2], pd[kCols / 2];
+#pragma unroll
+                for (int j = 0; j < kCols; j += 2) {
+                    const float p0 = vq && j < keys ? exp2f(fmaf(x[j], c_log2, -l2)) : 0.0f;
+                    const float p1 = vq && j + 1 < keys ? exp2f(fmaf(x[j + 1], c_log2, -l2)) : 0.0f;
+                    pp[j >> 1] = pack_bf16(p0, p1);
+                    pd[j >> 1] = pack_bf16(p0 * (y[j] - Dq), p1 * (y[j + 1] - Dq));
+                }
+                if (g >= 2 && !(ok = mbar_wait(bar(DS_EMPTY + sb), ((g >> 1) - 1) & 1, abort, s.wait_limit_ns)))
+                    break;
+                const uint32_t roff = (wtid >> 3) * 1024 + (wtid & 7) * 128;
+                const uint32_t prow = sbase + kSmP + sb * kDsBytes + roff, drow = sbase + kSmDs + sb * kDsBytes + roff;
+#pragma unroll
+                for (int c = 0; c < kCols / 8; ++c) {
+                    const uint32_t sw = ((wg * (kCols / 8) + c) ^ (wtid & 7)) << 4;
+                    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + sw), "r"(pp[4 * c]),
+                                 "r"(pp[4 * c + 1]), "r"(pp[4 * c + 2]), "r"(pp[4 * c + 3])
+                                 : "memory");
+                    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(drow + sw), "r"(pd[4 * c]),
+                                 "r"(pd[4 * c + 1]), "r"(pd[4 * c + 2]), "r"(pd[4 * c + 3])
+                                 : "memory");
+                }
+                fence_proxy_async_smem();
+                fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(DS_FULL + sb));
+            }
+            if (!ok) break;
+            // ---- epilogue: dv = low-rank + dV, dk = low-rank + R^T (dK / sqrt d); thread wtid
+            // holds d = wtid of this warpgroup's 32 keys; the pair partner d ^ 1 is lane ^ 1
+            if (!(ok = mbar_wait(bar(O_FULL + ob), (ko >> 1) & 1, abort, s.wait_limit_ns))) break;
+            fence_after_sync();
+            float av[kCols], ak[kCols];
+            ld_cols<kCols>(tmem + lane_off + 256 + ob * 64 + col0, av);
+            ld_cols<kCols>(tmem + lane_off + 384 + ob * 64 + col0, ak);
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
+            const int m = d >> 1;
+#pragma unroll
+            for (int j = 0; j < kCols; ++j) {
+                const float xk = ak[j] * 0.08838834764831845f;
+                const float other = __shfl_xor_sync(0xffffffffu, xk, 1);
+                if (j < keys) {
+                    const int nk = kb * 64 + col0 + j;
+                    const float2 cs = rope_cs(p.tab, s, nk, m);
+                    const float x0 = (d & 1) ? other : xk, x1 = (d & 1) ? xk : other;
+                    const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
+                                            : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
+                    const size_t e = base + (size_t)j * kDh;
+                    p.dk[e] = __float2bfloat16_rn(p.dk_lr[e] + r);
+                    p.dv[e] = __float2bfloat16_rn(p.dv_lr[e] + av[j]);
+                }
+            }
+            ++ko;
+        }
+        if (!ok) timeout(p, 3);
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    if (warp == kSWarp) tmem_dealloc(tmem, kTmemCols);
+}
+
 }  // namespace
 
 cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
@@ -389,7 +746,7 @@ cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* 
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    Params p;
+    dq::Params p;
     p.s = s;
     p.kv_idx = kv_idx;
     p.lse = lse;
@@ -400,11 +757,46 @@ cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* 
     p.status = status;
     p.total_items = s.B * s.H * s.nB;
     p.tiles = (s.n_keep + 1) / 2;
-    const size_t smem = kSmemTiles + sizeof(Smem);
+    const size_t smem = kSmemTiles + sizeof(dq::Smem);
     e = cudaFuncSetAttribute(sparse_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = p.total_items < nsm ? p.total_items : nsm;
     sparse_bwd_dq_tc_kernel<<<grid, kThreads, smem, st>>>(mq, mo, mk, mv, p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sparse_bwd_dkdv_tc(const Shape& s, const void* qr, const void* kr, const void* v, const void* dOs,
+                                      const int32_t* off, const int32_t* list, const float* lse, const float* Dv,
+                                      const float2* tab, const float* dk_lr, const float* dv_lr, void* dk, void* dv,
+                                      DeviceStatus* status, cudaStream_t st)
+{
+    CUtensorMap mk, mv, mq, mo;
+    if (!make_block_map(&mk, kr, s) || !make_block_map(&mv, v, s) || !make_chunk_map(&mq, qr, s) ||
+        !make_chunk_map(&mo, dOs, s))
+        return cudaErrorInvalidValue;
+    int dev = 0, nsm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    kv::Params p;
+    p.s = s;
+    p.off = off;
+    p.list = list;
+    p.lse = lse;
+    p.Dv = Dv;
+    p.dk_lr = dk_lr;
+    p.dv_lr = dv_lr;
+    p.tab = tab;
+    p.dk = static_cast<__nv_bfloat16*>(dk);
+    p.dv = static_cast<__nv_bfloat16*>(dv);
+    p.status = status;
+    p.total_items = s.B * s.H * s.nB;
+    const size_t smem = kv::kTiles + sizeof(kv::Smem);
+    e = cudaFuncSetAttribute(sparse_bwd_dkdv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int grid = p.total_items < nsm ? p.total_items : nsm;
+    sparse_bwd_dkdv_tc_kernel<<<grid, kThreads, smem, st>>>(mk, mv, mq, mo, p);
     return cudaGetLastError();
 }
 

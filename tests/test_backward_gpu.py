@@ -39,6 +39,8 @@ CASES = {
                           lowrank_act="tanh", lowrank_rope=2),
     # a rank that is not a multiple of 16 (the bf16 kernels run at 32 with zero rows of P)
     "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=76, dist="normal_gate"),
+    # one kept block of eight: half tiles on both sides, and key blocks no query block kept
+    "keep1of8": layer(T=2, Hh=16, Ww=16, H=2, r=32, keep=0.125, seed=77, dist="normal_gate"),
     # latent frames of the 480p layers: 74 blocks (the last of 8 tokens), 15 kept
     "frames_3x30x52": layer(T=3, Hh=30, Ww=52, H=2, r=32, keep=0.2, seed=75, dist="normal_gate"),
 }
