@@ -322,8 +322,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                     if (valid) {
                         const float2 l2 = *reinterpret_cast<const float2*>(&sm.lse2[col0 + q]);
                         const float2 dd = *reinterpret_cast<const float2*>(&sm.D[col0 + q]);
-                        const float p0 = q < rows ? exp2f(fmaf(x[q], c_log2, -l2.x)) : 0.0f;
-                        const float p1 = q + 1 < rows ? exp2f(fmaf(x[q + 1], c_log2, -l2.y)) : 0.0f;
+                        const float p0 = q < rows ? fast_exp2(fmaf(x[q], c_log2, -l2.x)) : 0.0f;
+                        const float p1 = q + 1 < rows ? fast_exp2(fmaf(x[q + 1], c_log2, -l2.y)) : 0.0f;
                         d0 = p0 * (y[q] - dd.x);
                         d1 = p1 * (y[q + 1] - dd.y);
                     }
@@ -346,7 +346,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             }
             if (!ok) break;
             // ---- epilogue: dq = low-rank rows + R(p)^T (dQ^T / sqrt d); thread wtid holds
-            // d = wtid of this warpgroup's 32 query rows; the pair partner d ^ 1 is lane ^ 1
+            // d = wtid of this warpgroup's 32 query rows; the pair partner d ^ 1 is lane ^ 1.
+            // The low-rank rows are read before the wait for the block's last dQ^T MMA.
+            const int d = wtid, m = d >> 1;
+            const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;
+            float lr[kCols];
+#pragma unroll
+            for (int q = 0; q < kCols; ++q) lr[q] = q < rows ? __ldg(p.dq_lr + base + (size_t)q * kDh) : 0.0f;
             if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
             float ov[kCols];
@@ -354,8 +360,6 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(O_EMPTY + ob));
-            const int d = wtid, m = d >> 1;
-            const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;
 #pragma unroll
             for (int q = 0; q < kCols; ++q) {
                 const float xv = ov[q] * 0.08838834764831845f;
@@ -367,7 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                     // R^T: (x0 c + x1 s, x1 c - x0 s)
                     const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
                                             : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
-                    p.dq[base + (size_t)q * kDh] = __float2bfloat16_rn(p.dq_lr[base + (size_t)q * kDh] + r);
+                    p.dq[base + (size_t)q * kDh] = __float2bfloat16_rn(lr[q] + r);
                 }
             }
         }
@@ -651,14 +655,25 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
             }
             const int32_t* l = p.list + (size_t)bh * nB * s.n_keep + e0;
             const int T = (len + 1) / 2, ob = ko & 1;
+            // this thread's query row of tile t: block (wtid < 64 ? l[2t] : l[2t + 1]), its lse and D,
+            // fetched one tile ahead
+            auto row_of = [&](int t, int& nq, float& l2q, float& Dqq) {
+                const int e = 2 * t + (wtid >> 6);
+                const int qblk = e < len ? __ldg(l + e) : -1;
+                nq = qblk >= 0 ? qblk * 64 + (wtid & 63) : s.N;
+                const bool v = nq < s.N;
+                l2q = v ? __ldg(p.lse + (size_t)bh * s.N + nq) * 1.4426950408889634f : 0.0f;
+                Dqq = v ? __ldg(p.Dv + (size_t)bh * s.N + nq) : 0.0f;
+            };
+            int n_nx;
+            float l2_nx, D_nx;
+            row_of(0, n_nx, l2_nx, D_nx);
             for (int t = 0; t < T; ++t, ++g) {
                 const int sb = g & 1;
-                const int qa = __ldg(l + 2 * t), qb2 = 2 * t + 1 < len ? __ldg(l + 2 * t + 1) : -1;
-                const int qblk = wtid < 64 ? qa : qb2;
-                const int n = qblk * 64 + (wtid & 63);
-                const bool vq = qblk >= 0 && n < s.N;
-                const float l2 = vq ? __ldg(p.lse + (size_t)bh * s.N + n) * 1.4426950408889634f : 0.0f;
-                const float Dq = vq ? __ldg(p.Dv + (size_t)bh * s.N + n) : 0.0f;
+                const int n = n_nx;
+                const float l2 = l2_nx, Dq = D_nx;
+                if (t + 1 < T) row_of(t + 1, n_nx, l2_nx, D_nx);
+                const bool vq = n < s.N;
                 if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
                 fence_after_sync();
                 float x[kCols], y[kCols];
@@ -670,8 +685,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
                 uint32_t pp[kCols / 2], pd[kCols / 2];
 #pragma unroll
                 for (int j = 0; j < kCols; j += 2) {
-                    const float p0 = vq && j < keys ? exp2f(fmaf(x[j], c_log2, -l2)) : 0.0f;
-                    const float p1 = vq && j + 1 < keys ? exp2f(fmaf(x[j + 1], c_log2, -l2)) : 0.0f;
+                    const float p0 = vq && j < keys ? fast_exp2(fmaf(x[j], c_log2, -l2)) : 0.0f;
+                    const float p1 = vq && j + 1 < keys ? fast_exp2(fmaf(x[j + 1], c_log2, -l2)) : 0.0f;
                     pp[j >> 1] = pack_bf16(p0, p1);
                     pd[j >> 1] = pack_bf16(p0 * (y[j] - Dq), p1 * (y[j + 1] - Dq));
                 }
@@ -696,7 +711,14 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
             }
             if (!ok) break;
             // ---- epilogue: dv = low-rank + dV, dk = low-rank + R^T (dK / sqrt d); thread wtid
-            // holds d = wtid of this warpgroup's 32 keys; the pair partner d ^ 1 is lane ^ 1
+            // holds d = wtid of this warpgroup's 32 keys; the pair partner d ^ 1 is lane ^ 1.
+            // The low-rank rows are read before the wait for the block's last MMAs.
+            float lk[kCols], lv[kCols];
+#pragma unroll
+            for (int j = 0; j < kCols; ++j) {
+                lk[j] = j < keys ? __ldg(p.dk_lr + base + (size_t)j * kDh) : 0.0f;
+                lv[j] = j < keys ? __ldg(p.dv_lr + base + (size_t)j * kDh) : 0.0f;
+            }
             if (!(ok = mbar_wait(bar(O_FULL + ob), (ko >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
             float av[kCols], ak[kCols];
@@ -717,8 +739,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
                     const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
                                             : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
                     const size_t e = base + (size_t)j * kDh;
-                    p.dk[e] = __float2bfloat16_rn(p.dk_lr[e] + r);
-                    p.dv[e] = __float2bfloat16_rn(p.dv_lr[e] + av[j]);
+                    p.dk[e] = __float2bfloat16_rn(lk[j] + r);
+                    p.dv[e] = __float2bfloat16_rn(lv[j] + av[j]);
                 }
             }
             ++ko;
