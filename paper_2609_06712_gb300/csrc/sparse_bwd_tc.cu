@@ -351,8 +351,12 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             const int d = wtid, m = d >> 1;
             const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;
             float lr[kCols];
+            float2 cs[kCols];
 #pragma unroll
-            for (int q = 0; q < kCols; ++q) lr[q] = q < rows ? __ldg(p.dq_lr + base + (size_t)q * kDh) : 0.0f;
+            for (int q = 0; q < kCols; ++q) {
+                lr[q] = q < rows ? __ldg(p.dq_lr + base + (size_t)q * kDh) : 0.0f;
+                cs[q] = rope_cs(p.tab, s, q < rows ? qb * 64 + col0 + q : 0, m);
+            }
             if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
             float ov[kCols];
@@ -365,12 +369,10 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                 const float xv = ov[q] * 0.08838834764831845f;
                 const float other = __shfl_xor_sync(0xffffffffu, xv, 1);
                 if (q < rows) {
-                    const int n = qb * 64 + col0 + q;
-                    const float2 cs = rope_cs(p.tab, s, n, m);
                     const float x0 = (d & 1) ? other : xv, x1 = (d & 1) ? xv : other;
                     // R^T: (x0 c + x1 s, x1 c - x0 s)
-                    const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
-                                            : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
+                    const float r = (d & 1) ? __fmaf_rn(x1, cs[q].x, -__fmul_rn(x0, cs[q].y))
+                                            : __fmaf_rn(x0, cs[q].x, __fmul_rn(x1, cs[q].y));
                     p.dq[base + (size_t)q * kDh] = __float2bfloat16_rn(lr[q] + r);
                 }
             }
@@ -655,24 +657,29 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
             }
             const int32_t* l = p.list + (size_t)bh * nB * s.n_keep + e0;
             const int T = (len + 1) / 2, ob = ko & 1;
-            // this thread's query row of tile t: block (wtid < 64 ? l[2t] : l[2t + 1]), its lse and D,
-            // fetched one tile ahead
-            auto row_of = [&](int t, int& nq, float& l2q, float& Dqq) {
+            // this thread's query row of tile t is in block l[2t + wtid / 64]; the block ids are
+            // fetched two tiles ahead, the row's lse and D one tile ahead
+            auto block_of = [&](int t) {
                 const int e = 2 * t + (wtid >> 6);
-                const int qblk = e < len ? __ldg(l + e) : -1;
+                return t < T && e < len ? __ldg(l + e) : -1;
+            };
+            auto row_of = [&](int qblk, int& nq, float& l2q, float& Dqq) {
                 nq = qblk >= 0 ? qblk * 64 + (wtid & 63) : s.N;
                 const bool v = nq < s.N;
                 l2q = v ? __ldg(p.lse + (size_t)bh * s.N + nq) * 1.4426950408889634f : 0.0f;
                 Dqq = v ? __ldg(p.Dv + (size_t)bh * s.N + nq) : 0.0f;
             };
-            int n_nx;
+            int n_nx, blk_nx2 = block_of(1);
             float l2_nx, D_nx;
-            row_of(0, n_nx, l2_nx, D_nx);
+            row_of(block_of(0), n_nx, l2_nx, D_nx);
             for (int t = 0; t < T; ++t, ++g) {
                 const int sb = g & 1;
                 const int n = n_nx;
                 const float l2 = l2_nx, Dq = D_nx;
-                if (t + 1 < T) row_of(t + 1, n_nx, l2_nx, D_nx);
+                if (t + 1 < T) {
+                    row_of(blk_nx2, n_nx, l2_nx, D_nx);
+                    blk_nx2 = block_of(t + 2);
+                }
                 const bool vq = n < s.N;
                 if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
                 fence_after_sync();
