@@ -37,6 +37,7 @@ CASES = {
                              lowrank_act="gelu", lowrank_rope=1),
     "tanh_none_b2": layer(T=3, Hh=6, Ww=8, B=2, H=2, r=32, keep=0.5, seed=74, dist="normal_gate",
                           lowrank_act="tanh", lowrank_rope=2),
+    "r128": layer(T=2, Hh=8, Ww=12, H=2, r=128, keep=0.3, seed=78, dist="normal_gate"),
     # a rank that is not a multiple of 16 (the bf16 kernels run at 32 with zero rows of P)
     "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=76, dist="normal_gate"),
     # one kept block of eight: half tiles on both sides, and key blocks no query block kept
