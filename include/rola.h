@@ -253,8 +253,7 @@ rola_status_t rola_forward_train(const rola_config_t* cfg, const void* q, const 
                                  int32_t* kv_idx_out, void* o_s, float* lse, float* C, void* ws,
                                  size_t ws_bytes, void* stream);
 
-/* Bytes of workspace rola_backward needs (256-byte aligned); 0 if cfg is
- * invalid or not supported by the backward pass (block_geometry CUBE). */
+/* Bytes of workspace rola_backward needs (256-byte aligned); 0 if cfg is invalid. */
 size_t rola_backward_workspace_bytes(const rola_config_t* cfg);
 
 /*
@@ -273,8 +272,8 @@ size_t rola_backward_workspace_bytes(const rola_config_t* cfg);
  *   dgate   : out, fp32 [B][N], dL/dg_p summed over the heads (for gate == NULL:
  *             the gradient at the constant sigmoid(gate_bias)), or NULL
  * Arithmetic is fp32 throughout (SIMT), accumulation of dq, dk, dv in fp32;
- * results are bitwise reproducible (fixed-order reductions).  Contiguous
- * 64-token blocks only (ROLA_BLOCK_CUBE returns ROLA_ERR_UNSUPPORTED).
+ * results are bitwise reproducible (fixed-order reductions).  Both block
+ * geometries.
  */
 rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void* k, const void* v,
                             const void* P_q, const void* P_k, const float* gate, const int32_t* kv_idx,

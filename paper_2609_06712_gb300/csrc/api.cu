@@ -209,22 +209,24 @@ rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& 
 // Backward workspace: the status word and RoPE table as in the forward
 // workspace, the rotated copies, fp32 gradient rows and partials.
 struct BwdWorkspace {
-    size_t status, table, qr, kr, qbar, kbar, dOs, Dv, dq, dk, dv, dg, partC, partPq, partPk, dC, tr_off, tr_list,
-        total;
+    size_t status, table, qr, kr, vp, qbar, kbar, dOs, Dv, dq, dk, dv, dg, partC, partPq, partPk, dC, tr_off, tr_list,
+        dOs_b, lse_b, Dv_b, total;
 };
 
 BwdWorkspace bwd_layout(const rola_config_t& c)
 {
     const Shape s = make_shape(c);
     const size_t esz = c.dtype == ROLA_BF16 ? 2 : 4;
-    const size_t bh = (size_t)c.B * c.H, rows = bh * c.N;
+    const size_t bh = (size_t)c.B * c.H, rows = bh * c.N, brows = bh * s.Np;   // token rows, block-ordered rows
     const size_t part = 4 * bh * s.nC * (size_t)c.r * kDh;
+    const size_t cube = s.cube ? 1 : 0;
     BwdWorkspace w;
     size_t off = 0;
     w.status = off; off = align_up(off + sizeof(DeviceStatus));
     w.table = off; off = align_up(off + sizeof(float2) * (size_t)(c.T + c.Hh + c.Ww) * kPairs);
-    w.qr = off; off = align_up(off + esz * rows * kDh);
-    w.kr = off; off = align_up(off + esz * rows * kDh);
+    w.qr = off; off = align_up(off + esz * brows * kDh);
+    w.kr = off; off = align_up(off + esz * brows * kDh);
+    w.vp = off; off = align_up(off + cube * esz * brows * kDh);
     w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.dOs = off; off = align_up(off + esz * rows * kDh);
@@ -239,6 +241,9 @@ BwdWorkspace bwd_layout(const rola_config_t& c)
     w.dC = off; off = align_up(off + 4 * bh * (size_t)c.r * kDh);
     w.tr_off = off; off = align_up(off + 4 * bh * (s.nB + 1));
     w.tr_list = off; off = align_up(off + 4 * bh * (size_t)s.nB * s.n_keep);
+    w.dOs_b = off; off = align_up(off + cube * esz * brows * kDh);
+    w.lse_b = off; off = align_up(off + cube * 4 * brows);
+    w.Dv_b = off; off = align_up(off + cube * 4 * brows);
     w.total = off;
     return w;
 }
@@ -450,7 +455,7 @@ rola_status_t rola_forward(const rola_config_t* cfg, const void* q, const void* 
 
 size_t rola_backward_workspace_bytes(const rola_config_t* cfg)
 {
-    if (validate(cfg) != ROLA_OK || cfg->block_geometry != ROLA_BLOCK_FLAT) return 0;
+    if (validate(cfg) != ROLA_OK) return 0;
     return bwd_layout(*cfg).total;
 }
 
@@ -460,7 +465,6 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
                             float* dP_q, float* dP_k, float* dgate, void* ws, size_t ws_bytes, void* stream)
 {
     ROLA_CHECK(validate(cfg));
-    if (cfg->block_geometry != ROLA_BLOCK_FLAT) return ROLA_ERR_UNSUPPORTED;
     const void* in[] = {q, k, v, P_q, P_k, kv_idx, o_s, lse, C, dO, dq, dk, dv, dP_q, dP_k};
     for (const void* p : in)
         if (!p || !aligned16(p)) return ROLA_ERR_INVALID_ARG;
@@ -472,8 +476,9 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
     const Shape s = make_shape(*cfg);
     ROLA_TRY(cudaMemsetAsync(at<uint8_t>(ws, w.status), 0, sizeof(DeviceStatus), st));
     ROLA_TRY(launch_rope_table(*cfg, at<float2>(ws, w.table), st));
-    ROLA_TRY(launch_rope_pool(*cfg, s, q, k, nullptr, at<float2>(ws, w.table), at<void>(ws, w.qr), at<void>(ws, w.kr),
-                              nullptr, at<float>(ws, w.qbar), at<float>(ws, w.kbar), st));
+    ROLA_TRY(launch_rope_pool(*cfg, s, q, k, s.cube ? v : nullptr, at<float2>(ws, w.table), at<void>(ws, w.qr),
+                              at<void>(ws, w.kr), s.cube ? at<void>(ws, w.vp) : nullptr, at<float>(ws, w.qbar),
+                              at<float>(ws, w.kbar), st));
     BackwardArgs a;
     a.q = q; a.k = k; a.v = v; a.P_q = P_q; a.P_k = P_k; a.o_s = o_s; a.dO = dO;
     a.C = C; a.gate = gate; a.lse = lse; a.kv_idx = kv_idx;
@@ -487,6 +492,10 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
     a.tr_off = at<int32_t>(ws, w.tr_off); a.tr_list = at<int32_t>(ws, w.tr_list);
     a.dq = dq; a.dk = dk; a.dv = dv; a.dP_q = dP_q; a.dP_k = dP_k; a.dgate = dgate;
     a.status = at<DeviceStatus>(ws, w.status);
+    a.v_blk = s.cube ? at<void>(ws, w.vp) : v;
+    a.dOs_blk = s.cube ? at<void>(ws, w.dOs_b) : nullptr;
+    a.lse_blk = s.cube ? at<float>(ws, w.lse_b) : nullptr;
+    a.Dv_blk = s.cube ? at<float>(ws, w.Dv_b) : nullptr;
     ROLA_TRY(launch_backward(cfg->dtype, s, a, st));
     return ROLA_OK;
 }

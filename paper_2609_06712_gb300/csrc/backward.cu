@@ -433,14 +433,15 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dq_kernel(Shape s, const T* __
     const SpSmem m = sp_smem(ssm);
     const int qb = blockIdx.x, bh = blockIdx.y;
     const int row = threadIdx.x >> 2, quarter = threadIdx.x & 3;
-    const size_t head = (size_t)bh * s.N * kDh;
-    const int n0 = qb * 64, n = n0 + row;
-    load_rows(m.Q, qr + head, n0, s.N);
-    load_rows(m.O, dOs + head, n0, s.N);
+    // q^r, k^r, v, dO^s, lse and D in block order (Np rows per head); dq rows by token
+    const size_t head = (size_t)bh * s.Np * kDh;
+    const int n0 = qb * 64, n = slot_token(s, qb, row);
+    load_rows(m.Q, qr + head, n0, s.Np);
+    load_rows(m.O, dOs + head, n0, s.Np);
     if (threadIdx.x < 64) {
-        const int nn = n0 + threadIdx.x;
-        m.lse[threadIdx.x] = nn < s.N ? lse[(size_t)bh * s.N + nn] : 0.0f;
-        m.D[threadIdx.x] = nn < s.N ? Dv[(size_t)bh * s.N + nn] : 0.0f;
+        const bool v = slot_token(s, qb, threadIdx.x) >= 0;
+        m.lse[threadIdx.x] = v ? lse[(size_t)bh * s.Np + n0 + threadIdx.x] : 0.0f;
+        m.D[threadIdx.x] = v ? Dv[(size_t)bh * s.Np + n0 + threadIdx.x] : 0.0f;
     }
     const float scale = 0.08838834764831845f;     // 1 / sqrt(128)
     float acc[32];
@@ -451,8 +452,8 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dq_kernel(Shape s, const T* __
         const int j = kept[it];
         if (j < 0 || j >= s.nB) continue;            // not a block id (the same for the whole CTA)
         __syncthreads();
-        load_rows(m.K, kr + head, j * 64, s.N);
-        load_rows(m.V, v + head, j * 64, s.N);
+        load_rows(m.K, kr + head, j * 64, s.Np);
+        load_rows(m.V, v + head, j * 64, s.Np);
         __syncthreads();
         for (int c = 0; c < 16; ++c) {
             const int col = quarter * 16 + c;
@@ -461,7 +462,7 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dq_kernel(Shape s, const T* __
                 sc = fmaf(m.Q[row * kLd + d], m.K[col * kLd + d], sc);
                 dp = fmaf(m.O[row * kLd + d], m.V[col * kLd + d], dp);
             }
-            const bool valid = n < s.N && j * 64 + col < s.N;
+            const bool valid = n >= 0 && slot_token(s, j, col) >= 0;
             const float p = valid ? expf(fmaf(sc, scale, -m.lse[row])) : 0.0f;
             m.S[row * 65 + col] = p * (dp - m.D[row]);
         }
@@ -475,9 +476,9 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dq_kernel(Shape s, const T* __
     }
 #pragma unroll
     for (int i = 0; i < 32; ++i) acc[i] *= scale;
-    rotate_back(s, tab, n, quarter, acc);
-    if (n < s.N) {
-        float* dst = dq_acc + head + (size_t)n * kDh;
+    rotate_back(s, tab, n >= 0 ? n : s.N, quarter, acc);
+    if (n >= 0) {
+        float* dst = dq_acc + ((size_t)bh * s.N + n) * kDh;
 #pragma unroll
         for (int i = 0; i < 32; ++i) dst[quarter + 4 * i] += acc[i];
     }
@@ -537,10 +538,11 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
     const SpSmem m = sp_smem(ssm);
     const int kb = blockIdx.x, bh = blockIdx.y;
     const int krow = threadIdx.x >> 2, quarter = threadIdx.x & 3;
-    const size_t head = (size_t)bh * s.N * kDh;
-    const int n = kb * 64 + krow;
-    load_rows(m.K, kr + head, kb * 64, s.N);
-    load_rows(m.V, v + head, kb * 64, s.N);
+    // q^r, k^r, v, dO^s, lse and D in block order (Np rows per head); dk, dv rows by token
+    const size_t head = (size_t)bh * s.Np * kDh;
+    const int n = slot_token(s, kb, krow);
+    load_rows(m.K, kr + head, kb * 64, s.Np);
+    load_rows(m.V, v + head, kb * 64, s.Np);
     const float scale = 0.08838834764831845f;
     float ak[32], av[32];
 #pragma unroll
@@ -551,12 +553,12 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
     for (int e = e0; e < e1; ++e) {
         const int qb = l[e];
         __syncthreads();
-        load_rows(m.Q, qr + head, qb * 64, s.N);
-        load_rows(m.O, dOs + head, qb * 64, s.N);
+        load_rows(m.Q, qr + head, qb * 64, s.Np);
+        load_rows(m.O, dOs + head, qb * 64, s.Np);
         if (threadIdx.x < 64) {
-            const int nn = qb * 64 + threadIdx.x;
-            m.lse[threadIdx.x] = nn < s.N ? lse[(size_t)bh * s.N + nn] : 0.0f;
-            m.D[threadIdx.x] = nn < s.N ? Dv[(size_t)bh * s.N + nn] : 0.0f;
+            const bool v = slot_token(s, qb, threadIdx.x) >= 0;
+            m.lse[threadIdx.x] = v ? lse[(size_t)bh * s.Np + qb * 64 + threadIdx.x] : 0.0f;
+            m.D[threadIdx.x] = v ? Dv[(size_t)bh * s.Np + qb * 64 + threadIdx.x] : 0.0f;
         }
         __syncthreads();
         for (int c = 0; c < 16; ++c) {
@@ -566,7 +568,7 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
                 sc = fmaf(m.Q[qc * kLd + d], m.K[krow * kLd + d], sc);
                 dp = fmaf(m.O[qc * kLd + d], m.V[krow * kLd + d], dp);
             }
-            const bool valid = n < s.N && qb * 64 + qc < s.N;
+            const bool valid = n >= 0 && slot_token(s, qb, qc) >= 0;
             const float p = valid ? expf(fmaf(sc, scale, -m.lse[qc])) : 0.0f;
             m.S[krow * 65 + qc] = p;
             m.S2[krow * 65 + qc] = p * (dp - m.D[qc]);
@@ -585,10 +587,10 @@ __global__ void __launch_bounds__(kBT) sparse_bwd_dkdv_kernel(Shape s, const T* 
     }
 #pragma unroll
     for (int i = 0; i < 32; ++i) ak[i] *= scale;
-    rotate_back(s, tab, n, quarter, ak);
-    if (n < s.N) {
-        float* dk = dk_acc + head + (size_t)n * kDh;
-        float* dv = dv_acc + head + (size_t)n * kDh;
+    rotate_back(s, tab, n >= 0 ? n : s.N, quarter, ak);
+    if (n >= 0) {
+        float* dk = dk_acc + ((size_t)bh * s.N + n) * kDh;
+        float* dv = dv_acc + ((size_t)bh * s.N + n) * kDh;
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
             dk[quarter + 4 * i] += ak[i];
@@ -1046,6 +1048,30 @@ cudaError_t launch_lr_mma(const Shape& s, const BackwardArgs& a, bool key_side, 
     }
 }
 
+// dO^s rows, lse and D from token order into block order (cube geometry):
+// row 64 b + i of the head's Np rows is slot i of block b (zeros for slots
+// outside the grid).  One CTA per (block, head).
+template <typename T>
+__global__ void __launch_bounds__(kBT) block_order_kernel(Shape s, const T* __restrict__ dOs,
+                                                          const float* __restrict__ lse, const float* __restrict__ Dv,
+                                                          T* __restrict__ dOs_b, float* __restrict__ lse_b,
+                                                          float* __restrict__ Dv_b)
+{
+    const int b = blockIdx.x, bh = blockIdx.y;
+    for (int e = threadIdx.x; e < 64 * kDh; e += kBT) {
+        const int i = e / kDh, d = e - i * kDh;
+        const int n = slot_token(s, b, i);
+        dOs_b[((size_t)bh * s.Np + (size_t)b * 64 + i) * kDh + d] =
+            n >= 0 ? dOs[((size_t)bh * s.N + n) * kDh + d] : from_f<T>(0.0f);
+    }
+    if (threadIdx.x < 64) {
+        const int n = slot_token(s, b, threadIdx.x);
+        const size_t r = (size_t)bh * s.Np + (size_t)b * 64 + threadIdx.x;
+        lse_b[r] = n >= 0 ? lse[(size_t)bh * s.N + n] : 0.0f;
+        Dv_b[r] = n >= 0 ? Dv[(size_t)bh * s.N + n] : 0.0f;
+    }
+}
+
 template <typename T>
 __global__ void store_grad_kernel(size_t n, const float* __restrict__ acc, T* __restrict__ out)
 {
@@ -1104,12 +1130,20 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
                                                      a.dv_acc, a.partPk);
     }
     reduce_chunks_kernel<<<red_h, 256, 0, st>>>(s, a.partPk, a.dP_k, true);
+    // the sparse kernels read v, dO^s, lse and D in block order (copies for cube blocks)
+    if (s.cube)
+        block_order_kernel<T><<<blocks, kBT, 0, st>>>(s, static_cast<const T*>(a.dOs), a.lse, a.Dv,
+                                                      static_cast<T*>(a.dOs_blk), a.lse_blk, a.Dv_blk);
+    const T* vb = static_cast<const T*>(s.cube ? a.v_blk : a.v);
+    const T* dOb = static_cast<const T*>(s.cube ? a.dOs_blk : a.dOs);
+    const float* lseb = s.cube ? a.lse_blk : a.lse;
+    const float* Dvb = s.cube ? a.Dv_blk : a.Dv;
     if constexpr (kMma) {
-        e = launch_sparse_bwd_dq_tc(s, qr, kr, v, a.dOs, a.kv_idx, a.lse, a.Dv, a.tab, a.dq_acc, a.dq, a.status, st);
+        e = launch_sparse_bwd_dq_tc(s, qr, kr, vb, dOb, a.kv_idx, lseb, Dvb, a.tab, a.dq_acc, a.dq, a.status, st);
         if (e != cudaSuccess) return e;
     } else {
-        sparse_bwd_dq_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, v, a.kv_idx, a.lse, a.Dv,
-                                                                  static_cast<const T*>(a.dOs), a.tab, a.dq_acc);
+        sparse_bwd_dq_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, vb, a.kv_idx, lseb, Dvb, dOb, a.tab,
+                                                                  a.dq_acc);
     }
     const size_t tsm = sizeof(int) * (size_t)s.nB;
     if (tsm > 48 * 1024) {
@@ -1118,13 +1152,12 @@ cudaError_t launch_backward_t(const Shape& s, const BackwardArgs& a, cudaStream_
     }
     mask_transpose_kernel<<<s.B * s.H, 1024, tsm, st>>>(s, a.kv_idx, a.tr_off, a.tr_list);
     if constexpr (kMma) {
-        e = launch_sparse_bwd_dkdv_tc(s, qr, kr, v, a.dOs, a.tr_off, a.tr_list, a.lse, a.Dv, a.tab, a.dk_acc, a.dv_acc,
+        e = launch_sparse_bwd_dkdv_tc(s, qr, kr, vb, dOb, a.tr_off, a.tr_list, lseb, Dvb, a.tab, a.dk_acc, a.dv_acc,
                                       a.dk, a.dv, a.status, st);
         if (e != cudaSuccess) return e;
     } else {
-        sparse_bwd_dkdv_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, v, a.tr_off, a.tr_list, a.lse, a.Dv,
-                                                                    static_cast<const T*>(a.dOs), a.tab, a.dk_acc,
-                                                                    a.dv_acc);
+        sparse_bwd_dkdv_kernel<T><<<blocks, kBT, kSpSmemBytes, st>>>(s, qr, kr, vb, a.tr_off, a.tr_list, lseb, Dvb,
+                                                                    dOb, a.tab, a.dk_acc, a.dv_acc);
         const size_t nel = (size_t)s.B * s.H * s.N * kDh;
         const int sg = 152 * 8;
         store_grad_kernel<T><<<sg, 256, 0, st>>>(nel, a.dq_acc, static_cast<T*>(a.dq));

@@ -85,6 +85,40 @@ __host__ __device__ __forceinline__ int cube_token(const Shape& s, CubeOrigin o,
     return (t < s.T && x < s.Hh && y < s.Ww) ? (t * s.Hh + x) * s.Ww + y : -1;
 }
 
+// Either geometry: the token of slot i of block b (-1 for a slot past the
+// sequence or outside the grid), and the validity of the 32 slots [c0, c0 + 32)
+// of block b as a bit mask.
+// (The template forms fix the geometry at compile time.)
+template <bool kCube>
+__device__ __forceinline__ int slot_token_g(const Shape& s, int b, int i)
+{
+    if constexpr (!kCube) return b * 64 + i < s.N ? b * 64 + i : -1;
+    else return cube_token(s, cube_origin_rcp(s, b), i);
+}
+__device__ __forceinline__ int slot_token(const Shape& s, int b, int i)
+{
+    return s.cube ? slot_token_g<true>(s, b, i) : slot_token_g<false>(s, b, i);
+}
+template <bool kCube>
+__device__ __forceinline__ uint32_t slot_mask32_g(const Shape& s, int b, int c0)
+{
+    if constexpr (!kCube) {
+        const int rem = s.N - b * 64 - c0;
+        return rem >= 32 ? 0xffffffffu : (rem <= 0 ? 0u : (1u << rem) - 1u);
+    }
+    else {
+        const CubeOrigin o = cube_origin_rcp(s, b);
+        uint32_t m = 0;
+        for (int i = 0; i < 32; ++i)
+            if (cube_token(s, o, c0 + i) >= 0) m |= 1u << i;
+        return m;
+    }
+}
+__device__ __forceinline__ uint32_t slot_mask32(const Shape& s, int b, int c0)
+{
+    return s.cube ? slot_mask32_g<true>(s, b, c0) : slot_mask32_g<false>(s, b, c0);
+}
+
 // Rotation (cos, sin) of pair m for the token at flat index n.
 __device__ __forceinline__ float2 rope_cs(const float2* __restrict__ tab, const Shape& s, int n, int m)
 {
@@ -167,6 +201,9 @@ struct BackwardArgs {
     const float2* tab;
     const void *qr, *kr;                                // rotated copies
     void* dOs;                                          // dL/dO^s, storage dtype
+    const void* v_blk;                                  // cube blocks: v, dO^s, lse, D in block order
+    void* dOs_blk;
+    float *lse_blk, *Dv_blk;
     float *Dv, *dq_acc, *dk_acc, *dv_acc, *dg_h;        // fp32 scratch
     float *partC, *partPq, *partPk, *dC;                // per-chunk partials, reduced dC
     int32_t *tr_off, *tr_list;                          // transposed mask

@@ -95,6 +95,7 @@ __device__ __forceinline__ void ld_cols(uint32_t taddr, float (&v)[NC])
     for (int c = 1; c < NC / 16; ++c) reg_fence(*reinterpret_cast<float(*)[16]>(&v[c * 16]));
 }
 
+template <bool kCube>
 __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                                                                        const __grid_constant__ CUtensorMap map_o,
                                                                        const __grid_constant__ CUtensorMap map_k,
@@ -288,12 +289,16 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             const int bh = item / nB, qb = item - bh * nB;
             const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
             const int ob = k & 1;
-            const int rows = min(64, s.N - qb * 64) - col0;     // query columns of this warpgroup inside the sequence
+            const uint32_t qmask = slot_mask32_g<kCube>(s, qb, col0);      // query columns of this warpgroup that are tokens
+            const int rows = min(64, s.N - qb * 64) - col0;                // (contiguous blocks: the first `rows` are)
+            auto colok = [&](int q) { if constexpr (kCube) return ((qmask >> q) & 1u) != 0; else return q < rows; };
             bar_sync(1 + wg, kWGThreads);                         // the previous block's columns are consumed
             if (wtid < kCols) {
-                const int n = qb * 64 + col0 + wtid;
-                sm.lse2[col0 + wtid] = wtid < rows ? p.lse[(size_t)bh * s.N + n] * 1.4426950408889634f : 0.0f;
-                sm.D[col0 + wtid] = wtid < rows ? p.Dv[(size_t)bh * s.N + n] : 0.0f;
+                // lse and D in block order: row 64 qb + slot of the head's Np rows
+                const size_t r = (size_t)bh * s.Np + (size_t)qb * 64 + col0 + wtid;
+                const bool v = (qmask >> wtid) & 1u;
+                sm.lse2[col0 + wtid] = v ? p.lse[r] * 1.4426950408889634f : 0.0f;
+                sm.D[col0 + wtid] = v ? p.Dv[r] : 0.0f;
             }
             bar_sync(1 + wg, kWGThreads);
             int ja_n = __ldg(kept);
@@ -306,7 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                     jb_n = 2 * t + 3 < s.n_keep ? __ldg(kept + 2 * t + 3) : -1;
                 }
                 const int blk = wtid < 64 ? ja : jb;
-                const bool valid = blk >= 0 && blk * 64 + (wtid & 63) < s.N;
+                const bool valid = blk >= 0 && slot_token_g<kCube>(s, blk, wtid & 63) >= 0;
                 if (!(ok = mbar_wait(bar(S_FULL + sb), (g >> 1) & 1, abort, s.wait_limit_ns))) break;
                 fence_after_sync();
                 float x[kCols], y[kCols];
@@ -322,8 +327,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                     if (valid) {
                         const float2 l2 = *reinterpret_cast<const float2*>(&sm.lse2[col0 + q]);
                         const float2 dd = *reinterpret_cast<const float2*>(&sm.D[col0 + q]);
-                        const float p0 = q < rows ? fast_exp2(fmaf(x[q], c_log2, -l2.x)) : 0.0f;
-                        const float p1 = q + 1 < rows ? fast_exp2(fmaf(x[q + 1], c_log2, -l2.y)) : 0.0f;
+                        const float p0 = colok(q) ? fast_exp2(fmaf(x[q], c_log2, -l2.x)) : 0.0f;
+                        const float p1 = colok(q + 1) ? fast_exp2(fmaf(x[q + 1], c_log2, -l2.y)) : 0.0f;
                         d0 = p0 * (y[q] - dd.x);
                         d1 = p1 * (y[q + 1] - dd.y);
                     }
@@ -349,13 +354,21 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             // d = wtid of this warpgroup's 32 query rows; the pair partner d ^ 1 is lane ^ 1.
             // The low-rank rows are read before the wait for the block's last dQ^T MMA.
             const int d = wtid, m = d >> 1;
-            const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;
+            const size_t head = (size_t)bh * s.N * kDh + d;
+            // token of column q (the block's slot col0 + q); tokens are rows of the head's N
+            auto tok = [&](int q) {
+                if constexpr (kCube) return (qmask >> q) & 1u ? slot_token_g<true>(s, qb, col0 + q) : -1;
+                else return q < rows ? qb * 64 + col0 + q : -1;
+            };
             float lr[kCols];
             float2 cs[kCols];
+            const size_t base = ((size_t)bh * s.N + (size_t)qb * 64 + col0) * kDh + d;   // contiguous blocks
 #pragma unroll
             for (int q = 0; q < kCols; ++q) {
-                lr[q] = q < rows ? __ldg(p.dq_lr + base + (size_t)q * kDh) : 0.0f;
-                cs[q] = rope_cs(p.tab, s, q < rows ? qb * 64 + col0 + q : 0, m);
+                const int n = tok(q);
+                if constexpr (kCube) lr[q] = n >= 0 ? __ldg(p.dq_lr + head + (size_t)n * kDh) : 0.0f;
+                else lr[q] = q < rows ? __ldg(p.dq_lr + base + (size_t)q * kDh) : 0.0f;
+                cs[q] = rope_cs(p.tab, s, n >= 0 ? n : 0, m);
             }
             if (!(ok = mbar_wait(bar(O_FULL + ob), (k >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
@@ -368,12 +381,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
             for (int q = 0; q < kCols; ++q) {
                 const float xv = ov[q] * 0.08838834764831845f;
                 const float other = __shfl_xor_sync(0xffffffffu, xv, 1);
-                if (q < rows) {
+                const int n = tok(q);
+                if (n >= 0) {
                     const float x0 = (d & 1) ? other : xv, x1 = (d & 1) ? xv : other;
                     // R^T: (x0 c + x1 s, x1 c - x0 s)
                     const float r = (d & 1) ? __fmaf_rn(x1, cs[q].x, -__fmul_rn(x0, cs[q].y))
                                             : __fmaf_rn(x0, cs[q].x, __fmul_rn(x1, cs[q].y));
-                    p.dq[base + (size_t)q * kDh] = __float2bfloat16_rn(lr[q] + r);
+                    p.dq[kCube ? head + (size_t)n * kDh : base + (size_t)q * kDh] = __float2bfloat16_rn(lr[q] + r);
                 }
             }
         }
@@ -440,6 +454,7 @@ __device__ __forceinline__ void timeout(const Params& p, int where)
 
 }  // namespace kv
 
+template <bool kCube>
 __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                                                                          const __grid_constant__ CUtensorMap map_v,
                                                                          const __grid_constant__ CUtensorMap map_q,
@@ -643,16 +658,24 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
         for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x) {
             int bh, kb, e0, len;
             range(item, bh, kb, e0, len);
-            const int keys = min(64, s.N - kb * 64) - col0;      // key columns of this warpgroup inside the sequence
+            const uint32_t kmask = slot_mask32_g<kCube>(s, kb, col0);      // key columns of this warpgroup that are tokens
+            const int keys = min(64, s.N - kb * 64) - col0;                // (contiguous blocks: the first `keys` are)
+            auto keyok = [&](int j) { if constexpr (kCube) return ((kmask >> j) & 1u) != 0; else return j < keys; };
             const int d = wtid;
-            const size_t base = ((size_t)bh * s.N + (size_t)kb * 64 + col0) * kDh + d;
+            const size_t head = (size_t)bh * s.N * kDh + d;
+            auto ktok = [&](int j) {
+                if constexpr (kCube) return (kmask >> j) & 1u ? slot_token_g<true>(s, kb, col0 + j) : -1;
+                else return j < keys ? kb * 64 + col0 + j : -1;
+            };
             if (len == 0) {
                 // no query block kept this key block: the low-rank part alone
-                for (int j = 0; j < kCols; ++j)
-                    if (j < keys) {
-                        p.dk[base + (size_t)j * kDh] = __float2bfloat16_rn(p.dk_lr[base + (size_t)j * kDh]);
-                        p.dv[base + (size_t)j * kDh] = __float2bfloat16_rn(p.dv_lr[base + (size_t)j * kDh]);
+                for (int j = 0; j < kCols; ++j) {
+                    const int n = ktok(j);
+                    if (n >= 0) {
+                        p.dk[head + (size_t)n * kDh] = __float2bfloat16_rn(p.dk_lr[head + (size_t)n * kDh]);
+                        p.dv[head + (size_t)n * kDh] = __float2bfloat16_rn(p.dv_lr[head + (size_t)n * kDh]);
                     }
+                }
                 continue;
             }
             const int32_t* l = p.list + (size_t)bh * nB * s.n_keep + e0;
@@ -663,11 +686,20 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
                 const int e = 2 * t + (wtid >> 6);
                 return t < T && e < len ? __ldg(l + e) : -1;
             };
+            // (lse and D in block order: row 64 qblk + slot of the head's Np rows; nq < N marks a token)
             auto row_of = [&](int qblk, int& nq, float& l2q, float& Dqq) {
-                nq = qblk >= 0 ? qblk * 64 + (wtid & 63) : s.N;
-                const bool v = nq < s.N;
-                l2q = v ? __ldg(p.lse + (size_t)bh * s.N + nq) * 1.4426950408889634f : 0.0f;
-                Dqq = v ? __ldg(p.Dv + (size_t)bh * s.N + nq) : 0.0f;
+                if constexpr (kCube) {
+                    const bool v = qblk >= 0 && slot_token_g<true>(s, qblk, wtid & 63) >= 0;
+                    nq = v ? 0 : s.N;
+                    const size_t r = (size_t)bh * s.Np + (size_t)(v ? qblk : 0) * 64 + (wtid & 63);
+                    l2q = v ? __ldg(p.lse + r) * 1.4426950408889634f : 0.0f;
+                    Dqq = v ? __ldg(p.Dv + r) : 0.0f;
+                } else {
+                    nq = qblk >= 0 ? qblk * 64 + (wtid & 63) : s.N;
+                    const bool v = nq < s.N;
+                    l2q = v ? __ldg(p.lse + (size_t)bh * s.N + nq) * 1.4426950408889634f : 0.0f;
+                    Dqq = v ? __ldg(p.Dv + (size_t)bh * s.N + nq) : 0.0f;
+                }
             };
             int n_nx, blk_nx2 = block_of(1);
             float l2_nx, D_nx;
@@ -692,8 +724,8 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
                 uint32_t pp[kCols / 2], pd[kCols / 2];
 #pragma unroll
                 for (int j = 0; j < kCols; j += 2) {
-                    const float p0 = vq && j < keys ? fast_exp2(fmaf(x[j], c_log2, -l2)) : 0.0f;
-                    const float p1 = vq && j + 1 < keys ? fast_exp2(fmaf(x[j + 1], c_log2, -l2)) : 0.0f;
+                    const float p0 = vq && keyok(j) ? fast_exp2(fmaf(x[j], c_log2, -l2)) : 0.0f;
+                    const float p1 = vq && keyok(j + 1) ? fast_exp2(fmaf(x[j + 1], c_log2, -l2)) : 0.0f;
                     pp[j >> 1] = pack_bf16(p0, p1);
                     pd[j >> 1] = pack_bf16(p0 * (y[j] - Dq), p1 * (y[j + 1] - Dq));
                 }
@@ -721,10 +753,17 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
             // holds d = wtid of this warpgroup's 32 keys; the pair partner d ^ 1 is lane ^ 1.
             // The low-rank rows are read before the wait for the block's last MMAs.
             float lk[kCols], lv[kCols];
+            const size_t base = ((size_t)bh * s.N + (size_t)kb * 64 + col0) * kDh + d;   // contiguous blocks
 #pragma unroll
             for (int j = 0; j < kCols; ++j) {
-                lk[j] = j < keys ? __ldg(p.dk_lr + base + (size_t)j * kDh) : 0.0f;
-                lv[j] = j < keys ? __ldg(p.dv_lr + base + (size_t)j * kDh) : 0.0f;
+                if constexpr (kCube) {
+                    const int n = ktok(j);
+                    lk[j] = n >= 0 ? __ldg(p.dk_lr + head + (size_t)n * kDh) : 0.0f;
+                    lv[j] = n >= 0 ? __ldg(p.dv_lr + head + (size_t)n * kDh) : 0.0f;
+                } else {
+                    lk[j] = j < keys ? __ldg(p.dk_lr + base + (size_t)j * kDh) : 0.0f;
+                    lv[j] = j < keys ? __ldg(p.dv_lr + base + (size_t)j * kDh) : 0.0f;
+                }
             }
             if (!(ok = mbar_wait(bar(O_FULL + ob), (ko >> 1) & 1, abort, s.wait_limit_ns))) break;
             fence_after_sync();
@@ -739,13 +778,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
             for (int j = 0; j < kCols; ++j) {
                 const float xk = ak[j] * 0.08838834764831845f;
                 const float other = __shfl_xor_sync(0xffffffffu, xk, 1);
-                if (j < keys) {
-                    const int nk = kb * 64 + col0 + j;
+                const int nk = ktok(j);
+                if (nk >= 0) {
                     const float2 cs = rope_cs(p.tab, s, nk, m);
                     const float x0 = (d & 1) ? other : xk, x1 = (d & 1) ? xk : other;
                     const float r = (d & 1) ? __fmaf_rn(x1, cs.x, -__fmul_rn(x0, cs.y))
                                             : __fmaf_rn(x0, cs.x, __fmul_rn(x1, cs.y));
-                    const size_t e = base + (size_t)j * kDh;
+                    const size_t e = kCube ? head + (size_t)nk * kDh : base + (size_t)j * kDh;
                     p.dk[e] = __float2bfloat16_rn(lk[j] + r);
                     p.dv[e] = __float2bfloat16_rn(lv[j] + av[j]);
                 }
@@ -766,9 +805,12 @@ cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* 
                                     const int32_t* kv_idx, const float* lse, const float* Dv, const float2* tab,
                                     const float* dq_lr, void* dq, DeviceStatus* status, cudaStream_t st)
 {
+    // the maps span the block-ordered rows (the token order itself for contiguous chunks)
+    Shape rows = s;
+    rows.N = s.Np;
     CUtensorMap mq, mo, mk, mv;
-    if (!make_block_map(&mq, qr, s) || !make_block_map(&mo, dOs, s) || !make_chunk_map(&mk, kr, s) ||
-        !make_chunk_map(&mv, v, s))
+    if (!make_block_map(&mq, qr, rows) || !make_block_map(&mo, dOs, rows) || !make_chunk_map(&mk, kr, rows) ||
+        !make_chunk_map(&mv, v, rows))
         return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -787,10 +829,11 @@ cudaError_t launch_sparse_bwd_dq_tc(const Shape& s, const void* qr, const void* 
     p.total_items = s.B * s.H * s.nB;
     p.tiles = (s.n_keep + 1) / 2;
     const size_t smem = kSmemTiles + sizeof(dq::Smem);
-    e = cudaFuncSetAttribute(sparse_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kernel = s.cube ? sparse_bwd_dq_tc_kernel<true> : sparse_bwd_dq_tc_kernel<false>;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = p.total_items < nsm ? p.total_items : nsm;
-    sparse_bwd_dq_tc_kernel<<<grid, kThreads, smem, st>>>(mq, mo, mk, mv, p);
+    kernel<<<grid, kThreads, smem, st>>>(mq, mo, mk, mv, p);
     return cudaGetLastError();
 }
 
@@ -799,9 +842,11 @@ cudaError_t launch_sparse_bwd_dkdv_tc(const Shape& s, const void* qr, const void
                                       const float2* tab, const float* dk_lr, const float* dv_lr, void* dk, void* dv,
                                       DeviceStatus* status, cudaStream_t st)
 {
+    Shape rows = s;
+    rows.N = s.Np;
     CUtensorMap mk, mv, mq, mo;
-    if (!make_block_map(&mk, kr, s) || !make_block_map(&mv, v, s) || !make_chunk_map(&mq, qr, s) ||
-        !make_chunk_map(&mo, dOs, s))
+    if (!make_block_map(&mk, kr, rows) || !make_block_map(&mv, v, rows) || !make_chunk_map(&mq, qr, rows) ||
+        !make_chunk_map(&mo, dOs, rows))
         return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -822,10 +867,11 @@ cudaError_t launch_sparse_bwd_dkdv_tc(const Shape& s, const void* qr, const void
     p.status = status;
     p.total_items = s.B * s.H * s.nB;
     const size_t smem = kv::kTiles + sizeof(kv::Smem);
-    e = cudaFuncSetAttribute(sparse_bwd_dkdv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kernel = s.cube ? sparse_bwd_dkdv_tc_kernel<true> : sparse_bwd_dkdv_tc_kernel<false>;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int grid = p.total_items < nsm ? p.total_items : nsm;
-    sparse_bwd_dkdv_tc_kernel<<<grid, kThreads, smem, st>>>(mk, mv, mq, mo, p);
+    kernel<<<grid, kThreads, smem, st>>>(mk, mv, mq, mo, p);
     return cudaGetLastError();
 }
 

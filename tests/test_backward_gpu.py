@@ -42,6 +42,9 @@ CASES = {
     "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=76, dist="normal_gate"),
     # one kept block of eight: half tiles on both sides, and key blocks no query block kept
     "keep1of8": layer(T=2, Hh=16, Ww=16, H=2, r=32, keep=0.125, seed=77, dist="normal_gate"),
+    # 4 x 4 x 4 cube blocks: ragged edge cubes, and a grid of whole cubes
+    "cube_5x9x13": layer(T=5, Hh=9, Ww=13, H=2, r=32, keep=0.3, seed=79, dist="normal_gate", block_geometry="cube"),
+    "cube_4x8x12": layer(T=4, Hh=8, Ww=12, H=2, r=16, keep=0.5, seed=80, block_geometry="cube"),
     # latent frames of the 480p layers: 74 blocks (the last of 8 tokens), 15 kept
     "frames_3x30x52": layer(T=3, Hh=30, Ww=52, H=2, r=32, keep=0.2, seed=75, dist="normal_gate"),
 }
