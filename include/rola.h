@@ -271,8 +271,9 @@ size_t rola_backward_workspace_bytes(const rola_config_t* cfg);
  *   dP_q, dP_k : out, fp32 [H][r][d_h], summed over the batch
  *   dgate   : out, fp32 [B][N], dL/dg_p summed over the heads (for gate == NULL:
  *             the gradient at the constant sigmoid(gate_bias)), or NULL
- * Arithmetic is fp32 throughout (SIMT), accumulation of dq, dk, dv in fp32;
- * results are bitwise reproducible (fixed-order reductions).  Both block
+ * bf16: tensor cores (tcgen05 for the block-sparse gradients, mma.sync for the
+ * low-rank ones) with fp32 accumulation; fp32: fp32 arithmetic throughout.
+ * Results are bitwise reproducible (fixed-order reductions).  Both block
  * geometries.
  */
 rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void* k, const void* v,

@@ -14,12 +14,14 @@
 //              dq^r = dS k^r / sqrt d,  dk^r = dS^T q^r / sqrt d,  dv += P^T dO^s
 //   RoPE       dq += R(p)^T dq^r,  dk += R(p)^T dk^r                        Sec. 3
 //
-// Arithmetic is fp32 (SIMT) for both storage types; q, k, v, O^s, dO are read
-// in the storage dtype, and the gradients of q, k, v are accumulated in fp32
-// workspace rows and converted once at the end.  Reductions over tokens (dC,
-// dP_q, dP_k) go through per-chunk partials summed in a fixed order, and the
-// key-side sparse gradients walk, for each key block, the query blocks that
-// kept it in ascending order, so results are bitwise reproducible.
+// bf16: the low-rank gradients run on mma.sync (this file) and the sparse ones
+// on tcgen05 (sparse_bwd_tc.cu), with fp32 accumulation; the fp32 validation
+// mode runs fp32 SIMT kernels throughout (this file).  The low-rank parts of
+// dq, dk, dv are fp32 workspace rows that the sparse kernels' epilogues add
+// before the single conversion to the storage type.  Reductions over tokens
+// (dC, dP_q, dP_k) go through per-chunk partials summed in a fixed order, and
+// the key-side sparse gradients walk, for each key block, the query blocks
+// that kept it in ascending order, so results are bitwise reproducible.
 #include <type_traits>
 
 #include "common.cuh"
