@@ -92,8 +92,10 @@ typedef struct {
     rola_dtype_t dtype;        /* ROLA_BF16 (default) or ROLA_FP32 */
     int32_t wait_limit_ms;     /* bound of every device-side wait (0 = 2000 ms); at most 60000 */
     int32_t debug_flags;       /* 0 normally.  ROLA_DEBUG_SKIP_FIRST_K_COPY makes each CTA of the
-                                  bf16 sparse kernel skip its first K copy, so a bounded wait runs
-                                  out and the call reports ROLA_ERR_TIMEOUT (tests the timeout path) */
+                                  bf16 sparse kernel skip its first K copy (of the bf16 backward
+                                  kernels: the first K pair, the first Q / dO pair), so a bounded
+                                  wait runs out and the call reports ROLA_ERR_TIMEOUT (tests the
+                                  timeout path) */
     int32_t lowrank_rope;      /* where the truncated RoPE sits in the low-rank features; one of
                                   rola_lowrank_rope_t, default ROLA_LOWRANK_ROPE_OUTSIDE */
     int32_t lowrank_act;       /* feature map phi of the low-rank features; one of

@@ -189,9 +189,11 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dq_tc_kernel(const __g
                 if (g >= NS) ok = mbar_wait(bar(empty0 + st), ((g / NS) - 1) & 1, abort, s.wait_limit_ns);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
-                if (lane == 0) mbar_expect_tx(bar(full0 + st), nblk * 16384u);
+                // test hook: the CTA's first K pair is never loaded, so the waits on it run out
+                const bool skip = !is_v && (s.debug_flags & ROLA_DEBUG_SKIP_FIRST_K_COPY) && g == 0;
+                if (lane == 0 && !skip) mbar_expect_tx(bar(full0 + st), nblk * 16384u);
                 __syncwarp();
-                if (lane < 4 && h < nblk)
+                if (lane < 4 && h < nblk && !skip)
                     tma_load_3d(sbase + ring + st * kPairBytes + kc * 16384 + h * 8192, map, bar(full0 + st), kc * 64,
                                 (h ? jb : ja) * 64, bh);
                 ++issued;
@@ -548,9 +550,11 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_bwd_dkdv_tc_kernel(const _
                 if (g >= QS) ok = mbar_wait(bar(QO_EMPTY + slot), ((g / QS) - 1) & 1, abort, s.wait_limit_ns);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
-                if (lane == 0) mbar_expect_tx(bar(QO_FULL + slot), nblk * 2 * 16384u);
+                // test hook: the CTA's first Q / dO pair is never loaded, so the waits on it run out
+                const bool skip = (s.debug_flags & ROLA_DEBUG_SKIP_FIRST_K_COPY) && g == 0;
+                if (lane == 0 && !skip) mbar_expect_tx(bar(QO_FULL + slot), nblk * 2 * 16384u);
                 __syncwarp();
-                if (lane < 8 && h < nblk)
+                if (lane < 8 && h < nblk && !skip)
                     tma_load_3d(sbase + kSmQO + slot * kQOBytes + (is_o ? kPairBytes : 0) + kc * 16384 + h * 8192,
                                 is_o ? &map_o : &map_q, bar(QO_FULL + slot), kc * 64, (h ? qb2 : qa) * 64, bh);
             }
