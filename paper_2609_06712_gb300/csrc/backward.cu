@@ -811,7 +811,7 @@ __device__ __forceinline__ void frag_features_bwd(const Shape& s, const float2* 
 }
 
 template <int R>
-__global__ void __launch_bounds__(kMT) lr_bwd_q_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
+__global__ void __launch_bounds__(kMT, R <= 32 ? 3 : 1) lr_bwd_q_mma_kernel(Shape s, const __nv_bfloat16* __restrict__ q,
                                                            const __nv_bfloat16* __restrict__ Pq,
                                                            const float* __restrict__ C,
                                                            const float* __restrict__ gate,
@@ -824,9 +824,10 @@ __global__ void __launch_bounds__(kMT) lr_bwd_q_mma_kernel(Shape s, const __nv_b
 {
     extern __shared__ __align__(128) uint8_t msm[];
     const uint32_t b0 = smem_u32(msm);
-    // layout: X [64] | P [R rows] | C [R rows] | F [64] | dY [64] | dU [64] (rows of 256 B)
+    // layout: X [64] | P [R rows] | C [R rows] | F [64] | dY [64] (rows of 256 B); dU takes F's place
+    // once the dC partial (F^T dY) is taken
     const uint32_t sX = b0, sP = b0 + kTile, sC = b0 + kTile + R * 256, sF = sC + R * 256, sY = sF + kTile,
-                   sU = sY + kTile;
+                   sU = sF;
     const int chunk = blockIdx.x, bh = blockIdx.y, h = bh % s.H, b = bh / s.H;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tig = lane & 3;
     const int n0 = chunk * 64, t0 = 16 * warp + g;
@@ -915,11 +916,6 @@ __global__ void __launch_bounds__(kMT) lr_bwd_q_mma_kernel(Shape s, const __nv_b
     float df[R / 8][4] = {};
     mma_dfrag_x_wt<R>(df, y, sC, lane);
     frag_features_bwd<R>(s, tab, u, df, n0, t0, tig, act);
-#pragma unroll
-    for (int nt = 0; nt < R / 8; ++nt) {
-        put_pair(msm, sU - b0, t0, 8 * nt + 2 * tig, df[nt][0], df[nt][1]);
-        put_pair(msm, sU - b0, t0 + 8, 8 * nt + 2 * tig, df[nt][2], df[nt][3]);
-    }
     // dq (low-rank part) = P_q^T du, fp32 rows
     {
         float dq[16][4] = {};
@@ -937,6 +933,13 @@ __global__ void __launch_bounds__(kMT) lr_bwd_q_mma_kernel(Shape s, const __nv_b
     __syncthreads();
     const size_t slot = ((size_t)bh * s.nC + chunk) * s.r * kDh;
     mma_outer<R>(sF, sY, s.r, partC + slot, warp, lane);
+    __syncthreads();                              // F consumed: du goes in its place
+#pragma unroll
+    for (int nt = 0; nt < R / 8; ++nt) {
+        put_pair(msm, sU - b0, t0, 8 * nt + 2 * tig, df[nt][0], df[nt][1]);
+        put_pair(msm, sU - b0, t0 + 8, 8 * nt + 2 * tig, df[nt][2], df[nt][3]);
+    }
+    __syncthreads();
     mma_outer<R>(sU, sX, s.r, partPq + slot, warp, lane);
 }
 
@@ -1008,8 +1011,9 @@ __global__ void __launch_bounds__(kMT) lr_bwd_k_mma_kernel(Shape s, const __nv_b
     mma_outer<R>(sU, sX, s.r, partPk + ((size_t)bh * s.nC + chunk) * s.r * kDh, warp, lane);
 }
 
+// three 64-row tiles and the two R-row weight tiles (both kernels)
 template <int R>
-size_t lr_mma_smem() { return 4 * (size_t)kTile + 2 * (size_t)R * 256; }
+size_t lr_mma_smem() { return 3 * (size_t)kTile + 2 * (size_t)R * 256; }
 
 template <int R>
 cudaError_t launch_lr_mma_r(const Shape& s, const BackwardArgs& a, bool key_side, cudaStream_t st)
@@ -1020,6 +1024,9 @@ cudaError_t launch_lr_mma_r(const Shape& s, const BackwardArgs& a, bool key_side
     if (!key_side) {
         cudaError_t e = cudaFuncSetAttribute(lr_bwd_q_mma_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(lr_bwd_q_mma_kernel<R>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         lr_bwd_q_mma_kernel<R><<<chunks, kMT, smem, st>>>(
             s, static_cast<const bf*>(a.q), static_cast<const bf*>(a.P_q), a.C, a.gate, static_cast<const bf*>(a.o_s),
@@ -1027,6 +1034,9 @@ cudaError_t launch_lr_mma_r(const Shape& s, const BackwardArgs& a, bool key_side
     } else {
         cudaError_t e = cudaFuncSetAttribute(lr_bwd_k_mma_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(lr_bwd_k_mma_kernel<R>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         lr_bwd_k_mma_kernel<R><<<chunks, kMT, smem, st>>>(s, static_cast<const bf*>(a.k), static_cast<const bf*>(a.v),
                                                           static_cast<const bf*>(a.P_k), a.dC, a.tab, a.dk_acc,
