@@ -68,15 +68,19 @@ def directional(O, cfg, x, mask, rope_mode, dO, name, delta, h):
     return (4 * f2 - f1) / 3, (4 * s2 - s1) / 3
 
 
-CASES = [("silu", 0), ("gelu", 1), ("tanh", 2), ("identity", 0), ("silu", 1)]
+# (feature map, RoPE placement, block geometry); the cube case has ragged edge cubes
+# (5 x 5 x 7 tokens: 2 x 2 x 2 cubes, 4 of 8 kept)
+CASES = [("silu", 0, "flat"), ("gelu", 1, "flat"), ("tanh", 2, "flat"), ("identity", 0, "flat"),
+         ("silu", 1, "flat"), ("silu", 0, "cube")]
 
 
-@pytest.mark.parametrize("act,rope_mode", CASES)
-def test_gradients_match_central_differences(oracle, act, rope_mode):
+@pytest.mark.parametrize("act,rope_mode,geometry", CASES)
+def test_gradients_match_central_differences(oracle, act, rope_mode, geometry):
     """Each gradient of L = sum(dO * O) dotted with a random direction equals the directional
     derivative of the (pinned) forward pass under the same fixed mask."""
     O = oracle
-    cfg = small_cfg(lowrank_act=act)
+    cfg = small_cfg(lowrank_act=act) if geometry == "flat" else \
+        small_cfg(lowrank_act=act, T=5, block_geometry="cube")
     x = draw(cfg)
     rng = np.random.default_rng(7)
     dO = rng.standard_normal((1, cfg["H"], cfg["N"], 128)).astype(np.float32)

@@ -57,6 +57,12 @@ MUTATIONS = {
     "bwd_silu_derivative": ("return sg * (1.0 + x * (1.0 - sg));", "return sg;"),
     "bwd_summary_value_grad": ("dv[head + (size_t)j * dh + d] += ft[aa] * dC[(size_t)aa * dh + d];",
                                "dv[head + (size_t)j * dh + d] += ft[aa] * dC[(size_t)aa * dh + (d + 1) % dh];"),
+    "bwd_inside_activation_point": ("w[a] = orc_activation_grad(c, w[a]) * df[a];",
+                                    "w[a] = orc_activation_grad(c, u[a]) * df[a];"),
+    "bwd_projection_grad_input": ("dP[(size_t)a * dh + d] += du[a] * (double)x[d];",
+                                  "dP[(size_t)a * dh + d] += du[a] * (double)x[(d + 1) % dh];"),
+    "bwd_key_grad_operand": ("dkr[(size_t)j * dh + d] += dsv * qp[d];", "dkr[(size_t)j * dh + d] += dsv * kq[d];"),
+    "bwd_gate_grad_rms": ("dg_bh[(size_t)bh * N + p] = rp * a;", "dg_bh[(size_t)bh * N + p] = a;"),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 
