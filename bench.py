@@ -294,7 +294,8 @@ def run_backward(args, cfg, c, x, stream, ws, rank):
         # dv, dk, dP_k on the key side: 11 products of 2 N d_h r flops)
         flops = 2.5 * sparse_fw + 11 * 2.0 * B * H * N * 128 * r
         if c.dtype == rola.ROLA_BF16:
-            # the sparse products run on the tensor cores (bf16 mma.sync, fp32 accumulation)
+            # the sparse gradient products run on the tcgen05 tensor cores (fp32 accumulation in TMEM),
+            # the low-rank ones on mma.sync
             peaks, src = load_peaks()
             peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
             bound, peak_src = "tensor", f"{src} bf16_tflops_sustained"

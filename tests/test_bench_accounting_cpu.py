@@ -1,0 +1,73 @@
+"""The bench's work accounting (CPU only): block sizes, the sparse FLOPs counted from
+the mask, the low-rank FLOPs and the summary's bytes.
+
+They are checked against independent counts: the oracle's block ids (numpy
+bincount), a brute-force loop over a random mask, the dense closed form
+4 B H L^2 d_h (App. D) when every block is kept, and the layer sizes of the
+Wan2.1-14B 720p layer (75600 tokens, 1182 blocks, the last of 16 tokens)."""
+import numpy as np
+import pytest
+import torch
+
+import bench
+from paper_2609_06712_gb300 import configs
+
+
+@pytest.mark.parametrize("name", ["tiny", "wan13b_480p", "wan14b_720p", "wan14b_720p_long"])
+def test_chunk_block_sizes(name):
+    cfg = configs.get(name)
+    sizes = bench.block_sizes(cfg)
+    N = cfg["N"]
+    assert len(sizes) == -(-N // 64) and sum(sizes) == N
+    assert all(s == 64 for s in sizes[:-1]) and 1 <= sizes[-1] <= 64
+
+
+def test_720p_layer_sizes():
+    sizes = bench.block_sizes(configs.get("wan14b_720p"))
+    assert len(sizes) == 1182 and sizes[-1] == 16
+
+
+@pytest.mark.parametrize("grid", [(5, 9, 13), (4, 8, 12), (1, 3, 2), (21, 45, 80)])
+def test_cube_block_sizes_match_the_oracle_block_ids(oracle, grid):
+    T, Hh, Ww = grid
+    cfg = configs.get("tiny", T=T, Hh=Hh, Ww=Ww, block_geometry="cube")
+    sizes = bench.block_sizes(cfg)
+    if T * Hh * Ww <= 20000:
+        ids = oracle.block_of(cfg)
+        assert sizes == np.bincount(ids, minlength=len(sizes)).tolist()
+    cubes = -(-T // 4) * -(-Hh // 4) * -(-Ww // 4)
+    assert len(sizes) == cubes and sum(sizes) == T * Hh * Ww and max(sizes) <= 64
+
+
+def test_sparse_flops_equal_a_brute_force_count():
+    rng = np.random.default_rng(5)
+    cfg = configs.get("tiny", T=3, Hh=7, Ww=11)             # 231 tokens: blocks of 64, 64, 64, 39
+    sizes = bench.block_sizes(cfg)
+    nB, n_keep, B, H = len(sizes), 2, 2, 3
+    kv = np.stack([np.sort(rng.choice(nB, n_keep, replace=False)) for _ in range(B * H * nB)])
+    kv = kv.reshape(B, H, nB, n_keep).astype(np.int32)
+    want = 0
+    for b in range(B):
+        for h in range(H):
+            for i in range(nB):
+                for j in kv[b, h, i]:
+                    want += 4 * 128 * sizes[i] * sizes[j]     # QK^T and PV, 2 flops per multiply-add
+    assert bench.sparse_flops_from_mask(torch.from_numpy(kv), sizes) == float(want)
+
+
+def test_every_block_kept_is_the_dense_closed_form():
+    cfg = configs.get("wan14b_720p")
+    sizes = bench.block_sizes(cfg)
+    nB, H = len(sizes), cfg["H"]
+    kv = torch.arange(nB, dtype=torch.int32).expand(1, H, nB, nB)
+    dense = 4.0 * 1 * H * cfg["N"] ** 2 * 128
+    assert bench.sparse_flops_from_mask(kv, sizes) == dense
+    assert dense == pytest.approx(117.05e12, rel=1e-4)
+
+
+def test_lowrank_flops_and_summary_bytes_at_720p():
+    B, H, N, r = 1, 40, 75600, 32
+    # App. D: 8 B H L d_h r; half of it is the summary, half the readout (~49.5 GFLOP each)
+    assert bench.lowrank_flops(B, H, N, 128, r) == pytest.approx(2 * 49.54e9, rel=1e-3)
+    # the summary reads k and v once in bf16: 2 B H N d_h 2 bytes
+    assert bench.summary_bytes(B, H, N, 128) == pytest.approx(1.548e9, rel=1e-3)
