@@ -32,6 +32,9 @@ MUTATIONS = {
     "pool_unrotated": ("mean[(size_t)blk * dh + d] += xr[d];", "mean[(size_t)blk * dh + d] += xi[d];"),
     "softmax_scale": ("double isd = 1.0 / sqrt((double)dh);\n    int ntask",
                       "double isd = 1.0;\n    int ntask"),
+    "ragged_keys_padded": ("for (int t = 0; t < nkeys; ++t) { s[t] = exp(s[t] - mx); den += s[t]; }",
+                           "for (int t = 0; t < nkeys; ++t) { s[t] = exp(s[t] - mx); den += s[t]; } "
+                           "den += (double)((64 - nkeys % 64) % 64) * exp(-mx);"),
     "cube_axis_stride": ("return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;",
                          "return ((t / CUBE) * ny + x / CUBE) * nx + y / CUBE;"),
     "cube_grid_rounding": ("int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;",
