@@ -71,3 +71,23 @@ def test_lowrank_flops_and_summary_bytes_at_720p():
     assert bench.lowrank_flops(B, H, N, 128, r) == pytest.approx(2 * 49.54e9, rel=1e-3)
     # the summary reads k and v once in bf16: 2 B H N d_h 2 bytes
     assert bench.summary_bytes(B, H, N, 128) == pytest.approx(1.548e9, rel=1e-3)
+
+
+def test_accounting_uses_the_printed_complexity_formulas():
+    """App. D's coefficients (tests/golden/paper_constants.json): C_sparse = 4 B H L^2 (1-S) d_h,
+    C_lowrank = 8 B H L d_h r, and with C_fusion = 2 B H L d_h the overhead
+    eta = (C_lowrank + C_fusion) / C_sparse = (2r + 0.5) / (L (1 - S))."""
+    import json
+    import os
+    gold = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "paper_constants.json")))["flops"]
+    B, H, L, d, r = 1, 40, 75600, 128, 32
+    assert bench.lowrank_flops(B, H, L, d, r) == gold["lowrank_coeff"] * B * H * L * d * r
+    sizes = bench.block_sizes(configs.get("wan14b_720p"))
+    nB = len(sizes)
+    kv = torch.arange(nB, dtype=torch.int32).expand(B, H, nB, nB)
+    assert bench.sparse_flops_from_mask(kv, sizes) == gold["sparse_coeff"] * B * H * L ** 2 * d
+    for keep in (0.05, 0.1, 0.2):
+        S = 1.0 - keep
+        c_sparse = gold["sparse_coeff"] * B * H * L ** 2 * (1 - S) * d
+        eta = (bench.lowrank_flops(B, H, L, d, r) + gold["fusion_coeff"] * B * H * L * d) / c_sparse
+        assert eta == pytest.approx((gold["eta_r_coeff"] * r + gold["eta_const"]) / (L * (1 - S)), rel=1e-12)
