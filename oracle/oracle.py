@@ -49,6 +49,7 @@ class OracleConfig(ctypes.Structure):
         ("rope_mode", ctypes.c_int32),
         ("act", ctypes.c_int32),
         ("geometry", ctypes.c_int32),
+        ("qblock", ctypes.c_int32),
     ]
 
 
@@ -71,6 +72,8 @@ def _get():
             lib.orc_num_blocks.argtypes = [cfgp]
             lib.orc_num_keep.argtypes = [cfgp]
             lib.orc_block_of.argtypes = [cfgp, ctypes.c_int]
+            lib.orc_num_qblocks.argtypes = [cfgp]
+            lib.orc_qblock_of.argtypes = [cfgp, ctypes.c_int]
             lib.orc_position.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.argtypes = [cfgp, ctypes.c_int, P]
             lib.orc_pair_angle.restype = ctypes.c_double
@@ -112,6 +115,10 @@ def make_config(cfg: dict, rope_mode: int = ROPE_OUTSIDE) -> OracleConfig:
     c.rope_mode = rope_mode
     c.act = ACTIVATIONS[cfg.get("lowrank_act", "silu")]
     c.geometry = GEOMETRIES[cfg.get("block_geometry", "flat")]
+    # query-block size of the contiguous geometry (0: the key blocks' size)
+    c.qblock = int(cfg.get("qblock", 0))
+    if c.qblock < 0 or (c.qblock and c.geometry != GEOMETRIES["flat"]):
+        raise ValueError("qblock is a size of contiguous query blocks (flat geometry only)")
     return c
 
 
@@ -166,6 +173,19 @@ def num_blocks(cfg: dict) -> int:
 def num_keep(cfg: dict) -> int:
     c = make_config(cfg)
     return _get().orc_num_keep(ctypes.byref(c))
+
+
+def num_qblocks(cfg: dict) -> int:
+    """Query blocks: chunks of cfg["qblock"] tokens if set, else the key blocks."""
+    c = make_config(cfg)
+    return _get().orc_num_qblocks(ctypes.byref(c))
+
+
+def qblock_of(cfg: dict) -> np.ndarray:
+    """Query-block id of every token [N]."""
+    c = make_config(cfg)
+    lib = _get()
+    return np.array([lib.orc_qblock_of(ctypes.byref(c), n) for n in range(c.N)], dtype=np.int64)
 
 
 def block_of(cfg: dict) -> np.ndarray:
@@ -224,7 +244,7 @@ def lowrank_summary(cfg: dict, k, v, Pk, rope_mode: int = ROPE_OUTSIDE):
 def _sel(cfg: dict, qblocks):
     if qblocks is None:
         return None
-    sel = np.zeros(num_blocks(cfg), dtype=np.uint8)
+    sel = np.zeros(num_qblocks(cfg), dtype=np.uint8)
     sel[np.asarray(qblocks, dtype=np.int64)] = 1
     return sel
 
@@ -297,11 +317,11 @@ def block_mask(cfg: dict, q, k):
     c = make_config(cfg)
     q, qp = _f32(q)
     k, kp = _f32(k)
-    nb, nk = num_blocks(cfg), num_keep(cfg)
-    idx = np.empty((c.B, c.H, nb, nk), dtype=np.int32)
-    scores = np.empty((c.B, c.H, nb, nb))
-    gap = np.empty((c.B, c.H, nb))
-    tau = np.empty((c.B, c.H, nb))
+    nb, nq, nk = num_blocks(cfg), num_qblocks(cfg), num_keep(cfg)
+    idx = np.empty((c.B, c.H, nq, nk), dtype=np.int32)
+    scores = np.empty((c.B, c.H, nq, nb))
+    gap = np.empty((c.B, c.H, nq))
+    tau = np.empty((c.B, c.H, nq))
     _get().orc_block_mask(ctypes.byref(c), qp, kp, idx.ctypes.data, scores.ctypes.data,
                           gap.ctypes.data, tau.ctypes.data)
     return idx, scores, gap, tau
@@ -335,18 +355,18 @@ def forward(cfg: dict, q, k, v, Pq, Pk, gate=None, mask_override=None, qblocks=N
     Pq, Pqp = _f32(Pq)
     Pk, Pkp = _f32(Pk)
     g = None if gate is None else np.ascontiguousarray(gate, dtype=np.float32)
-    nb, nk = num_blocks(cfg), num_keep(cfg)
+    nq, nk = num_qblocks(cfg), num_keep(cfg)
     mo = None if mask_override is None else np.ascontiguousarray(mask_override, dtype=np.int32)
     sel = _sel(cfg, qblocks)
     shape = (c.B, c.H, c.N, c.dh)
     o = np.full(shape, np.nan)
-    idx = np.empty((c.B, c.H, nb, nk), dtype=np.int32)
+    idx = np.empty((c.B, c.H, nq, nk), dtype=np.int32)
     o_s = np.empty(shape)
     C = np.empty((c.B, c.H, c.r, c.dh))
     z = np.empty((c.B, c.H, c.r))
     _get().orc_forward(ctypes.byref(c), qp, kp, vp, Pqp, Pkp, _ptr(g), _ptr(mo), _ptr(sel),
                        o.ctypes.data, idx.ctypes.data, o_s.ctypes.data, C.ctypes.data, z.ctypes.data)
     if sel is not None:
-        rows = sel.astype(bool)[block_of(cfg)]
+        rows = sel.astype(bool)[qblock_of(cfg)]
         o_s[:, :, ~rows, :] = np.nan
     return dict(o=o, kv_idx=idx, o_s=o_s, C=C, z=z)

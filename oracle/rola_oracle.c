@@ -29,6 +29,11 @@
  *                    1, the tiling of the sparse video attentions the paper
  *                    builds on), numbered t-major over the cube grid; edge
  *                    cubes hold the tokens that fall inside the grid.
+ *                    Geometry 0 may also give the query side longer chunks
+ *                    (qblock, e.g. 128 queries against 64-token key blocks,
+ *                    the b_q / b_kv tiling of those attentions): each query
+ *                    block is pooled, scored and given its n_keep key blocks
+ *                    as one unit.
  *   sparse branch    Sec. 3 (softmax(QK^T / sqrt d_h) V) restricted to the
  *                    kept key blocks; Alg. 1 sparse-branch steps.
  *   low-rank branch  Eq. (qklr): q~ = R_r(p) SiLU(P_q q^n), k~ = R_r(q)
@@ -44,7 +49,8 @@
  *
  * Layouts: q, k, v, o: [B][H][N][d_h]; P_q, P_k: [H][r][d_h];
  * C: [B][H][r][d_h]; z: [B][H][r]; gate: [B][N] (NULL -> sigmoid(gate_bias));
- * kv_idx: [B][H][nQB][n_keep] ascending.
+ * kv_idx: [B][H][nQB][n_keep] ascending, nQB the query blocks (the key
+ * blocks unless qblock is set).
  */
 #include <math.h>
 #include <stdint.h>
@@ -65,6 +71,8 @@ typedef struct {
     int32_t rope_mode;    /* 0: RoPE outside SiLU (RoLA), 1: inside, 2: none */
     int32_t act;          /* 0: SiLU, 1: identity, 2: tanh, 3: ReLU, 4: GELU */
     int32_t geometry;     /* 0: contiguous chunks of `block` tokens, 1: 4x4x4 cubes */
+    int32_t qblock;       /* geometry 0: tokens per query block (0: `block`); the key
+                             blocks keep `block` tokens.  Ignored by geometry 1. */
 } orc_cfg;
 
 enum { CUBE = 4 };        /* cube edge of geometry 1 (CUBE^3 == block == 64) */
@@ -88,6 +96,40 @@ int orc_block_of(const orc_cfg* c, int n)
     int t = n / (c->Hh * c->Ww), x = (n / c->Ww) % c->Hh, y = n % c->Ww;
     int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;
     return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;
+}
+
+/* Query blocks.  The block-sparse video attentions the paper builds on
+ * tile the query side more coarsely than the key side (b_q = 128 queries
+ * against b_kv = 64 keys); with qblock set, the query blocks of geometry 0
+ * are contiguous chunks of qblock tokens: pooled, scored and given their
+ * n_keep key blocks as one unit.  Otherwise they are the key blocks. */
+static int qblock_size(const orc_cfg* c)
+{
+    return (c->geometry != 1 && c->qblock > 0) ? c->qblock : c->block;
+}
+
+int orc_num_qblocks(const orc_cfg* c)
+{
+    if (c->geometry == 1) return orc_num_blocks(c);
+    int qb = qblock_size(c);
+    return (c->N + qb - 1) / qb;
+}
+
+int orc_qblock_of(const orc_cfg* c, int n)
+{
+    if (c->geometry == 1) return orc_block_of(c, n);
+    return n / qblock_size(c);
+}
+
+/* Members of every query block, ascending: list[b * qblock_size + i], i < cnt[b]. */
+static void qblock_members(const orc_cfg* c, int* list, int* cnt)
+{
+    int nQ = orc_num_qblocks(c), qb = qblock_size(c);
+    for (int b = 0; b < nQ; ++b) cnt[b] = 0;
+    for (int n = 0; n < c->N; ++n) {
+        int b = orc_qblock_of(c, n);
+        list[(size_t)b * qb + cnt[b]++] = n;
+    }
 }
 
 /* Members of every block in ascending token order: list[b * block + i] for
@@ -325,7 +367,7 @@ static void fuse(const orc_cfg* c, const double* os, const double* olr, double g
 /* Token list helper: the tokens of the selected query blocks (all if NULL). */
 static int token_in_selection(const orc_cfg* c, int n, const uint8_t* qb_sel)
 {
-    return qb_sel == NULL || qb_sel[orc_block_of(c, n)];
+    return qb_sel == NULL || qb_sel[orc_qblock_of(c, n)];
 }
 
 /* O = fusion(O^s, RMSNorm(q~^T C)) for the tokens of the selected query
@@ -460,18 +502,23 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
 {
     int BH = c->B * c->H, dh = c->dh, N = c->N, bs = c->block;
     int nB = orc_num_blocks(c), nk = orc_num_keep(c);
+    int nQ = orc_num_qblocks(c), qbs = qblock_size(c);
+    int pool = qbs > bs ? qbs : bs;                         /* most tokens a pooled mean sums */
     double isd = 1.0 / sqrt((double)dh);
     const double u = ldexp(1.0, -24);
     double* tcs = token_cs(c);
     int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
     int* count = (int*)malloc(sizeof(int) * (size_t)nB);
+    int* qmembers = (int*)malloc(sizeof(int) * (size_t)nQ * qbs);
+    int* qcount = (int*)malloc(sizeof(int) * (size_t)nQ);
     block_members(c, members, count);
+    qblock_members(c, qmembers, qcount);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int bh = 0; bh < BH; ++bh) {
-        size_t nbd = (size_t)nB * dh;
-        double* qb = (double*)calloc(nbd, sizeof(double));   /* pooled means */
+        size_t nbd = (size_t)nB * dh, nqd = (size_t)nQ * dh;
+        double* qb = (double*)calloc(nqd, sizeof(double));   /* pooled means */
         double* kb = (double*)calloc(nbd, sizeof(double));
-        double* qa = (double*)calloc(nbd, sizeof(double));   /* pooled |pair| magnitudes */
+        double* qa = (double*)calloc(nqd, sizeof(double));   /* pooled |pair| magnitudes */
         double* ka = (double*)calloc(nbd, sizeof(double));
         double* xr = (double*)malloc(sizeof(double) * (size_t)dh);
         double* xi = (double*)malloc(sizeof(double) * (size_t)dh);
@@ -480,25 +527,27 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
             const float* x = which == 0 ? q : k;
             double* mean = which == 0 ? qb : kb;
             double* mag = which == 0 ? qa : ka;
+            const int nblk = which == 0 ? nQ : nB;
+            const int* cntv = which == 0 ? qcount : count;
             for (int n = 0; n < N; ++n) {
                 size_t off = ((size_t)bh * N + n) * dh;
                 for (int d = 0; d < dh; ++d) xi[d] = (double)x[off + d];
                 rotate_pairs(dh / 2, tcs + (size_t)n * dh, xi, xr, dh);
-                int blk = orc_block_of(c, n);
+                int blk = which == 0 ? orc_qblock_of(c, n) : orc_block_of(c, n);
                 for (int d = 0; d < dh; ++d) {
                     mean[(size_t)blk * dh + d] += xr[d];
                     mag[(size_t)blk * dh + d] += fabs(xi[d & ~1]) + fabs(xi[d | 1]);
                 }
             }
-            for (int blk = 0; blk < nB; ++blk) {
-                int cnt = count[blk];
+            for (int blk = 0; blk < nblk; ++blk) {
+                int cnt = cntv[blk];
                 for (int d = 0; d < dh; ++d) {
                     mean[(size_t)blk * dh + d] /= (double)cnt;
                     mag[(size_t)blk * dh + d] /= (double)cnt;
                 }
             }
         }
-        for (int i = 0; i < nB; ++i) {
+        for (int i = 0; i < nQ; ++i) {
             const double* qi = qb + (size_t)i * dh;
             const double* qm = qa + (size_t)i * dh;
             double tmax = 0.0;
@@ -513,24 +562,26 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
                 }
                 row[j].s = s * isd;
                 row[j].j = j;
-                if (scores) scores[((size_t)bh * nB + i) * nB + j] = s * isd;
-                /* rotation (3u) + pooling over <= bs terms + 1 divide, per
+                if (scores) scores[((size_t)bh * nQ + i) * nB + j] = s * isd;
+                /* rotation (3u) + pooling over <= pool terms + 1 divide, per
                  * operand; dot product over dh terms; final scale. */
-                double e = u * ((double)(dh + 2) * a1 + (double)(bs + 4) * a2) * isd;
+                double e = u * ((double)(dh + 2) * a1 + (double)(pool + 4) * a2) * isd;
                 if (e > tmax) tmax = e;
             }
             qsort(row, (size_t)nB, sizeof(scored), cmp_scored);
-            int32_t* out = kv_idx + ((size_t)bh * nB + i) * nk;
+            int32_t* out = kv_idx + ((size_t)bh * nQ + i) * nk;
             for (int t = 0; t < nk; ++t) out[t] = row[t].j;
             qsort(out, (size_t)nk, sizeof(int32_t), cmp_int);
-            if (gap) gap[(size_t)bh * nB + i] = nk < nB ? row[nk - 1].s - row[nk].s : INFINITY;
-            if (tau) tau[(size_t)bh * nB + i] = 2.0 * 4.0 * tmax;
+            if (gap) gap[(size_t)bh * nQ + i] = nk < nB ? row[nk - 1].s - row[nk].s : INFINITY;
+            if (tau) tau[(size_t)bh * nQ + i] = 2.0 * 4.0 * tmax;
         }
         free(qb); free(kb); free(qa); free(ka); free(xr); free(xi); free(row);
     }
     free(tcs);
     free(members);
     free(count);
+    free(qmembers);
+    free(qcount);
 }
 
 /* ------------------------------------------------------------------ */
@@ -545,17 +596,20 @@ void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const
                      const int32_t* kv_idx, int n_keep, const uint8_t* qb_sel, double* o_s)
 {
     int BH = c->B * c->H, dh = c->dh, N = c->N, bs = c->block;
-    int nB = orc_num_blocks(c);
+    int nB = orc_num_blocks(c), nQ = orc_num_qblocks(c), qbs = qblock_size(c);
     double isd = 1.0 / sqrt((double)dh);
-    int ntask = BH * nB;
+    int ntask = BH * nQ;
     int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
     int* count = (int*)malloc(sizeof(int) * (size_t)nB);
+    int* qmembers = (int*)malloc(sizeof(int) * (size_t)nQ * qbs);
+    int* qcount = (int*)malloc(sizeof(int) * (size_t)nQ);
     block_members(c, members, count);
+    qblock_members(c, qmembers, qcount);
 #pragma omp parallel for schedule(dynamic, 1)
     for (int task = 0; task < ntask; ++task) {
-        int bh = task / nB, i = task % nB;
+        int bh = task / nQ, i = task % nQ;
         if (qb_sel && !qb_sel[i]) continue;
-        const int32_t* kept = kv_idx + ((size_t)bh * nB + i) * n_keep;
+        const int32_t* kept = kv_idx + ((size_t)bh * nQ + i) * n_keep;
         int nkeys = 0;
         for (int t = 0; t < n_keep; ++t) nkeys += count[kept[t]];
         int* keys = (int*)malloc(sizeof(int) * (size_t)nkeys);
@@ -563,8 +617,8 @@ void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const
         int kk = 0;
         for (int t = 0; t < n_keep; ++t)
             for (int m = 0; m < count[kept[t]]; ++m) keys[kk++] = members[(size_t)kept[t] * bs + m];
-        for (int mi = 0; mi < count[i]; ++mi) {
-            int p = members[(size_t)i * bs + mi];
+        for (int mi = 0; mi < qcount[i]; ++mi) {
+            int p = qmembers[(size_t)i * qbs + mi];
             const double* qp = qr + ((size_t)bh * N + p) * dh;
             double mx = -INFINITY;
             for (int t = 0; t < nkeys; ++t) {
@@ -589,6 +643,8 @@ void orc_sparse_attn(const orc_cfg* c, const double* qr, const double* kr, const
     }
     free(members);
     free(count);
+    free(qmembers);
+    free(qcount);
 }
 
 /* ------------------------------------------------------------------ */
@@ -606,8 +662,8 @@ void orc_forward(const orc_cfg* c, const float* q, const float* k, const float* 
                  double* o, int32_t* kv_idx_out, double* o_s_out, double* C_out, double* z_out)
 {
     size_t nel = (size_t)c->B * c->H * c->N * c->dh;
-    int nB = orc_num_blocks(c), nk = orc_num_keep(c);
-    size_t nmask = (size_t)c->B * c->H * nB * nk;
+    int nQ = orc_num_qblocks(c), nk = orc_num_keep(c);
+    size_t nmask = (size_t)c->B * c->H * nQ * nk;
     int32_t* mask = (int32_t*)malloc(sizeof(int32_t) * nmask);
     if (mask_override) memcpy(mask, mask_override, sizeof(int32_t) * nmask);
     else orc_block_mask(c, q, k, mask, NULL, NULL, NULL);
@@ -745,6 +801,10 @@ void orc_backward(const orc_cfg* c, const float* q, const float* k, const float*
     int* members = (int*)malloc(sizeof(int) * (size_t)nB * bs);
     int* count = (int*)malloc(sizeof(int) * (size_t)nB);
     block_members(c, members, count);
+    int nQ = orc_num_qblocks(c), qbs = qblock_size(c);
+    int* qmembers = (int*)malloc(sizeof(int) * (size_t)nQ * qbs);
+    int* qcount = (int*)malloc(sizeof(int) * (size_t)nQ);
+    qblock_members(c, qmembers, qcount);
     double* dPq_bh = (double*)calloc((size_t)BH * nrd, sizeof(double));
     double* dPk_bh = (double*)calloc((size_t)BH * nrd, sizeof(double));
     double* dg_bh = (double*)calloc((size_t)BH * N, sizeof(double));
@@ -815,8 +875,8 @@ void orc_backward(const orc_cfg* c, const float* q, const float* k, const float*
                                 dk + head + (size_t)j * dh, dPk_bh + (size_t)bh * nrd);
         }
         /* block-sparse softmax attention: s = q^r k^r / sqrt(d_h), P = softmax(s), O^s = P v */
-        for (int i = 0; i < nB; ++i) {
-            const int32_t* kept = kv_idx + ((size_t)bh * nB + i) * nk;
+        for (int i = 0; i < nQ; ++i) {
+            const int32_t* kept = kv_idx + ((size_t)bh * nQ + i) * nk;
             int nkeys = 0;
             for (int t = 0; t < nk; ++t) nkeys += count[kept[t]];
             int* keys = (int*)malloc(sizeof(int) * (size_t)nkeys);
@@ -825,8 +885,8 @@ void orc_backward(const orc_cfg* c, const float* q, const float* k, const float*
             int kk = 0;
             for (int t = 0; t < nk; ++t)
                 for (int m = 0; m < count[kept[t]]; ++m) keys[kk++] = members[(size_t)kept[t] * bs + m];
-            for (int mi = 0; mi < count[i]; ++mi) {
-                int p = members[(size_t)i * bs + mi];
+            for (int mi = 0; mi < qcount[i]; ++mi) {
+                int p = qmembers[(size_t)i * qbs + mi];
                 const double* qp = qr + head + (size_t)p * dh;
                 const double* dop = dOs + (size_t)p * dh;
                 double mx = -INFINITY;
@@ -886,6 +946,7 @@ void orc_backward(const orc_cfg* c, const float* q, const float* k, const float*
             dgate[(size_t)b * N + p] = sum;
         }
     free(qr); free(kr); free(os); free(C); free(tcs); free(members); free(count);
+    free(qmembers); free(qcount);
     free(dPq_bh); free(dPk_bh); free(dg_bh);
 }
 

@@ -69,9 +69,10 @@ def directional(O, cfg, x, mask, rope_mode, dO, name, delta, h):
 
 
 # (feature map, RoPE placement, block geometry); the cube case has ragged edge cubes
-# (5 x 5 x 7 tokens: 2 x 2 x 2 cubes, 4 of 8 kept)
+# (5 x 5 x 7 tokens: 2 x 2 x 2 cubes, 4 of 8 kept); "q128" takes 128-token query blocks
+# against 64-token key blocks (3 x 7 x 11 tokens: query blocks of 128 and 103, 2 of 4 kept)
 CASES = [("silu", 0, "flat"), ("gelu", 1, "flat"), ("tanh", 2, "flat"), ("identity", 0, "flat"),
-         ("silu", 1, "flat"), ("silu", 0, "cube")]
+         ("silu", 1, "flat"), ("silu", 0, "cube"), ("silu", 0, "q128")]
 
 
 @pytest.mark.parametrize("act,rope_mode,geometry", CASES)
@@ -79,8 +80,12 @@ def test_gradients_match_central_differences(oracle, act, rope_mode, geometry):
     """Each gradient of L = sum(dO * O) dotted with a random direction equals the directional
     derivative of the (pinned) forward pass under the same fixed mask."""
     O = oracle
-    cfg = small_cfg(lowrank_act=act) if geometry == "flat" else \
-        small_cfg(lowrank_act=act, T=5, block_geometry="cube")
+    if geometry == "flat":
+        cfg = small_cfg(lowrank_act=act)
+    elif geometry == "cube":
+        cfg = small_cfg(lowrank_act=act, T=5, block_geometry="cube")
+    else:
+        cfg = small_cfg(lowrank_act=act, T=3, Hh=7, Ww=11, qblock=128)
     x = draw(cfg)
     rng = np.random.default_rng(7)
     dO = rng.standard_normal((1, cfg["H"], cfg["N"], 128)).astype(np.float32)

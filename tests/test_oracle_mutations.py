@@ -35,6 +35,12 @@ MUTATIONS = {
     "ragged_keys_padded": ("for (int t = 0; t < nkeys; ++t) { s[t] = exp(s[t] - mx); den += s[t]; }",
                            "for (int t = 0; t < nkeys; ++t) { s[t] = exp(s[t] - mx); den += s[t]; } "
                            "den += (double)((64 - nkeys % 64) % 64) * exp(-mx);"),
+    "qblock_pool_divisor": ("const int* cntv = which == 0 ? qcount : count;",
+                            "const int* cntv = which == 0 ? count : count;"),
+    "qblock_sparse_rows": ("for (int mi = 0; mi < qcount[i]; ++mi) {\n            int p = qmembers",
+                           "for (int mi = 0; mi < qcount[i] && mi < bs; ++mi) {\n            int p = qmembers"),
+    "qblock_backward_rows": ("for (int mi = 0; mi < qcount[i]; ++mi) {\n                int p = qmembers",
+                             "for (int mi = 0; mi < qcount[i] && mi < bs; ++mi) {\n                int p = qmembers"),
     "cube_axis_stride": ("return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;",
                          "return ((t / CUBE) * ny + x / CUBE) * nx + y / CUBE;"),
     "cube_grid_rounding": ("int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;",

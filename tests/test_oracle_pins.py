@@ -567,3 +567,70 @@ def test_gate_pins(oracle):
         Xd = X.copy()
         Xd[:, :, d] += 0.5
         assert np.allclose(logit(O.gate(Xd, w, b0)) - logit(g), 0.5 * float(w[d]), rtol=0, atol=1e-9)
+
+
+# ---------------------------------------------------------------- 128-token query blocks
+
+def test_query_blocks_of_128_tokens(oracle):
+    """qblock = 128 (the b_q = 128 / b_kv = 64 tiling of the block-sparse attentions the paper builds
+    on): the query blocks are 128-token chunks, the last one ragged, and the key blocks stay 64-token
+    chunks; unset, both are the 64-token chunks.  Cube geometry takes no query-block size."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=9, Ww=10, qblock=128)       # 360 tokens: query blocks 128, 128, 104
+    assert O.num_qblocks(cfg) == 3 and O.num_blocks(cfg) == 6
+    assert np.array_equal(O.qblock_of(cfg), np.arange(360) // 128)
+    assert np.array_equal(O.block_of(cfg), np.arange(360) // 64)
+    base = small_cfg(T=4, Hh=9, Ww=10)
+    assert O.num_qblocks(base) == 6 and np.array_equal(O.qblock_of(base), np.arange(360) // 64)
+    with pytest.raises(ValueError):
+        O.make_config(small_cfg(T=4, Hh=8, Ww=8, qblock=128, block_geometry="cube"))
+
+
+def test_query_block_scores_are_count_weighted_chunk_scores(oracle):
+    """A 128-token query block's pooled mean is the count-weighted mean of its two 64-token halves'
+    means, and the score is linear in q_bar, so its score row is the count-weighted mean of the two
+    halves' rows (ragged tail: 104 = 64 + 40 tokens).  Its kept set is its n_keep best key blocks,
+    ties to the lower id, ascending."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=9, Ww=10, keep=0.34)
+    x = draw(cfg)
+    _, s64, _, _ = O.block_mask(cfg, x["q"], x["k"])
+    idx, s128, _, _ = O.block_mask(dict(cfg, qblock=128), x["q"], x["k"])
+    assert idx.shape == (1, cfg["H"], 3, 2) and s128.shape == (1, cfg["H"], 3, 6)
+    cnt = np.bincount(np.arange(cfg["N"]) // 64).astype(np.float64)
+    for I in range(3):
+        a, b = 2 * I, 2 * I + 1
+        want = (cnt[a] * s64[:, :, a] + cnt[b] * s64[:, :, b]) / (cnt[a] + cnt[b])
+        np.testing.assert_allclose(s128[:, :, I], want, rtol=1e-12, atol=1e-14)
+    for h in range(cfg["H"]):
+        for I in range(3):
+            order = sorted(range(6), key=lambda j: (-s128[0, h, I, j], j))
+            assert list(idx[0, h, I]) == sorted(order[:2])
+
+
+def test_query_block_sparse_branch_shares_the_mask_row(oracle):
+    """Every query of a 128-token block attends to that block's kept key blocks: the sparse branch
+    equals, bit for bit, the 64-token-chunk branch under the mask whose rows 2I and 2I + 1 are row I;
+    query-block selection and the full forward follow the 128-token blocks; keep = 1 is dense SDPA."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=9, Ww=10, keep=0.34, dist="normal_gate")
+    c128 = dict(cfg, qblock=128)
+    x = draw(cfg)
+    qr, kr = O.rope_full(cfg, x["q"]), O.rope_full(cfg, x["k"])
+    idx, _, _, _ = O.block_mask(c128, x["q"], x["k"])
+    got = O.sparse_attn(c128, qr, kr, x["v"], idx)
+    dup = np.ascontiguousarray(np.repeat(idx, 2, axis=2)[:, :, :6])
+    np.testing.assert_array_equal(got, O.sparse_attn(cfg, qr, kr, x["v"], dup))
+    sel = O.sparse_attn(c128, qr, kr, x["v"], idx, qblocks=[1])
+    np.testing.assert_array_equal(sel[:, :, 128:256], got[:, :, 128:256])
+    assert np.isnan(sel[:, :, :128]).all() and np.isnan(sel[:, :, 256:]).all()
+    fw = O.forward(c128, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"])
+    np.testing.assert_array_equal(fw["kv_idx"], idx)
+    np.testing.assert_array_equal(fw["o_s"], got)
+    fs = O.forward(c128, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], qblocks=[2])
+    np.testing.assert_array_equal(fs["o"][:, :, 256:], fw["o"][:, :, 256:])
+    assert np.isnan(fs["o"][:, :, :256]).all()
+    full = dict(c128, keep=1.0)
+    idx1, _, _, _ = O.block_mask(full, x["q"], x["k"])
+    np.testing.assert_allclose(O.sparse_attn(full, qr, kr, x["v"], idx1), sdpa64(qr, kr, x["v"]),
+                               rtol=1e-11, atol=1e-12)
