@@ -41,6 +41,7 @@ MUTATIONS = {
                            "for (int mi = 0; mi < qcount[i] && mi < bs; ++mi) {\n            int p = qmembers"),
     "qblock_backward_rows": ("for (int mi = 0; mi < qcount[i]; ++mi) {\n                int p = qmembers",
                              "for (int mi = 0; mi < qcount[i] && mi < bs; ++mi) {\n                int p = qmembers"),
+    "tau_fp64_roundoff": ("const double u = ldexp(1.0, -24);", "const double u = ldexp(1.0, -53);"),
     "cube_axis_stride": ("return ((t / CUBE) * nx + x / CUBE) * ny + y / CUBE;",
                          "return ((t / CUBE) * ny + x / CUBE) * nx + y / CUBE;"),
     "cube_grid_rounding": ("int nx = (c->Hh + CUBE - 1) / CUBE, ny = (c->Ww + CUBE - 1) / CUBE;",

@@ -140,6 +140,56 @@ def test_mask_is_the_best_subset_by_brute_force(oracle):
             assert gap[0, h, i] == pytest.approx(srt[nk - 1] - srt[nk], abs=1e-15)
 
 
+def fp32_block_scores(O, cfg, x, order, dot):
+    """Block scores evaluated in fp32 arithmetic: the rotated rows rounded to fp32, each block's sum
+    accumulated in fp32 (ascending, descending or numpy's pairwise order), the fp32 mean, and fp32 dot
+    products (sequential over d_h or a float32 matmul), scaled by fp32 1/sqrt(d_h)."""
+    qr = O.rope_full(cfg, x["q"]).astype(np.float32)[0]
+    kr = O.rope_full(cfg, x["k"]).astype(np.float32)[0]
+    H, N = cfg["H"], cfg["N"]
+    nb = -(-N // 64)
+
+    def pooled(xr):
+        out = np.zeros((H, nb, 128), np.float32)
+        for b in range(nb):
+            rows = xr[:, b * 64:min(N, (b + 1) * 64)]
+            if order == "pairwise":
+                acc = rows.sum(axis=1, dtype=np.float32)
+            else:
+                seq = rows if order == "ascending" else rows[:, ::-1]
+                acc = np.zeros((H, 128), np.float32)
+                for t in range(seq.shape[1]):
+                    acc = acc + seq[:, t]
+            out[:, b] = acc / np.float32(rows.shape[1])
+        return out
+
+    qb, kb = pooled(qr), pooled(kr)
+    if dot == "sequential":
+        s = np.zeros((H, nb, nb), np.float32)
+        for d in range(128):
+            s = s + qb[:, :, None, d] * kb[:, None, :, d]
+    else:
+        s = np.matmul(qb, kb.transpose(0, 2, 1))
+    return s * np.float32(1.0 / math.sqrt(128))
+
+
+@pytest.mark.parametrize("dist", ["normal", "rmsnorm"])
+def test_near_tie_bound_covers_fp32_scores(oracle, dist):
+    """The near-tie rule (reading 12) rests on tau / 8 bounding how far an fp32 evaluation of a score
+    row can sit from the fp64 one: checked for fp32 evaluations in six summation orders.  The bound
+    must also stay meaningful: below 1e-3 of the largest score."""
+    O = oracle
+    cfg = small_cfg(T=4, Hh=9, Ww=10, dist=dist)             # 360 tokens: 6 blocks, the last of 40
+    x = draw(cfg)
+    _, s64, _, tau = O.block_mask(cfg, x["q"], x["k"])
+    bound = tau[0] / 8
+    assert (bound > 0).all() and bound.max() <= 1e-3 * np.abs(s64).max()
+    for order in ("ascending", "descending", "pairwise"):
+        for dot in ("sequential", "matmul"):
+            err = np.abs(fp32_block_scores(O, cfg, x, order, dot).astype(np.float64) - s64[0])
+            assert (err <= bound[:, :, None]).all(), (order, dot, float((err / bound[:, :, None]).max()))
+
+
 def test_mask_closed_form_single_token(oracle):
     """Pooling divides by the block's own token count (the ragged last block too);
     ties go to the lower key block.  q and k are zero except one token whose
