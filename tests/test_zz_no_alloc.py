@@ -6,7 +6,8 @@ serving).  This entry point keeps its scratch in a static device array inside
 the library.  The GPU test checks it against the workspace-based
 rola_lowrank_summary, through the C ABI, on two calls in a row (the second
 call reuses the array the first one left behind).  This file is collected
-last, so a run that stops at the first failure has run everything else.
+next to last (before the guard canaries), so a run that stops at the first
+failure has run the parity tests first.
 """
 import ctypes
 
