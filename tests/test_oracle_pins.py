@@ -384,6 +384,29 @@ def test_summary_form_equals_explicit_quadratic_form(oracle):
     np.testing.assert_allclose(z, kt.sum(axis=2), rtol=1e-12, atol=1e-12)
 
 
+@pytest.mark.parametrize("r", [16, 64])
+def test_even_odd_split_evaluation_equals_interleaved(oracle, r):
+    """T3 / Sec. 4.5: P's rows taken as the even rows then the odd rows, SiLU applied to both halves,
+    element i of the first half rotated with element i of the second half by pair i's angle, and the
+    result put back in interleaved order, is the oracle's interleaved feature vector (numpy matmuls;
+    r = 64 spans temporal and height pairs)."""
+    O = oracle
+    cfg = small_cfg(r=r, T=2, Hh=3, Ww=4)
+    x = draw(cfg)
+    want = O.lowrank_features(cfg, x["k"], x["P_k"])
+    P, k = x["P_k"].astype(np.float64), x["k"].astype(np.float64)
+    got = np.empty_like(want)
+    for n in range(cfg["N"]):
+        pos = O.position(cfg, n)
+        ang = np.array([O.pair_angle(cfg, m, pos) for m in range(r // 2)])
+        for h in range(cfg["H"]):
+            ue, uo = P[h, 0::2] @ k[0, h, n], P[h, 1::2] @ k[0, h, n]
+            ae, ao = ue / (1 + np.exp(-ue)), uo / (1 + np.exp(-uo))
+            got[0, h, n, 0::2] = ae * np.cos(ang) - ao * np.sin(ang)
+            got[0, h, n, 1::2] = ae * np.sin(ang) + ao * np.cos(ang)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-13)
+
+
 def test_features_identity_projection_reduces_to_silu_then_rope(oracle):
     """With r = d_h and P = I the feature map of Eq. (qklr) is R(p) SiLU(x): torch's
     SiLU, then the full RoPE; the inside variant is SiLU(R(p) x)."""
