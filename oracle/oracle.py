@@ -25,10 +25,11 @@ _lib = None
 
 
 def build(force: bool = False) -> str:
-    """Compile rola_oracle.c into liboracle.so with gcc (-O2, OpenMP, no fast-math)."""
+    """Compile rola_oracle.c into liboracle.so with gcc (-O2, OpenMP, no fast-math, and no
+    contraction of a * b + c into an fma, so each expression rounds as written on every host)."""
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".tmp{os.getpid()}"
-        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c99",
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c99", "-ffp-contract=off",
                                "-o", tmp, _SRC, "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
@@ -90,6 +91,7 @@ def _get():
             lib.orc_lowrank_explicit.argtypes = [cfgp, P, P, P, P, P, P]
             lib.orc_rope_full.argtypes = [cfgp, P, P]
             lib.orc_block_mask.argtypes = [cfgp, P, P, P, P, P, P]
+            lib.orc_block_mask_f32.argtypes = [cfgp, P, P, P, P]
             lib.orc_sparse_attn.argtypes = [cfgp, P, P, P, P, ctypes.c_int, P, P]
             lib.orc_forward.argtypes = [cfgp, P, P, P, P, P, P, P, P, P, P, P, P, P]
             lib.orc_gate.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, ctypes.c_double, P]
@@ -325,6 +327,22 @@ def block_mask(cfg: dict, q, k):
     _get().orc_block_mask(ctypes.byref(c), qp, kp, idx.ctypes.data, scores.ctypes.data,
                           gap.ctypes.data, tau.ctypes.data)
     return idx, scores, gap, tau
+
+
+def block_mask_f32(cfg: dict, q, k):
+    """The block mask as an fp32 decision (the precision of the CUDA path), every rounding fixed:
+    fp32 (cos, sin) table, fma rotation, pairwise pooling over the block's slots, one divide,
+    ascending-d fma chain, one scale product, ties to the lower block.
+
+    Returns (kv_idx int32 [B,H,nQB,n_keep] ascending, fp32 scores [B,H,nQB,nKB] as float64)."""
+    c = make_config(cfg)
+    q, qp = _f32(q)
+    k, kp = _f32(k)
+    nb, nq, nk = num_blocks(cfg), num_qblocks(cfg), num_keep(cfg)
+    idx = np.empty((c.B, c.H, nq, nk), dtype=np.int32)
+    scores = np.empty((c.B, c.H, nq, nb))
+    _get().orc_block_mask_f32(ctypes.byref(c), qp, kp, idx.ctypes.data, scores.ctypes.data)
+    return idx, scores
 
 
 def sparse_attn(cfg: dict, qr, kr, v, kv_idx, qblocks=None) -> np.ndarray:

@@ -489,13 +489,25 @@ static int cmp_int(const void* a, const void* b)
  *   scores [B][H][nQB][nKB]      s_ij = q_bar_i . k_bar_j / sqrt(dh)
  *   gap    [B][H][nQB]           s_(n_keep) - s_(n_keep+1) in descending order
  *                                (+inf when n_keep == nKB)
- *   tau    [B][H][nQB]           an upper bound on the difference between this
- *                                score row and one evaluated in fp32 arithmetic
- *                                (u = 2^-24) in any summation order, times 2
- *                                (two scores enter a comparison) times a safety
- *                                factor 4.  A row with gap <= tau is a
- *                                near-tie row: more than one kept set is a
- *                                correct fp32 answer there.
+ *   tau    [B][H][nQB]           twice the largest, over the row, of a
+ *                                rigorous bound on |s32 - s| for the fp32
+ *                                evaluation of orc_block_mask_f32 (u = 2^-24),
+ *                                two scores entering every comparison.  A row
+ *                                with gap > tau keeps the same set in fp32 and
+ *                                in exact arithmetic; a row with gap <= tau is
+ *                                a near-tie row, where the fp32 decision may
+ *                                keep another valid set.
+ *
+ * The bound, per score, first order in u with a relative slack of 2^-12 for
+ * the higher-order terms (Higham, Accuracy and Stability of Numerical
+ * Algorithms, Sec. 3.1 and 4.2): a rotated coordinate y = x0 c - x1 s is off
+ * by at most 3u (|x0| + |x1|) (c and s rounded once each, one product, one
+ * fma); a pairwise sum over L levels adds gamma_L sum |y|; the division adds
+ * u; so a pooled mean is off by at most (L + 4) u M_d, M_d the pooled
+ * |x0| + |x1| of coordinate d's pair.  The d_h-term fma chain adds
+ * gamma_dh sum |q_bar_d k_bar_d|, the scale (rounded once, one product) 2u of
+ * |s|.  With a1 = sum |q_bar_d| |k_bar_d| and a2 = sum (M^q_d |k_bar_d| +
+ * |q_bar_d| M^k_d):  |s32 - s| <= u ((d_h + 2) a1 + (L + 4) a2) / sqrt(d_h).
  */
 void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* kv_idx,
                     double* scores, double* gap, double* tau)
@@ -503,7 +515,9 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
     int BH = c->B * c->H, dh = c->dh, N = c->N, bs = c->block;
     int nB = orc_num_blocks(c), nk = orc_num_keep(c);
     int nQ = orc_num_qblocks(c), qbs = qblock_size(c);
-    int pool = qbs > bs ? qbs : bs;                         /* most tokens a pooled mean sums */
+    int pool = qbs > bs ? qbs : bs;                         /* most slots a pooled mean sums */
+    int levels = 0;                                         /* pairwise-summation depth, ceil(log2 pool) */
+    while ((1 << levels) < pool) ++levels;
     double isd = 1.0 / sqrt((double)dh);
     const double u = ldexp(1.0, -24);
     double* tcs = token_cs(c);
@@ -563,9 +577,9 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
                 row[j].s = s * isd;
                 row[j].j = j;
                 if (scores) scores[((size_t)bh * nQ + i) * nB + j] = s * isd;
-                /* rotation (3u) + pooling over <= pool terms + 1 divide, per
-                 * operand; dot product over dh terms; final scale. */
-                double e = u * ((double)(dh + 2) * a1 + (double)(pool + 4) * a2) * isd;
+                /* per operand: rotation 3u, pairwise pooling over `levels`
+                 * levels, one divide; dot product over dh terms; scale 2u. */
+                double e = u * ((double)(dh + 2) * a1 + (double)(levels + 4) * a2) * isd * (1.0 + ldexp(1.0, -12));
                 if (e > tmax) tmax = e;
             }
             qsort(row, (size_t)nB, sizeof(scored), cmp_scored);
@@ -573,7 +587,7 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
             for (int t = 0; t < nk; ++t) out[t] = row[t].j;
             qsort(out, (size_t)nk, sizeof(int32_t), cmp_int);
             if (gap) gap[(size_t)bh * nQ + i] = nk < nB ? row[nk - 1].s - row[nk].s : INFINITY;
-            if (tau) tau[(size_t)bh * nQ + i] = 2.0 * 4.0 * tmax;
+            if (tau) tau[(size_t)bh * nQ + i] = 2.0 * tmax;
         }
         free(qb); free(kb); free(qa); free(ka); free(xr); free(xi); free(row);
     }
@@ -582,6 +596,140 @@ void orc_block_mask(const orc_cfg* c, const float* q, const float* k, int32_t* k
     free(count);
     free(qmembers);
     free(qcount);
+}
+
+/*
+ * The block mask as an fp32 decision.  Keeping the n_keep largest scores turns
+ * floating-point values into integers, so the checker takes that decision in
+ * the precision the CUDA path takes it in, fp32, with every rounding fixed by
+ * the following evaluation (the definition above, step by step, in fp32):
+ *   table    (c, s) of a pair: the fp64 cos / sin of the fp64 pair angle of
+ *            orc_pair_angle, each rounded once to fp32;
+ *   rotate   y0 = fma(x0, c, -(x1 s)), y1 = fma(x0, s, x1 c): each product
+ *            and each fma rounded to fp32;
+ *   pool     pairwise summation (Higham, Accuracy and Stability of Numerical
+ *            Algorithms, Sec. 4.2) of the block's slots in slot order:
+ *            sum(x[0..n)) = sum(x[0..h)) + sum(x[h..n)), h = floor(n/2), the
+ *            slots being
+ *            the `block` (query side: qblock) positions of a chunk, or the
+ *            CUBE^3 positions 16 dt + 4 dx + dy of a cube; a slot outside the
+ *            sequence or the grid holds +0.  Then one fp32 division by the
+ *            number of tokens the block holds;
+ *   score    an fp32 fma chain over d = 0, 1, ..., d_h - 1 starting from +0,
+ *            then one fp32 product with the fp32 rounding of 1/sqrt(d_h);
+ *   select   the n_keep largest of a row, ties to the lower block index
+ *            (+0 and -0 are equal), listed ascending.
+ * Outputs: kv_idx [B][H][nQB][n_keep]; scores32 [B][H][nQB][nKB] (may be
+ * NULL), the fp32 scores widened to double.
+ */
+static float pairwise_f32(const float* x, int n)
+{
+    if (n == 1) return x[0];
+    return pairwise_f32(x, n / 2) + pairwise_f32(x + n / 2, n - n / 2);
+}
+
+/* Token held by slot i of block b (-1: an empty slot); query side when qside. */
+static int slot_token(const orc_cfg* c, int b, int i, int qside)
+{
+    if (c->geometry == 1) {
+        int cubes_x = (c->Hh + CUBE - 1) / CUBE;          /* cube grid, t-major numbering */
+        int cubes_y = (c->Ww + CUBE - 1) / CUBE;
+        int ct = b / (cubes_x * cubes_y), cx = (b / cubes_y) % cubes_x, cy = b % cubes_y;
+        int t = CUBE * ct + i / (CUBE * CUBE), x = CUBE * cx + (i / CUBE) % CUBE, y = CUBE * cy + i % CUBE;
+        if (t >= c->T || x >= c->Hh || y >= c->Ww) return -1;
+        return (t * c->Hh + x) * c->Ww + y;
+    }
+    int size = qside ? qblock_size(c) : c->block;
+    int n = b * size + i;
+    return n < c->N ? n : -1;
+}
+
+typedef struct { float s; int j; } scored32;
+
+static int cmp_scored32(const void* a, const void* b)
+{
+    const scored32* x = (const scored32*)a;
+    const scored32* y = (const scored32*)b;
+    if (x->s > y->s) return -1;
+    if (x->s < y->s) return 1;
+    return (x->j > y->j) - (x->j < y->j);
+}
+
+void orc_block_mask_f32(const orc_cfg* c, const float* q, const float* k, int32_t* kv_idx, double* scores32)
+{
+    int BH = c->B * c->H, dh = c->dh, N = c->N;
+    int nB = orc_num_blocks(c), nk = orc_num_keep(c), nQ = orc_num_qblocks(c);
+    int kslots = c->geometry == 1 ? CUBE * CUBE * CUBE : c->block;
+    int qslots = c->geometry == 1 ? kslots : qblock_size(c);
+    const float scale = (float)(1.0 / sqrt((double)dh));
+    /* the fp32 (cos, sin) of every pair at every token */
+    float* tab = (float*)malloc(sizeof(float) * (size_t)N * dh);
+#pragma omp parallel for schedule(static)
+    for (int n = 0; n < N; ++n) {
+        double pos[3];
+        orc_position(c, n, pos);
+        for (int m = 0; m < dh / 2; ++m) {
+            double a = orc_pair_angle(c, m, pos);
+            tab[(size_t)n * dh + 2 * m] = (float)cos(a);
+            tab[(size_t)n * dh + 2 * m + 1] = (float)sin(a);
+        }
+    }
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bh = 0; bh < BH; ++bh) {
+        float* qbar = (float*)malloc(sizeof(float) * (size_t)nQ * dh);
+        float* kbar = (float*)malloc(sizeof(float) * (size_t)nB * dh);
+        int maxslots = qslots > kslots ? qslots : kslots;
+        float* col = (float*)malloc(sizeof(float) * (size_t)maxslots * dh);   /* [slot][d] rotated rows */
+        scored32* row = (scored32*)malloc(sizeof(scored32) * (size_t)nB);
+        for (int which = 0; which < 2; ++which) {
+            const float* x = which == 0 ? q : k;
+            float* mean = which == 0 ? qbar : kbar;
+            int nblk = which == 0 ? nQ : nB, slots = which == 0 ? qslots : kslots;
+            float* vals = (float*)malloc(sizeof(float) * (size_t)slots);
+            for (int b = 0; b < nblk; ++b) {
+                int cnt = 0;
+                for (int i = 0; i < slots; ++i) {
+                    int n = slot_token(c, b, i, which == 0);
+                    float* yr = col + (size_t)i * dh;
+                    if (n < 0) {
+                        for (int d = 0; d < dh; ++d) yr[d] = 0.0f;
+                        continue;
+                    }
+                    ++cnt;
+                    const float* xn = x + ((size_t)bh * N + n) * dh;
+                    const float* cs = tab + (size_t)n * dh;
+                    for (int m = 0; m < dh / 2; ++m) {
+                        float x0 = xn[2 * m], x1 = xn[2 * m + 1], cm = cs[2 * m], sm = cs[2 * m + 1];
+                        float p1 = x1 * sm, p2 = x1 * cm;
+                        yr[2 * m] = fmaf(x0, cm, -p1);
+                        yr[2 * m + 1] = fmaf(x0, sm, p2);
+                    }
+                }
+                for (int d = 0; d < dh; ++d) {
+                    for (int i = 0; i < slots; ++i) vals[i] = col[(size_t)i * dh + d];
+                    mean[(size_t)b * dh + d] = pairwise_f32(vals, slots) / (float)cnt;
+                }
+            }
+            free(vals);
+        }
+        for (int i = 0; i < nQ; ++i) {
+            const float* qi = qbar + (size_t)i * dh;
+            for (int j = 0; j < nB; ++j) {
+                const float* kj = kbar + (size_t)j * dh;
+                float acc = 0.0f;
+                for (int d = 0; d < dh; ++d) acc = fmaf(qi[d], kj[d], acc);
+                row[j].s = acc * scale;
+                row[j].j = j;
+                if (scores32) scores32[((size_t)bh * nQ + i) * nB + j] = (double)row[j].s;
+            }
+            qsort(row, (size_t)nB, sizeof(scored32), cmp_scored32);
+            int32_t* out = kv_idx + ((size_t)bh * nQ + i) * nk;
+            for (int t = 0; t < nk; ++t) out[t] = row[t].j;
+            qsort(out, (size_t)nk, sizeof(int32_t), cmp_int);
+        }
+        free(qbar); free(kbar); free(col); free(row);
+    }
+    free(tab);
 }
 
 /* ------------------------------------------------------------------ */

@@ -18,15 +18,18 @@
 // (k, v and q boxes of 32 x 128, 8 KB each), which keeps a CTA small enough
 // that two fit on an SM for r <= 48 (16 warps per SM hide the latency of the
 // dependent MMA and rotation chains).  Per half, 8 warps:
-//   rotate q, k (thread = token row mod 16 x 8 coordinates), store q^r, k^r,
-//   pool into registers; U = K P_k^T (mma.sync; warp = 16 tokens x a quarter
-//   or half of the r columns); k~ = R_r SiLU(U) to shared memory; the half's
+//   rotate q, k (thread = two neighbouring token rows x 8 coordinates), store
+//   q^r, k^r, pool; U = K P_k^T (mma.sync; warp = 16 tokens x a quarter or
+//   half of the r columns); k~ = R_r SiLU(U) to shared memory; the half's
 //   barrier; C^T += V^T k~ (warp = 16 of the 128 d columns, all r rows).
-// After the second half the row partials of the pooling are summed into the
-// block means.  The rotation, the pooling order (a thread adds its tokens
-// rs, rs + 16, rs + 32, rs + 48 in that order, then the 16 row partials are
-// added in order) and the divisions are those of the stand-alone rotate +
-// pool kernel, so both produce the same bits.
+// The block means are pairwise sums (the summation order the block mask is
+// defined with, every rounding fixed, so the decision is the same on any
+// kernel that evaluates it): a thread adds its two rows 2a, 2a + 1, the 16
+// lanes a of a half-warp add those nodes in a butterfly (levels 2-5 of the
+// tree over the half's 32 rows, each lane ending with one of the 16 pooled
+// coordinates), and after the second half the two halves' nodes are added
+// and divided by the block's token count -- the same bits as the stand-alone
+// rotate + pool kernel.
 //
 // The loads of half-stage i + S - 1 are issued (by lane 0 of warps 0-2, one
 // box each) right after half-stage i's barrier, when every thread is done
@@ -77,8 +80,8 @@ struct Layout {
         stage_bytes = fuse ? 3 * kHalf : 2 * kHalf;
         P = stages * stage_bytes;                                 // P_k of the current head, r rows x 256 B
         kt = P + R * 256;                                         // k~, two buffers of 32 rows
-        part = kt + 2 * kHalfRows * (2 * R + 16);                 // pooling partials [q|k][16][128] fp32
-        zsm = part + (fuse ? 2 * 16 * 128 * 4 : 0);
+        part = kt + 2 * kHalfRows * (2 * R + 16);
+        zsm = part;
         bars = zsm + 2 * R * 4;                                   // full[kMaxStages], abort
         total = bars + kMaxStages * 8 + 16;
     }
@@ -102,21 +105,46 @@ __device__ __forceinline__ void record_timeout(const Params& p, int where)
     if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = where;
 }
 
-// Rotates the 8 bf16 coordinates in w (4 pairs, (cos, sin) in cs), stores
-// them as bf16 at dst and adds the fp32 rotated values to acc.
-__device__ __forceinline__ void rotate8(const uint4& w, const float2 (&cs)[4], __nv_bfloat16* dst, float (&acc)[8])
+// Rotates the 8 bf16 coordinates in w (4 pairs, (cos, sin) in cs) into y
+// (fp32) and, for a token inside the sequence, stores them as bf16 at dst;
+// a token past the end gives y = +0 (an empty slot of the pairwise sum).
+__device__ __forceinline__ void rotate8(const uint4& w, const float2 (&cs)[4], __nv_bfloat16* dst, bool valid,
+                                        float (&y)[8])
 {
     const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
     uint32_t out[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         const float2 x = unpack_bf16(wv[q]);
-        const float2 y = rope_rotate(x.x, x.y, cs[q]);
-        out[q] = pack_bf16(y.x, y.y);
-        acc[2 * q] += y.x;
-        acc[2 * q + 1] += y.y;
+        const float2 r = rope_rotate(x.x, x.y, cs[q]);
+        out[q] = pack_bf16(r.x, r.y);
+        y[2 * q] = valid ? r.x : 0.0f;
+        y[2 * q + 1] = valid ? r.y : 0.0f;
     }
-    *reinterpret_cast<uint4*>(dst) = make_uint4(out[0], out[1], out[2], out[3]);
+    if (valid) *reinterpret_cast<uint4*>(dst) = make_uint4(out[0], out[1], out[2], out[3]);
+}
+
+// Levels 2-5 of the pairwise sum over a half's 32 rows: v holds this lane's
+// level-1 nodes (rows 2a, 2a + 1) of 16 pooled coordinates; the 16 lanes
+// a = lane mod 16 exchange halves of v in a butterfly (xor 1, 2, 4, 8), each
+// step adding the nodes of two neighbouring row ranges, so that lane a ends
+// with the node of all 32 rows for coordinate bitrev4(a) in v[0].  IEEE
+// addition commutes, so which lane holds the left operand does not matter.
+__device__ __forceinline__ void pairwise_butterfly(float (&v)[16], int a)
+{
+#pragma unroll
+    for (int lvl = 0; lvl < 4; ++lvl) {
+        const int off = 1 << lvl, half = 8 >> lvl;
+        const bool upper = (a >> lvl) & 1;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            if (i < half) {
+                const float keep = upper ? v[i + half] : v[i];
+                const float send = upper ? v[i] : v[i + half];
+                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+            }
+        }
+    }
 }
 
 __device__ __forceinline__ uint4 lds128(uint32_t a)
@@ -151,7 +179,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     const int S = lay.stages;
     const uint32_t sbase = smem_u32(smem);
     const uint32_t sP = sbase + lay.P, sKt = sbase + lay.kt;
-    float* part = reinterpret_cast<float*>(smem + lay.part);
     float* zsm = reinterpret_cast<float*>(smem + lay.zsm);
     const uint32_t full0 = sbase + lay.bars;
     volatile int* abort = reinterpret_cast<volatile int*>(smem + lay.bars + kMaxStages * 8);
@@ -174,6 +201,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     // warps 0, 1, 2 issue the k, v, q boxes; thread 0 also arms the barrier
     const uint32_t bytes = fuse ? 3 * kHalf : 2 * kHalf;
     auto issue = [&](int j) {
+        // test hook: the CTA's first half-stage is never loaded (nor its bytes armed), so the waits on it run out
+        if ((s.debug_flags & ROLA_DEBUG_SKIP_FIRST_K_COPY) && j == 0) return;
         const int u = u0 + (j >> 1), bh = u / s.nC, row = (u - bh * s.nC) * 64 + (j & 1) * kHalfRows;
         const uint32_t dst = sbase + (j % S) * lay.stage_bytes, bar = full0 + 8 * (j % S);
         if (tid == 0) {
@@ -191,7 +220,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
     const int mt = warp & 1, cg = warp >> 1;        // U: tokens 16 mt .. +15 of the half, column group cg
     const bool u_warp = cg < C::NSPLIT;             // (with two column groups, warps 4-7 skip U)
-    const int rs = tid >> 4, c8 = tid & 15;         // rotation: rows rs, rs + 16 of the half; 8 coordinates
+    // rotation and pooling: rows 2 pa, 2 pa + 1 of the half, 8 coordinates; the
+    // two rows are read in the order psw gives, so that a half-warp's 16-byte
+    // shared loads fall on 8 distinct bank groups
+    const int pa = tid & 15, c8 = tid >> 4, psw = (pa >> 2) & 1;
+    const int pel = ((pa & 1) << 3) | ((pa & 2) << 1) | ((pa & 4) >> 1) | ((pa & 8) >> 3);   // bitrev4(pa)
     const int hw = s.Hh * s.Ww;
     int axis[4];
 #pragma unroll
@@ -272,9 +305,9 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     {
         const int blk0 = u0 - (u0 / s.nC) * s.nC;
         position(blk0 * kBlock + mt * 16 + g, kt_t, kt_x, kt_y);
-        position(blk0 * kBlock + rs, rt_t, rt_x, rt_y);
+        position(blk0 * kBlock + 2 * pa, rt_t, rt_x, rt_y);
     }
-    float accq[8], acck[8];                         // pooling partials of the current block (both halves)
+    float pool0 = 0.0f;                             // pairwise node of the block's first half (element pel)
     int i = 0;                                      // half-stage index
     for (; i < count; ++i) {
         const int u = u0 + (i >> 1), h = i & 1;
@@ -296,13 +329,9 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
             bar_sync(1, kThreads);
             if (hb >= 0) {                         // a new head starts at its block 0
                 position(mt * 16 + g, kt_t, kt_x, kt_y);
-                position(rs, rt_t, rt_x, rt_y);
+                position(2 * pa, rt_t, rt_x, rt_y);
             }
             hb = bh;
-        }
-        if (h == 0) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) accq[e] = acck[e] = 0.0f;
         }
         const uint32_t stage = sbase + st * lay.stage_bytes;
         const uint32_t kb = stage, vb = stage + kHalf, qb = stage + 2 * kHalf;
@@ -328,37 +357,46 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
             for (int j = 0; j < 2; ++j) {
 #pragma unroll
                 for (int q = 0; q < 4; ++q) cs[j][q] = __ldg(p.tab + table_row(axis[q], t, x, y) * kPairs + c8 * 4 + q);
-                advance(16, t, x, y);
+                advance(1, t, x, y);
             }
         }
         advance(kHalfRows, kt_t, kt_x, kt_y);          // the next half's positions
         advance(kHalfRows, rt_t, rt_x, rt_y);
-        const bool ok = mbar_wait(full0 + 8 * st, (i / S) & 1, abort, s.wait_limit_ns);
+        // warp-uniform, so that the warp-wide shuffles and MMAs below see every lane
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(full0 + 8 * st, (i / S) & 1, abort, s.wait_limit_ns));
         if (ok) {
             if (fuse) {
-                // ---- rotate q and k, store q^r and k^r, pool (same order as the stand-alone kernel)
+                // ---- rotate q and k, store q^r and k^r, pool (pairwise, the stand-alone kernel's bits)
                 uint4 wq[2], wk[2];
 #pragma unroll
                 for (int j = 0; j < 2; ++j) {
-                    wq[j] = lds128(qb + hsw(rs + 16 * j, c8));
-                    wk[j] = lds128(kb + hsw(rs + 16 * j, c8));
+                    const int row = 2 * pa + (j ^ psw);
+                    wq[j] = lds128(qb + hsw(row, c8));
+                    wk[j] = lds128(kb + hsw(row, c8));
                 }
+                float v[16];
 #pragma unroll
-                for (int j = 0; j < 2; ++j) {
-                    const int n = n_half + rs + 16 * j;
-                    if (n < s.N) {
-                        const size_t go = ((size_t)bh * s.N + n) * kDh + c8 * 8;
-                        rotate8(wq[j], cs[j], p.qr + go, accq);
-                        rotate8(wk[j], cs[j], p.kr + go, acck);
+                for (int e = 0; e < 2; ++e) {           // row 2 pa + e, loaded by load e ^ psw
+                    const int n = n_half + 2 * pa + e;
+                    const bool valid = n < s.N;
+                    const size_t go = ((size_t)bh * s.N + (valid ? n : 0)) * kDh + c8 * 8;
+                    float yq[8], yk[8];
+                    rotate8((e ^ psw) ? wq[1] : wq[0], cs[e], p.qr + go, valid, yq);
+                    rotate8((e ^ psw) ? wk[1] : wk[0], cs[e], p.kr + go, valid, yk);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {               // level 1: row 2 pa + row 2 pa + 1
+                        v[c] = e ? v[c] + yq[c] : yq[c];
+                        v[8 + c] = e ? v[8 + c] + yk[c] : yk[c];
                     }
                 }
-                if (h == 1) {
-                    float* pq = part + (0 * 16 + rs) * kDh + c8 * 8;
-                    float* pk = part + (1 * 16 + rs) * kDh + c8 * 8;
-                    reinterpret_cast<float4*>(pq)[0] = make_float4(accq[0], accq[1], accq[2], accq[3]);
-                    reinterpret_cast<float4*>(pq)[1] = make_float4(accq[4], accq[5], accq[6], accq[7]);
-                    reinterpret_cast<float4*>(pk)[0] = make_float4(acck[0], acck[1], acck[2], acck[3]);
-                    reinterpret_cast<float4*>(pk)[1] = make_float4(acck[4], acck[5], acck[6], acck[7]);
+                pairwise_butterfly(v, pa);
+                if (h == 0) {
+                    pool0 = v[0];
+                } else {
+                    // the top node: first half + second half, then the mean over the block's tokens
+                    const int cnt = min(kBlock, s.N - blk * kBlock);
+                    float* dst = pel < 8 ? p.qbar : p.kbar;
+                    dst[((size_t)bh * s.nC + blk) * kDh + c8 * 8 + (pel & 7)] = (pool0 + v[0]) / (float)cnt;
                 }
             }
             if (u_warp) {
@@ -412,16 +450,6 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
         if (i >= 1 && issued < count) {       // half-stage i - 1 is done everywhere: refill its stage
             issue(issued);
             ++issued;
-        }
-        if (fuse && h == 1) {
-            // ---- block means: threads 0-127 q, 128-255 k; 16 row partials in order
-            const int which = tid >> 7, d = tid & 127;
-            const float* src = part + (which * 16) * kDh + d;
-            float sum = 0.0f;
-#pragma unroll
-            for (int r = 0; r < 16; ++r) sum += src[r * kDh];
-            const int cnt = min(kBlock, s.N - blk * kBlock);
-            (which ? p.kbar : p.qbar)[((size_t)bh * s.nC + blk) * kDh + d] = sum / (float)cnt;
         }
         // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 32 tokens
 #pragma unroll

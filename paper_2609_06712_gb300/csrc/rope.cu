@@ -45,7 +45,24 @@ cudaError_t launch_rope_table(const rola_config_t& cfg, float2* tab, cudaStream_
 // rotate + pool: one CTA per (64-token block, head, q|k).  256 threads: 16 per
 // token row (8 coordinates = 4 pairs each), 16 rows per pass, 4 passes.  Writes
 // the rotated rows in the storage dtype and the fp32 block mean of the
-// fp32-rotated (unrounded) values.
+// fp32-rotated (unrounded) values.  The block mean is the pairwise sum of the
+// block's 64 slots in slot order (slots past the sequence hold +0), divided
+// once by the token count: the evaluation order the block mask is defined
+// with, so that every kernel computing it gives the same bits.
+
+// Pairwise sum of the 64 values col[0], col[stride], ..., col[63 stride]:
+// sum(x[0..n)) = sum(x[0..n/2)) + sum(x[n/2..n)), evaluated level by level.
+__device__ __forceinline__ float pairwise64(const float* col, int stride)
+{
+    float v[kBlock];
+#pragma unroll
+    for (int i = 0; i < kBlock; ++i) v[i] = col[i * stride];
+#pragma unroll
+    for (int w = 1; w < kBlock; w *= 2)
+#pragma unroll
+        for (int i = 0; i < kBlock; i += 2 * w) v[i] = v[i] + v[i + w];
+    return v[0];
+}
 
 template <typename T>
 struct Vec8;
@@ -91,7 +108,7 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
                                                         T* __restrict__ kr, float* __restrict__ qbar,
                                                         float* __restrict__ kbar)
 {
-    __shared__ float part[16][kDh];
+    __shared__ __align__(16) float rot[kBlock][kDh];      // fp32 rotated rows, slot order
     const int blk = blockIdx.x, bh = blockIdx.y;
     const T* x = blockIdx.z == 0 ? q : k;
     T* xr = blockIdx.z == 0 ? qr : kr;
@@ -118,12 +135,11 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
         const int m = c8 * 4 + p;
         axis[p] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
     }
-    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 #pragma unroll
     for (int pass = 0; pass < kPasses; ++pass) {
         const int n = n0 + 16 * pass;
+        float o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
         if (n < s.N) {
-            float o[8];
 #pragma unroll
             for (int p = 0; p < 4; ++p) {
                 const int row = axis[p] == 0 ? t : (axis[p] == 1 ? s.T + xx : s.T + s.Hh + yy);
@@ -133,9 +149,10 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
                 o[2 * p + 1] = y.y;
             }
             Vec8<T>::store(xr + ((size_t)bh * s.N + n) * kDh + c8 * 8, o);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) acc[i] += o[i];
         }
+        float4* dst = reinterpret_cast<float4*>(&rot[rsub + 16 * pass][c8 * 8]);
+        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
         yy += 16;                           // advance to the token 16 further on
         while (yy >= s.Ww) {
             yy -= s.Ww;
@@ -145,15 +162,10 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
             }
         }
     }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) part[rsub][c8 * 8 + i] = acc[i];
     __syncthreads();
     if (threadIdx.x < kDh) {
-        float sum = 0.0f;
-#pragma unroll
-        for (int r = 0; r < 16; ++r) sum += part[r][threadIdx.x];
         const int cnt = min(kBlock, s.N - blk * kBlock);
-        xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = sum / (float)cnt;
+        xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = pairwise64(&rot[0][threadIdx.x], kDh) / (float)cnt;
     }
 }
 
@@ -172,7 +184,7 @@ __global__ void __launch_bounds__(256) rope_pool_cube_kernel(Shape s, const T* _
                                                              T* __restrict__ kr, T* __restrict__ vp,
                                                              float* __restrict__ qbar, float* __restrict__ kbar)
 {
-    __shared__ float part[16][kDh];
+    __shared__ __align__(16) float rot[kBlock][kDh];      // fp32 rotated rows, slot order
     const int blk = blockIdx.x, bh = blockIdx.y, z = blockIdx.z;
     const T* x = z == 0 ? q : (z == 1 ? k : v);
     T* xr = z == 0 ? qr : (z == 1 ? kr : vp);
@@ -193,7 +205,6 @@ __global__ void __launch_bounds__(256) rope_pool_cube_kernel(Shape s, const T* _
         axis[p] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
     }
     const int xx = o.x + (rsub >> 2), yy = o.y + (rsub & 3);
-    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 #pragma unroll
     for (int dt = 0; dt < kPasses; ++dt) {
         const int slot = rsub + 16 * dt;
@@ -213,22 +224,21 @@ __global__ void __launch_bounds__(256) rope_pool_cube_kernel(Shape s, const T* _
                     out[2 * p] = y.x;
                     out[2 * p + 1] = y.y;
                 }
-#pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i] += out[i];
             }
         }
         Vec8<T>::store(xr + ((size_t)bh * s.Np + (size_t)blk * kBlock + slot) * kDh + c8 * 8, out);
+        if (z != 2) {
+            float4* dst = reinterpret_cast<float4*>(&rot[slot][c8 * 8]);
+            dst[0] = make_float4(out[0], out[1], out[2], out[3]);
+            dst[1] = make_float4(out[4], out[5], out[6], out[7]);
+        }
     }
     if (z == 2) return;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) part[rsub][c8 * 8 + i] = acc[i];
     __syncthreads();
     if (threadIdx.x < kDh) {
-        float sum = 0.0f;
-#pragma unroll
-        for (int r = 0; r < 16; ++r) sum += part[r][threadIdx.x];
         const int cnt = min(4, s.T - o.t) * min(4, s.Hh - o.x) * min(4, s.Ww - o.y);
-        (z == 0 ? qbar : kbar)[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = sum / (float)cnt;
+        (z == 0 ? qbar : kbar)[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] =
+            pairwise64(&rot[0][threadIdx.x], kDh) / (float)cnt;
     }
 }
 

@@ -95,8 +95,7 @@ def test_forward(rl, act, dname, tdt):
     torch.cuda.synchronize()
     assert rl.get_device_status(ws) == rl.ROLA_OK
     res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], mask_override=kv.cpu().numpy())
-    idx, scores, gap, tau = O.block_mask(cfg, h["q"], h["k"])
-    check_mask(kv.cpu().numpy(), idx, scores, gap, tau, nB)
+    check_mask(cfg, h, kv.cpu().numpy(), f"forward {act} {dname}")
     assert_close(to_np(out), res["o"], dname == "bf16", f"O[forward,{act},{dname}]")
 
 

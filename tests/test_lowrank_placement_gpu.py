@@ -96,8 +96,7 @@ def test_forward(rl, mode, dname, tdt):
     # the GPU's mask (the mask does not depend on the low-rank placement) is handed to the oracle
     res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], mask_override=kv.cpu().numpy(),
                     rope_mode=o_mode)
-    idx, scores, gap, tau = O.block_mask(cfg, h["q"], h["k"])
-    check_mask(kv.cpu().numpy(), idx, scores, gap, tau, nB)
+    check_mask(cfg, h, kv.cpu().numpy(), f"forward {mode} {dname}")
     assert_close(to_np(out), res["o"], dname == "bf16", f"O[forward,{mode},{dname}]")
 
 

@@ -73,6 +73,14 @@ MUTATIONS = {
                                   "dP[(size_t)a * dh + d] += du[a] * (double)x[(d + 1) % dh];"),
     "bwd_key_grad_operand": ("dkr[(size_t)j * dh + d] += dsv * qp[d];", "dkr[(size_t)j * dh + d] += dsv * kq[d];"),
     "bwd_gate_grad_rms": ("dg_bh[(size_t)bh * N + p] = rp * a;", "dg_bh[(size_t)bh * N + p] = a;"),
+    "f32_pool_sequential": ("return pairwise_f32(x, n / 2) + pairwise_f32(x + n / 2, n - n / 2);",
+                            "return x[0] + pairwise_f32(x + 1, n - 1);"),
+    "f32_rotation_sign": ("yr[2 * m] = fmaf(x0, cm, -p1);", "yr[2 * m] = fmaf(x0, cm, p1);"),
+    "f32_pool_divisor": ("pairwise_f32(vals, slots) / (float)cnt;", "pairwise_f32(vals, slots) / (float)slots;"),
+    "f32_tie_order": ("return (x->j > y->j) - (x->j < y->j);", "return (x->j < y->j) - (x->j > y->j);"),
+    "f32_scale_dropped": ("row[j].s = acc * scale;", "row[j].s = acc;"),
+    "f32_cube_slot_order": ("x = CUBE * cx + (i / CUBE) % CUBE, y = CUBE * cy + i % CUBE;",
+                            "x = CUBE * cx + i % CUBE, y = CUBE * cy + (i / CUBE) % CUBE;"),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 
@@ -85,7 +93,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     mutated = tmp_path / "mut.c"
     mutated.write_text(src.replace(old, new))
     lib = tmp_path / "libmut.so"
-    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c99", "-o", str(lib),
+    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c99", "-ffp-contract=off", "-o", str(lib),
                            str(mutated), "-lm"])
     env = dict(os.environ, ORACLE_LIB=str(lib), OMP_NUM_THREADS="4")
     res = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",

@@ -140,54 +140,99 @@ def test_mask_is_the_best_subset_by_brute_force(oracle):
             assert gap[0, h, i] == pytest.approx(srt[nk - 1] - srt[nk], abs=1e-15)
 
 
-def fp32_block_scores(O, cfg, x, order, dot):
-    """Block scores evaluated in fp32 arithmetic: the rotated rows rounded to fp32, each block's sum
-    accumulated in fp32 (ascending, descending or numpy's pairwise order), the fp32 mean, and fp32 dot
-    products (sequential over d_h or a float32 matmul), scaled by fp32 1/sqrt(d_h)."""
-    qr = O.rope_full(cfg, x["q"]).astype(np.float32)[0]
-    kr = O.rope_full(cfg, x["k"]).astype(np.float32)[0]
-    H, N = cfg["H"], cfg["N"]
-    nb = -(-N // 64)
-
-    def pooled(xr):
-        out = np.zeros((H, nb, 128), np.float32)
-        for b in range(nb):
-            rows = xr[:, b * 64:min(N, (b + 1) * 64)]
-            if order == "pairwise":
-                acc = rows.sum(axis=1, dtype=np.float32)
-            else:
-                seq = rows if order == "ascending" else rows[:, ::-1]
-                acc = np.zeros((H, 128), np.float32)
-                for t in range(seq.shape[1]):
-                    acc = acc + seq[:, t]
-            out[:, b] = acc / np.float32(rows.shape[1])
-        return out
-
-    qb, kb = pooled(qr), pooled(kr)
-    if dot == "sequential":
-        s = np.zeros((H, nb, nb), np.float32)
-        for d in range(128):
-            s = s + qb[:, :, None, d] * kb[:, None, :, d]
-    else:
-        s = np.matmul(qb, kb.transpose(0, 2, 1))
-    return s * np.float32(1.0 / math.sqrt(128))
+def wide_range(cfg, seed):
+    """q, k with per-token magnitudes spread over six decades (10^-3 .. 10^3): pooled sums that
+    cancel and round, the hard case for the fp32 evaluation of the block scores."""
+    rng = np.random.default_rng(seed)
+    shape = (cfg["B"], cfg["H"], cfg["N"], 128)
+    scale = 10.0 ** rng.uniform(-3, 3, size=shape[:3] + (1,))
+    return {n: (rng.standard_normal(shape) * scale).astype(np.float32) for n in ("q", "k")}
 
 
-@pytest.mark.parametrize("dist", ["normal", "rmsnorm"])
-def test_near_tie_bound_covers_fp32_scores(oracle, dist):
-    """The near-tie rule (reading 12) rests on tau / 8 bounding how far an fp32 evaluation of a score
-    row can sit from the fp64 one: checked for fp32 evaluations in six summation orders.  The bound
-    must also stay meaningful: below 1e-3 of the largest score."""
+@pytest.mark.parametrize("geometry", ["flat", "cube"])
+@pytest.mark.parametrize("dist", ["normal", "rmsnorm", "wide"])
+def test_fp32_decision_within_the_near_tie_bound(oracle, dist, geometry):
+    """The block mask is an fp32 decision (reading 11).  tau / 2 is a rigorous bound on how far the
+    oracle's fp32 evaluation of a score sits from the fp64 one (first-order error analysis of the
+    rotation, the pairwise pooling, the division, the fma chain and the scale); checked at every
+    (i, j) on three input distributions and both block geometries.  Rows with gap > tau then keep the
+    same blocks in fp32 and in fp64.  The bound stays meaningful: below 1e-3 of the largest score."""
     O = oracle
-    cfg = small_cfg(T=4, Hh=9, Ww=10, dist=dist)             # 360 tokens: 6 blocks, the last of 40
-    x = draw(cfg)
-    _, s64, _, tau = O.block_mask(cfg, x["q"], x["k"])
-    bound = tau[0] / 8
+    cfg = small_cfg(T=4, Hh=9, Ww=10, dist="rmsnorm" if dist == "rmsnorm" else "normal",
+                    block_geometry=geometry)            # 360 tokens: 6 ragged chunks / 6 ragged cubes
+    x = wide_range(cfg, 5) if dist == "wide" else draw(cfg)
+    idx, s64, gap, tau = O.block_mask(cfg, x["q"], x["k"])
+    idx32, s32 = O.block_mask_f32(cfg, x["q"], x["k"])
+    bound = tau / 2
     assert (bound > 0).all() and bound.max() <= 1e-3 * np.abs(s64).max()
-    for order in ("ascending", "descending", "pairwise"):
-        for dot in ("sequential", "matmul"):
-            err = np.abs(fp32_block_scores(O, cfg, x, order, dot).astype(np.float64) - s64[0])
-            assert (err <= bound[:, :, None]).all(), (order, dot, float((err / bound[:, :, None]).max()))
+    err = np.abs(s32 - s64)
+    assert (err <= bound[..., None]).all(), float((err / bound[..., None]).max())
+    assert (err > 0).any()                              # fp32 really rounds here
+    far = gap > tau
+    assert far.any() and (idx32[far] == idx[far]).all()
+
+
+def test_fp32_pooling_is_pairwise_in_slot_order(oracle):
+    """The fp32 block mean is the pairwise sum (Higham, Accuracy and Stability of Numerical Algorithms,
+    Sec. 4.2) of the block's slots in slot order, divided once by the token count; closed forms where
+    the order decides the rounding.  Coordinate 0 of pair 0 (temporal, angle t = 0 in the first frame)
+    is not rotated and every other coordinate is 0; the key block's mean in coordinate 0 is 1 (chunks)
+    or 1/4 (cubes), so the score is the fp32 product of the pooled query value, that mean and
+    fl(1/sqrt(128))."""
+    O = oracle
+    scale = np.float32(1.0 / math.sqrt(128.0))
+    # chunks: 64 tokens of frame 0, token 0 holds 2^24 and tokens 1..63 hold 1.  Pairwise: the first
+    # pair rounds 2^24 + 1 to 2^24 (ties to even) and every later level is exact, 2^24 + 62; the
+    # sequential sum would lose all 63 ones and the exact sum is 2^24 + 63.
+    cfg = small_cfg(T=2, Hh=8, Ww=8, H=1, keep=0.5)
+    q = np.zeros((1, 1, cfg["N"], 128), np.float32)
+    k = np.zeros_like(q)
+    q[0, 0, :64, 0] = 1.0
+    q[0, 0, 0, 0] = 2.0 ** 24
+    k[0, 0, :, 0] = 1.0
+    _, s32 = O.block_mask_f32(cfg, q, k)
+    assert s32[0, 0, 0, 0] == np.float32(np.float32(2.0 ** 24 + 62) / np.float32(64)) * scale
+    assert s32[0, 0, 0, 0] == np.float32(262144.96875) * scale
+    assert np.float32(262144.0) * scale != np.float32(262144.96875) * scale
+    # cubes: a 4 x 4 x 8 grid holds two cubes; in cube 0, (dx, dy) = (0, 0) holds 2^24, (0, 1) holds 1,
+    # (1, 0) holds 2 (frame 0).  Slot 16 dt + 4 dx + dy: the pair (slot 0, slot 1) rounds 2^24 + 1 to
+    # 2^24, the 2 joins at the third level exactly: 2^24 + 2.  With dx and dy swapped in the slot
+    # number the pair would hold 2^24 + 2 and the 1 would round the total to 2^24 + 4.
+    cfg = small_cfg(T=4, Hh=4, Ww=8, H=1, keep=0.5, block_geometry="cube")
+    q = np.zeros((1, 1, cfg["N"], 128), np.float32)
+    k = np.zeros_like(q)
+    tok = lambda t, xx, y: (t * 4 + xx) * 8 + y
+    q[0, 0, tok(0, 0, 0), 0] = 2.0 ** 24
+    q[0, 0, tok(0, 0, 1), 0] = 1.0
+    q[0, 0, tok(0, 1, 0), 0] = 2.0
+    for xx in range(4):
+        for y in range(4):
+            k[0, 0, tok(0, xx, y), 0] = 1.0        # cube 0's key mean in coordinate 0: 16 / 64 = 1/4 exactly
+    _, s32 = O.block_mask_f32(cfg, q, k)
+    assert s32[0, 0, 0, 0] == np.float32(262144.03125 / 4) * scale     # (2^24 + 2) / 64, times 1/4
+    assert np.float32(262144.0625 / 4) * scale != np.float32(262144.03125 / 4) * scale
+
+
+def test_fp32_decision_ties_and_brute_force(oracle):
+    """The fp32 decision keeps, per row, the n_keep-subset with the largest fp32 score sum (brute
+    force over all subsets on the tiny layer, whose fp32 scores are distinct), and breaks an exact
+    tie toward the lower block: an all-zero query row keeps block 0."""
+    O = oracle
+    cfg = configs.get("tiny")
+    x = draw(cfg)
+    idx32, s32 = O.block_mask_f32(cfg, x["q"], x["k"])
+    nb, nk = s32.shape[-1], idx32.shape[-1]
+    for h in range(cfg["H"]):
+        for i in range(nb):
+            s = s32[0, h, i]
+            assert len(set(s.tolist())) == nb
+            best = max(itertools.combinations(range(nb), nk), key=lambda S: sum(s[list(S)]))
+            assert list(best) == list(idx32[0, h, i])
+    cfg = small_cfg(keep=0.5)                               # two blocks, n_keep = 1
+    q = np.zeros((1, cfg["H"], cfg["N"], 128), np.float32)
+    k = draw(cfg)["k"]
+    idx32, s32 = O.block_mask_f32(cfg, q, k)
+    assert (s32 == 0).all() and (idx32 == 0).all()
 
 
 def test_mask_closed_form_single_token(oracle):
