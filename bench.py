@@ -34,11 +34,32 @@ sys.path.insert(0, ROOT)
 METRIC = "RoLA attn layer ms & tokens/s (Wan2.1-14B 720p shape); % of TC/HBM roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the current sparse
-# kernel from one ncu capture of the 480p layer (12 heads x 32760 tokens), scaled
-# to a launch by heads x tokens (the traffic is the streaming q^r, k^r, v reads and
-# the O^s write, which grow in proportion).  Set to None whenever the kernel changes.
-SPARSE_TRAFFIC_PER_HEAD_TOKEN = (303.265280e6 + 86.776064e6) / (12 * 32760)
+# The ncu summary that carries the sparse kernel's DRAM traffic per (head, token), and
+# the sources its capture was taken on.
+SPARSE_PROFILE = os.path.join(ROOT, "profiles", "sparse_attn_tc_wan13b_480p.md")
+SPARSE_SOURCES = ["sparse_attn_tc.cu", "common.cuh", "tcgen05.cuh", "tensor_map.cuh"]
+
+
+def sparse_traffic_per_head_token():
+    """dram__bytes_read.sum + dram__bytes_write.sum of the sparse kernel per (head, token),
+    from the committed ncu summary, or None when the kernel's sources have changed since
+    that capture (their sha256 no longer matches the one the summary records)."""
+    import hashlib
+    try:
+        text = open(SPARSE_PROFILE).read()
+    except OSError:
+        return None
+    fields = dict(line.split(": ", 1) for line in text.splitlines()
+                  if line.startswith(("traffic_bytes_per_head_token: ", "kernel_sources_sha256: ")))
+    if len(fields) != 2:
+        return None
+    h = hashlib.sha256()
+    for f in SPARSE_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_06712_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest() != fields["kernel_sources_sha256"].strip():
+        return None
+    return float(fields["traffic_bytes_per_head_token"])
 
 
 def load_peaks():
@@ -329,6 +350,14 @@ def run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank):
         "apply": (lambda: rola.lowrank_apply(c, x["q"], x["P_q"], C, x["gate"], o, o, wsb), 3 * tensor_bytes,
                   "read q, O^s; write O"),
     }
+    if args.entry == "out_proj":
+        d_model = cfg["H"] * 128
+        wo = (torch.randn((d_model, d_model), device=o.device) / d_model ** 0.5).to(torch.bfloat16)
+        bo = 0.1 * torch.randn((d_model,), device=o.device)
+        ybuf = torch.empty((cfg["B"], cfg["N"], d_model), dtype=torch.bfloat16, device=o.device)
+        calls["out_proj"] = (lambda: rola.out_proj(c, o, wo, bo, ybuf, wsb),
+                             tensor_bytes + 2.0 * d_model * d_model + 2.0 * cfg["B"] * cfg["N"] * d_model,
+                             "Y = concat_h(O) W_o^T + b_o (tcgen05 GEMM): read O, W_o; write Y")
     fn, nbytes, what = calls[args.entry]
     for _ in range(args.warmup):
         fn()
@@ -346,8 +375,15 @@ def run_entry(args, cfg, c, x, o, kv, wsb, stream, ws, rank):
         peaks, src = load_peaks()
         hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
         names = {"mask": "rola_block_mask", "summary": "rola_lowrank_summary", "sparse": "rola_sparse_attn",
-                 "apply": "rola_lowrank_apply"}
+                 "apply": "rola_lowrank_apply", "out_proj": "rola_out_proj"}
+        extra = {}
+        if args.entry == "out_proj":
+            fl = 2.0 * cfg["B"] * cfg["N"] * (cfg["H"] * 128) ** 2
+            bf16_peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+            extra = {"flops_per_call": fl, "achieved_tflops": fl / (ms * 1e-3) / 1e12, "bf16_peak_tflops": bf16_peak,
+                     "frac_of_burst": fl / (ms * 1e-3) / 1e12 / bf16_peak}
         print(json.dumps({"entry": names[args.entry], "ms_per_call": ms, "unit": "ms", "steps": args.steps, "warmup": args.warmup,
+                          **extra,
                           "bytes_per_call": nbytes, "achieved_gbs": nbytes / (ms * 1e-3) / 1e9, "hbm_peak_gbs": hbm,
                           "note": what, "config": {"workload": cfg["name"], "H": cfg["H"], "N": cfg["N"],
                                                    "r": cfg["r"], "keep": cfg["keep"]}}), flush=True)
@@ -369,7 +405,7 @@ def main():
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--entry", default="forward", choices=["forward", "mask", "summary", "sparse", "apply",
+    ap.add_argument("--entry", default="forward", choices=["forward", "mask", "summary", "sparse", "apply", "out_proj",
                                                            "backward"],
                     help="time one per-stage entry point alone instead of the layer")
     args = ap.parse_args()
@@ -460,13 +496,18 @@ def main():
     fl = sparse_flops_from_mask(kv, block_sizes(cfg))
     sp_ms = stage_ms["sparse_attn"]
     achieved = fl / (sp_ms * 1e-3) / 1e12
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-    traffic = None
-    if SPARSE_TRAFFIC_PER_HEAD_TOKEN is not None and geometry == "flat":
-        traffic = SPARSE_TRAFFIC_PER_HEAD_TOKEN * cfg["B"] * cfg["H"] * cfg["N"]
+    # burst peak: the timed region is well under a second and ran at full SM clock (the
+    # sustained figure was measured over 4 s under the power cap, at a lower clock)
+    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    tph = sparse_traffic_per_head_token() if geometry == "flat" else None
+    traffic = None if tph is None else tph * cfg["B"] * cfg["H"] * cfg["N"]
     roofline = {"bound": "tensor", "kernel": "sparse_attn", "achieved": achieved, "peak": peak,
                 "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
-                "peak_source": f"{peak_src} bf16_tflops_sustained",
+                "peak_source": f"{peak_src} bf16_tflops (burst: sub-second timed region at full clock)",
+                "frac_of_sustained": achieved / peak_sus,
+                "traffic_source": (None if traffic is None else
+                                   "profiles/sparse_attn_tc_wan13b_480p.md, per (head, token) x B*H*N"),
                 "algorithmic_flops_per_launch": fl, "ms_per_launch": sp_ms}
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     tensor_bytes = summary_bytes(cfg["B"], cfg["H"], cfg["N"], 128) / 2      # one [B,H,N,128] bf16 tensor
@@ -514,6 +555,30 @@ def main():
                          "frac": gate_bytes / (gate_ms * 1e-3) / 1e9 / hbm,
                          "note": f"X [B][N][{d_model}] bf16 read once ({xg['X'].numel() * 2 / 1e6:.0f} MB)"}
     del xg, gbuf
+
+    # ---- the output projection Y = concat_h(O) W_o^T + b_o on the layer's output o (the block's
+    # last step; a tcgen05 GEMM, B*N x d_model x H*128), timed on its own
+    wo = (torch.randn((d_model, d_model), device=dev) / d_model ** 0.5).to(torch.bfloat16)
+    bo = 0.1 * torch.randn((d_model,), device=dev)
+    ybuf = torch.empty((cfg["B"], cfg["N"], d_model), dtype=torch.bfloat16, device=dev)
+    for _ in range(3):
+        rola.out_proj(c, o, wo, bo, ybuf, wsb)
+    torch.cuda.synchronize()
+    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for _ in range(10):
+        rola.out_proj(c, o, wo, bo, ybuf, wsb)
+    p1.record(stream)
+    torch.cuda.synchronize()
+    assert rola.get_device_status(wsb) == rola.ROLA_OK
+    proj_ms = p0.elapsed_time(p1) / 10
+    proj_flops = 2.0 * cfg["B"] * cfg["N"] * d_model * d_model
+    secondary["out_proj"] = {"bound": "tensor", "ms": proj_ms, "flops": proj_flops,
+                             "achieved_tflops": proj_flops / (proj_ms * 1e-3) / 1e12, "peak_tflops": peak,
+                             "frac": proj_flops / (proj_ms * 1e-3) / 1e12 / peak,
+                             "note": f"Y [B][N][{d_model}] = concat_h(O) W_o^T + b_o, bf16 in/out, fp32 accumulation; "
+                                     "peak = measured bf16 burst"}
+    del wo, bo, ybuf
 
     # ---- end to end through the public API with host buffers
     # Every step copies its inputs from pinned host memory and reads its output

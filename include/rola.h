@@ -93,9 +93,9 @@ typedef struct {
     int32_t wait_limit_ms;     /* bound of every device-side wait (0 = 2000 ms); at most 60000 */
     int32_t debug_flags;       /* 0 normally.  ROLA_DEBUG_SKIP_FIRST_K_COPY makes each CTA of the
                                   bf16 sparse kernel skip its first K copy (of the bf16 backward
-                                  kernels: the first K pair, the first Q / dO pair), so a bounded
-                                  wait runs out and the call reports ROLA_ERR_TIMEOUT (tests the
-                                  timeout path) */
+                                  kernels: the first K pair, the first Q / dO pair; of the bf16
+                                  pre-pass: its first k, v, q load), so a bounded wait runs out
+                                  and the call reports ROLA_ERR_TIMEOUT (tests the timeout path) */
     int32_t lowrank_rope;      /* where the truncated RoPE sits in the low-rank features; one of
                                   rola_lowrank_rope_t, default ROLA_LOWRANK_ROPE_OUTSIDE */
     int32_t lowrank_act;       /* feature map phi of the low-rank features; one of
@@ -314,6 +314,48 @@ rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g
                         int32_t d_model, float* gate, void* stream);
 
 /*
+ * Output projection of the attention block (Alg. 1, last step, "merge heads,
+ * output projection"): per token the heads' fused outputs are concatenated,
+ * head-major, and multiplied by W_o:
+ *   Y[b][n][f] = sum_{h,d} O[b][h][n][d] * W_o[f][128 h + d]  (+ b_o[f])
+ *   O    : [B][H][N][128], cfg->dtype -- the output of rola_forward, read in
+ *          place (the concatenation is the GEMM's K index, no copy is made)
+ *   W_o  : [d_model][H*128], cfg->dtype (row f = output feature f, the
+ *          nn.Linear weight layout)
+ *   b_o  : [d_model] fp32, or NULL for no bias
+ *   Y    : out, [B][N][d_model], cfg->dtype, caller-allocated
+ *   ws   : at least 256 bytes, 256-byte aligned (the module's workspace will
+ *          do); only its status word is used: cleared, then set to
+ *          ROLA_ERR_TIMEOUT if a bounded device wait expires
+ * d_model must be a positive multiple of 64; O, W_o, Y (and b_o) 16-byte
+ * aligned.  bf16: tcgen05 tensor-core GEMM with fp32 accumulation in TMEM, one
+ * bf16 rounding of each output; fp32: plain fp32 arithmetic (validation).
+ * Uses cfg->B, H, N, dtype and wait_limit_ms.
+ */
+rola_status_t rola_out_proj(const rola_config_t* cfg, const void* O, const void* W_o, const float* b_o,
+                            int32_t d_model, void* Y, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * The attention block after the QKV projection and the pre-RoPE norms
+ * (Alg. 1 from the gate on): the token gate from the block input X
+ * (rola_gate), the RoLA module on q, k, v (rola_forward, with that gate), and
+ * the output projection (rola_out_proj), in this order on `stream`.
+ *   X, w_g, b_g, d_model : as rola_gate (d_model also the width of Y and W_o)
+ *   q, k, v, P_q, P_k    : as rola_forward
+ *   W_o, b_o             : as rola_out_proj
+ *   gate : out, fp32 [B][N], the gate values (caller-owned scratch)
+ *   o    : out, [B][H][N][128], the module's per-head output
+ *   Y    : out, [B][N][d_model]
+ *   kv_idx_out : nullable, as rola_forward
+ *   ws   : rola_workspace_bytes(cfg) bytes; rola_get_device_status(ws)
+ *          afterwards covers the module and the projection
+ */
+rola_status_t rola_attention_block(const rola_config_t* cfg, const void* X, const void* w_g, float b_g,
+                                   int32_t d_model, const void* q, const void* k, const void* v, const void* P_q,
+                                   const void* P_k, const void* W_o, const float* b_o, float* gate, void* o, void* Y,
+                                   int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
  * rola_lowrank_summary_static: the low-rank summary (C and optionally z, as
  * rola_lowrank_summary computes them) for callers that cannot give the
  * library any device scratch -- e.g. a plugin whose host framework owns the
@@ -329,11 +371,17 @@ rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g
  * array, so calls whose executions overlap on the GPU (other streams, other
  * host threads) race and must be serialised by the caller.
  *   k, v, P_k, C, z : as rola_lowrank_summary (device pointers, caller-owned)
- * Returns ROLA_ERR_UNSUPPORTED when the layer's scratch (table plus one
- * partial per head, 4*(r*d_h + r) bytes per head) exceeds the 16 MiB array,
- * and the usual validation codes otherwise.  When the array cannot hold the
+ * Returns ROLA_ERR_UNSUPPORTED when the layer's least scratch exceeds the
+ * 16 MiB array: a 256-byte status word, the RoPE table of
+ * (T + Hh + Ww) * 64 * 8 bytes rounded up to 256, and one partial slot per
+ * head, B*H*4*(rp*128 + rp) bytes with rp = r rounded up to a multiple of 16;
+ * the usual validation codes otherwise.  When the array cannot hold the
  * regular number of splits it uses fewer, so C may differ from
  * rola_lowrank_summary's in the last bits (same fixed-order sum, coarser split).
+ * There is no status word for the caller to read: if a bounded device wait
+ * of the bf16 kernel gives up (cfg->wait_limit_ms), C and z come back filled
+ * with NaN.  ROLA_DEBUG_SKIP_FIRST_K_COPY makes every CTA of that kernel skip
+ * its first load, so its waits run out (tests this path).
  */
 rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, const void* k, const void* v,
                                           const void* P_k, float* C, float* z, void* stream);

@@ -95,6 +95,7 @@ def _get():
             lib.orc_sparse_attn.argtypes = [cfgp, P, P, P, P, ctypes.c_int, P, P]
             lib.orc_forward.argtypes = [cfgp, P, P, P, P, P, P, P, P, P, P, P, P, P]
             lib.orc_gate.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, ctypes.c_double, P]
+            lib.orc_out_proj.argtypes = [ctypes.c_int] * 5 + [P] * 5
             _lib = lib
     return _lib
 
@@ -287,6 +288,25 @@ def gate(X, w, b: float) -> np.ndarray:
     g = np.empty((B, N))
     _get().orc_gate(B, N, D, Xp, wp, float(b), g.ctypes.data)
     return g
+
+
+def out_proj(O, W, bias=None, rows=None) -> np.ndarray:
+    """Output projection of the block (Alg. 1, last step): the heads of O [B][H][N][dh] concatenated
+    per token (head-major), times W^T, W [d_model][H*dh] (+ bias [d_model]) -> Y [B][N][d_model].
+    ``rows``: token indices to compute (the other rows are NaN); None computes every token."""
+    O = np.ascontiguousarray(O, dtype=np.float64)
+    W, Wp = _f32(W)
+    B, H, N, dh = O.shape
+    d_model = W.shape[0]
+    assert W.shape == (d_model, H * dh)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    sel = None
+    if rows is not None:
+        sel = np.zeros(N, dtype=np.uint8)
+        sel[np.asarray(rows, dtype=np.int64)] = 1
+    Y = np.full((B, N, d_model), np.nan)
+    _get().orc_out_proj(B, N, H, dh, d_model, O.ctypes.data, Wp, _ptr(b), _ptr(sel), Y.ctypes.data)
+    return Y
 
 
 def lowrank_explicit(cfg: dict, q, k, v, Pq, Pk, rope_mode: int = ROPE_OUTSIDE) -> np.ndarray:

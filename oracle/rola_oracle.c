@@ -1112,3 +1112,30 @@ void orc_gate(int B, int N, int D, const float* X, const float* w, double b, dou
         g[p] = 1.0 / (1.0 + exp(-logit));
     }
 }
+
+/* Output projection (Alg. 1, last step, "merge heads, output projection"):
+ * the heads' fused outputs are concatenated per token, o_cat[n] =
+ * (O^fused_1[n], ..., O^fused_H[n]) (length H * dh, head-major), and
+ * Y[b][n][f] = sum_k o_cat[n][k] W[f][k] (+ bias[f]).  O is [B][H][N][dh]
+ * (double), W [d_model][H * dh] (the row of output feature f), bias
+ * [d_model] or NULL, Y [B][N][d_model].  Only the tokens with rows[n] != 0
+ * are computed (rows NULL: all); the others are left untouched. */
+void orc_out_proj(int B, int N, int H, int dh, int d_model, const double* O, const float* W, const float* bias,
+                  const uint8_t* rows, double* Y)
+{
+    int K = H * dh;
+#pragma omp parallel for schedule(dynamic, 16)
+    for (long p = 0; p < (long)B * N; ++p) {
+        int b = (int)(p / N), n = (int)(p % N);
+        if (rows && !rows[n]) continue;
+        double* cat = (double*)malloc(sizeof(double) * (size_t)K);
+        for (int h = 0; h < H; ++h)
+            for (int d = 0; d < dh; ++d) cat[h * dh + d] = O[(((size_t)b * H + h) * N + n) * dh + d];
+        for (int f = 0; f < d_model; ++f) {
+            double y = bias ? (double)bias[f] : 0.0;
+            for (int k = 0; k < K; ++k) y += cat[k] * (double)W[(size_t)f * K + k];
+            Y[(size_t)p * d_model + f] = y;
+        }
+        free(cat);
+    }
+}

@@ -8,6 +8,12 @@ using namespace rola;
 
 namespace rola {
 
+// The output projection (out_proj.cu).
+cudaError_t launch_out_proj(int B, int N, int H, int d_model, const void* O, const void* W, const float* bias,
+                            void* Y, DeviceStatus* status, uint64_t wait_limit_ns, cudaStream_t st);
+cudaError_t launch_out_proj_f32(int B, int N, int H, int d_model, const float* O, const float* W, const float* bias,
+                                float* Y, cudaStream_t st);
+
 int num_blocks_of(const rola_config_t& c)
 {
     if (c.block_geometry == ROLA_BLOCK_CUBE)
@@ -322,6 +328,28 @@ rola_status_t forward_impl(const rola_config_t* cfg, const void* q, const void* 
 }
 
 
+// Y = concat_h(O) W_o^T (+ b_o); `clear` clears the status word first (every entry point
+// does; the block entry point keeps the forward's).
+rola_status_t out_proj_impl(const rola_config_t* cfg, const void* O, const void* W_o, const float* b_o,
+                            int32_t d_model, void* Y, void* ws, size_t ws_bytes, cudaStream_t st, bool clear)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!O || !W_o || !Y || d_model < 64 || d_model % 64 != 0) return ROLA_ERR_INVALID_ARG;
+    if (!aligned16(O) || !aligned16(W_o) || !aligned16(Y) || (b_o && !aligned16(b_o))) return ROLA_ERR_INVALID_ARG;
+    if ((int64_t)cfg->B * cfg->N * d_model > ((int64_t)1 << 40)) return ROLA_ERR_UNSUPPORTED;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) || ws_bytes < sizeof(DeviceStatus))
+        return ROLA_ERR_WORKSPACE;
+    if (clear) ROLA_TRY(cudaMemsetAsync(ws, 0, sizeof(DeviceStatus), st));
+    const Shape s = make_shape(*cfg);
+    if (cfg->dtype == ROLA_BF16)
+        ROLA_TRY(launch_out_proj(cfg->B, cfg->N, cfg->H, d_model, O, W_o, b_o, Y, static_cast<DeviceStatus*>(ws),
+                                 s.wait_limit_ns, st));
+    else
+        ROLA_TRY(launch_out_proj_f32(cfg->B, cfg->N, cfg->H, d_model, static_cast<const float*>(O),
+                                     static_cast<const float*>(W_o), b_o, static_cast<float*>(Y), st));
+    return ROLA_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -509,6 +537,26 @@ rola_status_t rola_gate(const rola_config_t* cfg, const void* X, const void* w_g
     ROLA_TRY(launch_gate(cfg->dtype, (long long)cfg->B * cfg->N, d_model, X, w_g, b_g, gate,
                          static_cast<cudaStream_t>(stream)));
     return ROLA_OK;
+}
+
+rola_status_t rola_out_proj(const rola_config_t* cfg, const void* O, const void* W_o, const float* b_o,
+                            int32_t d_model, void* Y, void* ws, size_t ws_bytes, void* stream)
+{
+    return out_proj_impl(cfg, O, W_o, b_o, d_model, Y, ws, ws_bytes, static_cast<cudaStream_t>(stream), true);
+}
+
+rola_status_t rola_attention_block(const rola_config_t* cfg, const void* X, const void* w_g, float b_g,
+                                   int32_t d_model, const void* q, const void* k, const void* v, const void* P_q,
+                                   const void* P_k, const void* W_o, const float* b_o, float* gate, void* o, void* Y,
+                                   int32_t* kv_idx_out, void* ws, size_t ws_bytes, void* stream)
+{
+    ROLA_CHECK(validate(cfg));
+    if (!gate || !o) return ROLA_ERR_INVALID_ARG;
+    ROLA_CHECK(check_ws(*cfg, ws, ws_bytes));
+    ROLA_CHECK(rola_gate(cfg, X, w_g, b_g, d_model, gate, stream));
+    ROLA_CHECK(rola_forward(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, ws_bytes, stream));
+    // the projection records into the status word the forward cleared, without clearing it again
+    return out_proj_impl(cfg, o, W_o, b_o, d_model, Y, ws, ws_bytes, static_cast<cudaStream_t>(stream), false);
 }
 
 rola_status_t rola_get_device_status(const void* ws, void* stream)

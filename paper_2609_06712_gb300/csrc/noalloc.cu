@@ -16,12 +16,13 @@
 //
 // Every call shares the one array and it keeps the last call's contents.
 // Everything a call reads from it, the call has written first (the status
-// word is cleared, the table and every partial are overwritten in full).  A
-// device-side wait that gives up (bf16 kernel, bounded waits) is recorded in
-// that status word only; no call reports it.  Calls
-// whose executions overlap on the GPU -- on different streams, or from
-// different host threads -- race on the array and must be serialised by the
-// caller.
+// word is cleared, the table and every partial are overwritten in full) --
+// except when a bounded device wait of the bf16 kernel gives up: that kernel
+// then stops without writing its partials, so the call's last kernel, seeing
+// the status word set, overwrites C and z with NaN (the caller has no
+// workspace whose status it could read).  Calls whose executions overlap on
+// the GPU -- on different streams, or from different host threads -- race on
+// the array and must be serialised by the caller.
 #include <mutex>
 
 #include "common.cuh"
@@ -56,6 +57,18 @@ cudaError_t scratch_address(void** out)
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// After the combine: if a wait of the pre-pass gave up, C and z hold sums of stale
+// partials, so they become NaN.  Nothing is written when the status word is clear.
+__global__ void poison_on_timeout_kernel(const DeviceStatus* status, float* C, int nC, float* z, int nz)
+{
+    if (status->code == 0) return;
+    const float nan = __int_as_float(0x7fc00000);
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nC + nz; i += gridDim.x * blockDim.x) {
+        if (i < nC) C[i] = nan;
+        else if (z) z[i - nC] = nan;
+    }
+}
 
 }  // namespace
 }  // namespace rola
@@ -96,6 +109,10 @@ extern "C" rola_status_t rola_lowrank_summary_static(const rola_config_t* cfg, c
                            cs) != cudaSuccess ||
             launch_prepass_combine(s, ctas, partials, C, z, nullptr, cs) != cudaSuccess)
             return ROLA_ERR_CUDA;
+        const int nC = (int)(bh * (size_t)s.r * kDh), nz = z ? (int)(bh * (size_t)s.r) : 0;
+        poison_on_timeout_kernel<<<(nC + nz + 255) / 256 < 1024 ? (nC + nz + 255) / 256 : 1024, 256, 0, cs>>>(
+            status, C, nC, z, nz);
+        if (cudaGetLastError() != cudaSuccess) return ROLA_ERR_CUDA;
     } else {
         int nsplit = summary_splits(s);
         if ((size_t)nsplit > fit / bh) nsplit = (int)(fit / bh);

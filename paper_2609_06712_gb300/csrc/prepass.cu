@@ -18,18 +18,17 @@
 // (k, v and q boxes of 32 x 128, 8 KB each), which keeps a CTA small enough
 // that two fit on an SM for r <= 48 (16 warps per SM hide the latency of the
 // dependent MMA and rotation chains).  Per half, 8 warps:
-//   rotate q, k (thread = two neighbouring token rows x 8 coordinates), store
-//   q^r, k^r, pool; U = K P_k^T (mma.sync; warp = 16 tokens x a quarter or
-//   half of the r columns); k~ = R_r SiLU(U) to shared memory; the half's
+//   rotate q, k (warp w = token rows 4w .. 4w + 3, lane = 4 coordinates),
+//   store q^r, k^r, pool; U = K P_k^T (mma.sync; warp = 16 tokens x a quarter
+//   or half of the r columns); k~ = R_r SiLU(U) to shared memory; the half's
 //   barrier; C^T += V^T k~ (warp = 16 of the 128 d columns, all r rows).
 // The block means are pairwise sums (the summation order the block mask is
 // defined with, every rounding fixed, so the decision is the same on any
-// kernel that evaluates it): a thread adds its two rows 2a, 2a + 1, the 16
-// lanes a of a half-warp add those nodes in a butterfly (levels 2-5 of the
-// tree over the half's 32 rows, each lane ending with one of the 16 pooled
-// coordinates), and after the second half the two halves' nodes are added
-// and divided by the block's token count -- the same bits as the stand-alone
-// rotate + pool kernel.
+// kernel that evaluates it): a thread adds its four rows as a tree (levels 1
+// and 2), writes those nodes to a double-buffered shared tile, and after the
+// half's barrier thread c adds the 8 nodes of column c (levels 3-5); after the
+// second half the two halves' nodes are added and divided by the block's
+// token count -- the same bits as the stand-alone rotate + pool kernel.
 //
 // The loads of half-stage i + S - 1 are issued (by lane 0 of warps 0-2, one
 // box each) right after half-stage i's barrier, when every thread is done
@@ -80,8 +79,8 @@ struct Layout {
         stage_bytes = fuse ? 3 * kHalf : 2 * kHalf;
         P = stages * stage_bytes;                                 // P_k of the current head, r rows x 256 B
         kt = P + R * 256;                                         // k~, two buffers of 32 rows
-        part = kt + 2 * kHalfRows * (2 * R + 16);
-        zsm = part;
+        part = kt + 2 * kHalfRows * (2 * R + 16);                 // pooling nodes [2][8][q|k 256] fp32
+        zsm = part + (fuse ? 2 * 8 * 256 * 4 : 0);
         bars = zsm + 2 * R * 4;                                   // full[kMaxStages], abort
         total = bars + kMaxStages * 8 + 16;
     }
@@ -105,54 +104,32 @@ __device__ __forceinline__ void record_timeout(const Params& p, int where)
     if (atomicCAS(&p.status->code, 0, (int)ROLA_ERR_TIMEOUT) == 0) p.status->where = where;
 }
 
-// Rotates the 8 bf16 coordinates in w (4 pairs, (cos, sin) in cs) into y
+// Rotates the 4 bf16 coordinates in w (2 pairs, (cos, sin) in cs) into y
 // (fp32) and, for a token inside the sequence, stores them as bf16 at dst;
 // a token past the end gives y = +0 (an empty slot of the pairwise sum).
-__device__ __forceinline__ void rotate8(const uint4& w, const float2 (&cs)[4], __nv_bfloat16* dst, bool valid,
-                                        float (&y)[8])
+__device__ __forceinline__ void rotate4(const uint2& w, const float2 (&cs)[2], __nv_bfloat16* dst, bool valid,
+                                        float (&y)[4])
 {
-    const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
-    uint32_t out[4];
+    const uint32_t wv[2] = {w.x, w.y};
+    uint32_t out[2];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < 2; ++q) {
         const float2 x = unpack_bf16(wv[q]);
         const float2 r = rope_rotate(x.x, x.y, cs[q]);
         out[q] = pack_bf16(r.x, r.y);
         y[2 * q] = valid ? r.x : 0.0f;
         y[2 * q + 1] = valid ? r.y : 0.0f;
     }
-    if (valid) *reinterpret_cast<uint4*>(dst) = make_uint4(out[0], out[1], out[2], out[3]);
+    if (valid) *reinterpret_cast<uint2*>(dst) = make_uint2(out[0], out[1]);
 }
 
-// Levels 2-5 of the pairwise sum over a half's 32 rows: v holds this lane's
-// level-1 nodes (rows 2a, 2a + 1) of 16 pooled coordinates; the 16 lanes
-// a = lane mod 16 exchange halves of v in a butterfly (xor 1, 2, 4, 8), each
-// step adding the nodes of two neighbouring row ranges, so that lane a ends
-// with the node of all 32 rows for coordinate bitrev4(a) in v[0].  IEEE
-// addition commutes, so which lane holds the left operand does not matter.
-__device__ __forceinline__ void pairwise_butterfly(float (&v)[16], int a)
+__device__ __forceinline__ uint2 lds64(uint32_t a)
 {
-#pragma unroll
-    for (int lvl = 0; lvl < 4; ++lvl) {
-        const int off = 1 << lvl, half = 8 >> lvl;
-        const bool upper = (a >> lvl) & 1;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            if (i < half) {
-                const float keep = upper ? v[i + half] : v[i];
-                const float send = upper ? v[i] : v[i + half];
-                v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
-            }
-        }
-    }
-}
-
-__device__ __forceinline__ uint4 lds128(uint32_t a)
-{
-    uint4 w;
-    asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];\n" : "=r"(w.x), "=r"(w.y), "=r"(w.z), "=r"(w.w) : "r"(a));
+    uint2 w;
+    asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];\n" : "=r"(w.x), "=r"(w.y) : "r"(a));
     return w;
 }
+
 
 // SiLU with the approximate divide (the features enter the MMA in bf16).  The
 // kernel is instantiated for it and for ActAblation (the other feature maps).
@@ -220,16 +197,15 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
     const int mt = warp & 1, cg = warp >> 1;        // U: tokens 16 mt .. +15 of the half, column group cg
     const bool u_warp = cg < C::NSPLIT;             // (with two column groups, warps 4-7 skip U)
-    // rotation and pooling: rows 2 pa, 2 pa + 1 of the half, 8 coordinates; the
-    // two rows are read in the order psw gives, so that a half-warp's 16-byte
-    // shared loads fall on 8 distinct bank groups
-    const int pa = tid & 15, c8 = tid >> 4, psw = (pa >> 2) & 1;
-    const int pel = ((pa & 1) << 3) | ((pa & 2) << 1) | ((pa & 4) >> 1) | ((pa & 8) >> 3);   // bitrev4(pa)
+    // rotation and pooling: rows 4 warp .. 4 warp + 3 of the half, coordinates
+    // 4 lane .. 4 lane + 3 (pairs 2 lane, 2 lane + 1); a warp's 8-byte shared
+    // loads cover one whole row
+    const int cq = lane;
     const int hw = s.Hh * s.Ww;
-    int axis[4];
+    int axis[2];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int m = c8 * 4 + q;
+    for (int q = 0; q < 2; ++q) {
+        const int m = cq * 2 + q;
         axis[q] = m < s.pt ? 0 : (m < s.pt + s.px ? 1 : 2);
     }
     int kaxis[NTW];                                 // axis of pair nt * 4 + t4 of each of this warp's n-tiles
@@ -305,9 +281,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
     {
         const int blk0 = u0 - (u0 / s.nC) * s.nC;
         position(blk0 * kBlock + mt * 16 + g, kt_t, kt_x, kt_y);
-        position(blk0 * kBlock + 2 * pa, rt_t, rt_x, rt_y);
+        position(blk0 * kBlock + 4 * warp, rt_t, rt_x, rt_y);
     }
-    float pool0 = 0.0f;                             // pairwise node of the block's first half (element pel)
+    float pool0 = 0.0f;                             // pairwise node of the block's first half, column tid
+    float* nodes = reinterpret_cast<float*>(smem + lay.part);
     int i = 0;                                      // half-stage index
     for (; i < count; ++i) {
         const int u = u0 + (i >> 1), h = i & 1;
@@ -329,7 +306,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
             bar_sync(1, kThreads);
             if (hb >= 0) {                         // a new head starts at its block 0
                 position(mt * 16 + g, kt_t, kt_x, kt_y);
-                position(2 * pa, rt_t, rt_x, rt_y);
+                position(4 * warp, rt_t, rt_x, rt_y);
             }
             hb = bh;
         }
@@ -349,14 +326,14 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
                 advance(8, t, x, y);
             }
         }
-        // (cos, sin) of the rotation's pairs for this thread's two rows
-        float2 cs[2][4];
+        // (cos, sin) of the rotation's pairs for this thread's four rows
+        float2 cs[4][2];
         if (fuse) {
             int t = rt_t, x = rt_x, y = rt_y;
 #pragma unroll
-            for (int j = 0; j < 2; ++j) {
+            for (int j = 0; j < 4; ++j) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) cs[j][q] = __ldg(p.tab + table_row(axis[q], t, x, y) * kPairs + c8 * 4 + q);
+                for (int q = 0; q < 2; ++q) cs[j][q] = __ldg(p.tab + table_row(axis[q], t, x, y) * kPairs + cq * 2 + q);
                 advance(1, t, x, y);
             }
         }
@@ -366,38 +343,35 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
         const bool ok = __all_sync(0xffffffffu, mbar_wait(full0 + 8 * st, (i / S) & 1, abort, s.wait_limit_ns));
         if (ok) {
             if (fuse) {
-                // ---- rotate q and k, store q^r and k^r, pool (pairwise, the stand-alone kernel's bits)
-                uint4 wq[2], wk[2];
+                // ---- rotate q and k, store q^r and k^r, pool levels 1-2 (pairwise, the stand-alone kernel's bits)
+                uint2 wq[4], wk[4];
 #pragma unroll
-                for (int j = 0; j < 2; ++j) {
-                    const int row = 2 * pa + (j ^ psw);
-                    wq[j] = lds128(qb + hsw(row, c8));
-                    wk[j] = lds128(kb + hsw(row, c8));
+                for (int j = 0; j < 4; ++j) {
+                    const uint32_t a = hsw(4 * warp + j, cq >> 1) + (cq & 1) * 8;
+                    wq[j] = lds64(qb + a);
+                    wk[j] = lds64(kb + a);
                 }
-                float v[16];
+                float yq[4][4], yk[4][4];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {           // row 2 pa + e, loaded by load e ^ psw
-                    const int n = n_half + 2 * pa + e;
+                for (int j = 0; j < 4; ++j) {
+                    const int n = n_half + 4 * warp + j;
                     const bool valid = n < s.N;
-                    const size_t go = ((size_t)bh * s.N + (valid ? n : 0)) * kDh + c8 * 8;
-                    float yq[8], yk[8];
-                    rotate8((e ^ psw) ? wq[1] : wq[0], cs[e], p.qr + go, valid, yq);
-                    rotate8((e ^ psw) ? wk[1] : wk[0], cs[e], p.kr + go, valid, yk);
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) {               // level 1: row 2 pa + row 2 pa + 1
-                        v[c] = e ? v[c] + yq[c] : yq[c];
-                        v[8 + c] = e ? v[8 + c] + yk[c] : yk[c];
-                    }
+                    const size_t go = ((size_t)bh * s.N + (valid ? n : 0)) * kDh + cq * 4;
+                    rotate4(wq[j], cs[j], p.qr + go, valid, yq[j]);
+                    rotate4(wk[j], cs[j], p.kr + go, valid, yk[j]);
                 }
-                pairwise_butterfly(v, pa);
-                if (h == 0) {
-                    pool0 = v[0];
-                } else {
-                    // the top node: first half + second half, then the mean over the block's tokens
-                    const int cnt = min(kBlock, s.N - blk * kBlock);
-                    float* dst = pel < 8 ? p.qbar : p.kbar;
-                    dst[((size_t)bh * s.nC + blk) * kDh + c8 * 8 + (pel & 7)] = (pool0 + v[0]) / (float)cnt;
-                }
+                float4 nq, nk;                           // (y0 + y1) + (y2 + y3) per coordinate
+                nq.x = (yq[0][0] + yq[1][0]) + (yq[2][0] + yq[3][0]);
+                nq.y = (yq[0][1] + yq[1][1]) + (yq[2][1] + yq[3][1]);
+                nq.z = (yq[0][2] + yq[1][2]) + (yq[2][2] + yq[3][2]);
+                nq.w = (yq[0][3] + yq[1][3]) + (yq[2][3] + yq[3][3]);
+                nk.x = (yk[0][0] + yk[1][0]) + (yk[2][0] + yk[3][0]);
+                nk.y = (yk[0][1] + yk[1][1]) + (yk[2][1] + yk[3][1]);
+                nk.z = (yk[0][2] + yk[1][2]) + (yk[2][2] + yk[3][2]);
+                nk.w = (yk[0][3] + yk[1][3]) + (yk[2][3] + yk[3][3]);
+                float* nb = nodes + (buf * 8 + warp) * 256;
+                reinterpret_cast<float4*>(nb)[cq] = nq;
+                reinterpret_cast<float4*>(nb + 128)[cq] = nk;
             }
             if (u_warp) {
                 // ---- U = K P_k^T for tokens 16 mt .. +15 of the half and this warp's n-tiles
@@ -450,6 +424,21 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
         if (i >= 1 && issued < count) {       // half-stage i - 1 is done everywhere: refill its stage
             issue(issued);
             ++issued;
+        }
+        if (fuse) {
+            // ---- pooling levels 3-5: column tid (q: 0..127, k: 128..255) over the 8 nodes of this half
+            // (the buffer is written again two halves on, after every thread has passed the next barrier)
+            const float* nb = nodes + buf * 8 * 256 + tid;
+            const float half_sum = ((nb[0] + nb[256]) + (nb[512] + nb[768])) +
+                                   ((nb[1024] + nb[1280]) + (nb[1536] + nb[1792]));
+            if (h == 0) {
+                pool0 = half_sum;
+            } else {
+                // the top node: first half + second half, then the mean over the block's tokens
+                const int cnt = min(kBlock, s.N - blk * kBlock);
+                (tid < kDh ? p.qbar : p.kbar)[((size_t)bh * s.nC + blk) * kDh + (tid & (kDh - 1))] =
+                    (pool0 + half_sum) / (float)cnt;
+            }
         }
         // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 32 tokens
 #pragma unroll

@@ -85,6 +85,8 @@ def _load():
         "rola_backward_workspace_bytes": (S, [cfgp]),
         "rola_backward": (st, [cfgp] + [P] * 18 + [S, P]),
         "rola_gate": (st, [cfgp, P, P, ctypes.c_float, ctypes.c_int32, P, P]),
+        "rola_out_proj": (st, [cfgp, P, P, P, ctypes.c_int32, P, P, S, P]),
+        "rola_attention_block": (st, [cfgp, P, P, ctypes.c_float, ctypes.c_int32] + [P] * 12 + [S, P]),
         "rola_get_device_status": (st, [P, P]),
         "rola_status_string": (ctypes.c_char_p, [st]),
     }
@@ -221,6 +223,20 @@ def gate(c, X, w_g, b_g: float, gate_out, stream=None):
     """Token gate g = sigmoid(X w_g + b_g) into gate_out (fp32 [B][N]); X [B][N][d_model]."""
     _check(_lib.rola_gate(ctypes.byref(c), _p(X), _p(w_g), float(b_g), int(X.shape[-1]), _p(gate_out),
                           _stream(stream)), "rola_gate")
+
+
+def out_proj(c, O, W_o, b_o, Y, ws, stream=None):
+    """Y = concat_h(O) W_o^T (+ b_o): O [B][H][N][128], W_o [d_model][H*128], b_o fp32 [d_model] or
+    None, Y [B][N][d_model] (the block's output projection)."""
+    _check(_lib.rola_out_proj(ctypes.byref(c), _p(O), _p(W_o), _p(b_o), int(W_o.shape[0]), _p(Y), _p(ws),
+                              ws.numel(), _stream(stream)), "rola_out_proj")
+
+
+def attention_block(c, X, w_g, b_g: float, q, k, v, P_q, P_k, W_o, b_o, gate, o, Y, kv_idx_out, ws, stream=None):
+    """The block after the QKV projection: gate from X, the RoLA module, the output projection."""
+    _check(_lib.rola_attention_block(ctypes.byref(c), _p(X), _p(w_g), float(b_g), int(X.shape[-1]), _p(q), _p(k),
+                                     _p(v), _p(P_q), _p(P_k), _p(W_o), _p(b_o), _p(gate), _p(o), _p(Y),
+                                     _p(kv_idx_out), _p(ws), ws.numel(), _stream(stream)), "rola_attention_block")
 
 
 def forward_timed(c, q, k, v, P_q, P_k, gate, o, kv_idx_out, ws, events, stream=None):

@@ -91,6 +91,8 @@ def call_all(rl, c, ws_bytes=1 << 30, ptr=0x10000, ws=0x100000):
         L.rola_lowrank_summary(b, p, p, p, p, None, w, ws_bytes, None),
         L.rola_lowrank_apply(b, p, p, p, None, p, p, w, ws_bytes, None),
         L.rola_forward(b, p, p, p, p, p, None, p, None, w, ws_bytes, None),
+        L.rola_out_proj(b, p, p, None, 256, p, w, ws_bytes, None),
+        L.rola_attention_block(b, p, p, -1.946, 256, p, p, p, p, p, p, None, p, p, p, None, w, ws_bytes, None),
     ]
 
 
@@ -168,7 +170,9 @@ def test_null_and_misaligned_pointers(rl):
 def test_workspace_checks(rl):
     c = cfg_tiny(rl)
     need = rl.workspace_bytes(c)
-    assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws_bytes=need - 1))
+    short = call_all(rl, c, ws_bytes=need - 1)
+    del short[5]                       # rola_out_proj needs only the 256-byte status word
+    assert all(s == rl.ROLA_ERR_WORKSPACE for s in short)
     assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws=0x100080))   # not 256-aligned
     assert all(s == rl.ROLA_ERR_WORKSPACE for s in call_all(rl, c, ws=0))
 
@@ -227,3 +231,21 @@ def test_gate_arguments_are_checked_before_launch(rl):
     assert L.rola_gate(b, ok, ok, float("nan"), 128, ok, None) == rl.ROLA_ERR_INVALID_ARG
     c.N = 1000                                   # N != T * Hh * Ww
     assert L.rola_gate(b, ok, ok, -1.946, 128, ok, None) == rl.ROLA_ERR_INVALID_ARG
+
+
+def test_out_proj_arguments_are_checked_before_launch(rl):
+    """rola_out_proj: d_model a positive multiple of 64, 16-byte aligned operands, and a 256-byte
+    aligned status word of at least 256 bytes -- each refused before any launch."""
+    L = rl.library()
+    P = ctypes.c_void_p
+    c = cfg_tiny(rl)
+    b, p, w = ctypes.byref(c), P(0x10000), P(0x100000)
+    assert L.rola_out_proj(b, p, p, None, 96, p, w, 4096, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_out_proj(b, p, p, None, 0, p, w, 4096, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_out_proj(b, P(0x10008), p, None, 128, p, w, 4096, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_out_proj(b, p, p, ctypes.cast(P(0x10004), ctypes.POINTER(ctypes.c_float)), 128, p, w, 4096,
+                           None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_out_proj(b, None, p, None, 128, p, w, 4096, None) == rl.ROLA_ERR_INVALID_ARG
+    assert L.rola_out_proj(b, p, p, None, 128, p, w, 128, None) == rl.ROLA_ERR_WORKSPACE
+    assert L.rola_out_proj(b, p, p, None, 128, p, P(0x100010), 4096, None) == rl.ROLA_ERR_WORKSPACE
+    assert L.rola_out_proj(b, p, p, None, 128, p, None, 4096, None) == rl.ROLA_ERR_WORKSPACE

@@ -91,3 +91,20 @@ def test_accounting_uses_the_printed_complexity_formulas():
         c_sparse = gold["sparse_coeff"] * B * H * L ** 2 * (1 - S) * d
         eta = (bench.lowrank_flops(B, H, L, d, r) + gold["fusion_coeff"] * B * H * L * d) / c_sparse
         assert eta == pytest.approx((gold["eta_r_coeff"] * r + gold["eta_const"]) / (L * (1 - S)), rel=1e-12)
+
+
+def test_sparse_traffic_follows_the_committed_capture(tmp_path, monkeypatch):
+    """roofline.traffic comes from the committed ncu summary only while the kernel's sources
+    are the ones that capture was taken on: a summary recording another source hash, or one
+    without the two fields, gives None (the bench then reports traffic: null)."""
+    tph = bench.sparse_traffic_per_head_token()
+    assert tph is not None and 900.0 < tph < 1100.0      # q^r + k^r + v read, O^s written: ~4 x 256 B
+    text = open(bench.SPARSE_PROFILE).read()
+    stale = tmp_path / "stale.md"
+    stale.write_text(text.replace("kernel_sources_sha256: ", "kernel_sources_sha256: 0"))
+    monkeypatch.setattr(bench, "SPARSE_PROFILE", str(stale))
+    assert bench.sparse_traffic_per_head_token() is None
+    bare = tmp_path / "bare.md"
+    bare.write_text("\n".join(l for l in text.splitlines() if not l.startswith("traffic_bytes")))
+    monkeypatch.setattr(bench, "SPARSE_PROFILE", str(bare))
+    assert bench.sparse_traffic_per_head_token() is None

@@ -81,6 +81,10 @@ MUTATIONS = {
     "f32_scale_dropped": ("row[j].s = acc * scale;", "row[j].s = acc;"),
     "f32_cube_slot_order": ("x = CUBE * cx + (i / CUBE) % CUBE, y = CUBE * cy + i % CUBE;",
                             "x = CUBE * cx + i % CUBE, y = CUBE * cy + (i / CUBE) % CUBE;"),
+    "out_proj_concat_order": ("cat[h * dh + d] = O[", "cat[d * H + h] = O["),
+    "out_proj_transposed_weight": ("y += cat[k] * (double)W[(size_t)f * K + k];",
+                                   "y += cat[k] * (double)W[((size_t)k * d_model + f) % ((size_t)K * d_model)];"),
+    "out_proj_bias_dropped": ("double y = bias ? (double)bias[f] : 0.0;", "double y = 0.0;"),
     "readout_index": ("s += qt[a] * Cb[(size_t)a * dh + d];", "s += qt[a] * Cb[(size_t)d * c->r % (c->r * dh) + a];"),
 }
 

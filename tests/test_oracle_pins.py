@@ -152,7 +152,7 @@ def wide_range(cfg, seed):
 @pytest.mark.parametrize("geometry", ["flat", "cube"])
 @pytest.mark.parametrize("dist", ["normal", "rmsnorm", "wide"])
 def test_fp32_decision_within_the_near_tie_bound(oracle, dist, geometry):
-    """The block mask is an fp32 decision (reading 11).  tau / 2 is a rigorous bound on how far the
+    """The block mask is an fp32 decision.  tau / 2 is a rigorous bound on how far the
     oracle's fp32 evaluation of a score sits from the fp64 one (first-order error analysis of the
     rotation, the pairwise pooling, the division, the fma chain and the scale); checked at every
     (i, j) on three input distributions and both block geometries.  Rows with gap > tau then keep the
@@ -752,3 +752,26 @@ def test_query_block_sparse_branch_shares_the_mask_row(oracle):
     idx1, _, _, _ = O.block_mask(full, x["q"], x["k"])
     np.testing.assert_allclose(O.sparse_attn(full, qr, kr, x["v"], idx1), sdpa64(qr, kr, x["v"]),
                                rtol=1e-11, atol=1e-12)
+
+
+def test_out_proj_pins(oracle):
+    """Output projection (Alg. 1, last step): the heads concatenated per token in head order, times
+    W_o^T, plus the bias.  Pinned by a numpy matmul of the concatenation on small integer inputs
+    (exact in fp64) with a rectangular W_o, by the head selection (W_o's identity block at head h
+    returns head h's rows), and by O = 0 giving the bias."""
+    O = oracle
+    rng = np.random.default_rng(7)
+    B, H, N, dh, dm = 2, 3, 5, 4, 7
+    Oh = rng.integers(-3, 4, size=(B, H, N, dh)).astype(np.float64)
+    W = rng.integers(-2, 3, size=(dm, H * dh)).astype(np.float32)
+    b = rng.integers(-5, 6, size=dm).astype(np.float32)
+    cat = np.concatenate([Oh[:, h] for h in range(H)], axis=-1)          # [B, N, H*dh]
+    assert (O.out_proj(Oh, W, b) == cat @ W.T.astype(np.float64) + b).all()
+    assert (O.out_proj(Oh, W) == cat @ W.T.astype(np.float64)).all()
+    for h in range(H):
+        Wh = np.zeros((dh, H * dh), np.float32)
+        Wh[:, h * dh:(h + 1) * dh] = np.eye(dh)
+        assert (O.out_proj(Oh, Wh) == Oh[:, h]).all()
+    assert (O.out_proj(np.zeros_like(Oh), W, b) == np.broadcast_to(b, (B, N, dm))).all()
+    part = O.out_proj(Oh, W, b, rows=[1, 3])
+    assert np.isnan(part[:, [0, 2, 4]]).all() and (part[:, [1, 3]] == (cat @ W.T.astype(np.float64) + b)[:, [1, 3]]).all()

@@ -1,4 +1,6 @@
-"""Guard canaries: no entry point writes outside the buffers it is given.
+"""Guard canaries: no entry point writes outside the buffers it is given (every
+output of every entry point, the workspace-free summary and the token gate
+included).
 
 compute-sanitizer is closed on this machine, so every output and workspace is
 placed inside a larger buffer whose margins (8 KB on each side) hold a fixed
@@ -88,6 +90,16 @@ def test_no_store_outside_the_given_buffers(rl, layer, dname, tdt):
     rl.backward(c, q, k, v, Pq, Pk, g, kv2, o_s2, lse, C2, dO, G(row, tdt), G(row, tdt), G(row, tdt),
                 G(Pq.shape, torch.float32), G(Pk.shape, torch.float32),
                 G((B, N), torch.float32) if g is not None else None, bws)
+    # the summary without a workspace (its scratch is the library's own array)
+    Cs, zs = G((B, H, r, 128), torch.float32), G((B, H, r), torch.float32)
+    st = rl.library().rola_lowrank_summary_static(
+        ctypes.byref(c), ctypes.c_void_p(k.data_ptr()), ctypes.c_void_p(v.data_ptr()), ctypes.c_void_p(Pk.data_ptr()),
+        ctypes.c_void_p(Cs.data_ptr()), ctypes.c_void_p(zs.data_ptr()),
+        ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert st == rl.ROLA_OK
+    # the token gate from a block input of d_model = 8 * 40 (a ragged last warp tile)
+    xg = inputs.make_gate_inputs(B, N, 320, dtype=tdt, device="cuda", seed=5)
+    rl.gate(c, xg["X"], xg["w_g"], xg["b_g"], G((B, N), torch.float32))
     torch.cuda.synchronize()
     assert rl.get_device_status(ws) == rl.ROLA_OK and rl.get_device_status(bws) == rl.ROLA_OK
     bad = [i for i, t in enumerate(guards) if not t.intact()]
