@@ -32,9 +32,9 @@
 //   warp  9    TMA producer: the V blocks
 //   warp 10    Q K^T issuer and TMEM owner
 //   warp 11    P V issuer
-// Buffers: K pairs in a 3-deep ring and V blocks in a 5-deep ring of single
-// blocks (the L2 -> shared-memory latency under load is ~2 us, so the bytes in
-// flight set the pace; 224 KB of the 227 KB go to tiles); S^T, P^T and O^T double-buffered, so the next tile's Q K^T
+// Buffers: K pairs in a 2-deep ring and V blocks in a 7-deep ring of single
+// blocks (a V block is needed a softmax later than its K pair, so V gets the
+// deeper ring; 224 KB of the 227 KB go to tiles); S^T, P^T and O^T double-buffered, so the next tile's Q K^T
 // runs while the current tile's softmax does and the next query block's
 // first tiles run while the current one's epilogue does; Q single-buffered.  Every wait on an
 // mbarrier is bounded (2 s); a wait that gives up records ROLA_ERR_TIMEOUT
@@ -64,8 +64,8 @@ constexpr int kWGThreads = 128;
 constexpr uint32_t kQBytes = 64 * 128 * 2;          // one query block
 constexpr uint32_t kKVBytes = 128 * 128 * 2;        // a pair of key blocks
 constexpr uint32_t kPBytes = 128 * 64 * 2;          // P^T tile
-constexpr int KS = 3;                               // K ring: pairs of key blocks ([chunk][block][row])
-constexpr int VB = 5;                               // V ring: single key blocks (16 KB, [chunk][row])
+constexpr int KS = 2;                               // K ring: pairs of key blocks ([chunk][block][row])
+constexpr int VB = 7;                               // V ring: single key blocks (16 KB, [chunk][row])
 constexpr uint32_t kVBlockBytes = 64 * 128 * 2;
 constexpr uint32_t kSmemQ = 0;
 constexpr uint32_t kSmemK = kSmemQ + kQBytes;
@@ -84,6 +84,7 @@ enum Bar { Q_FULL = 0, Q_EMPTY = 1, K_FULL = 2, K_EMPTY = K_FULL + KS, V_FULL = 
 struct Smem {
     alignas(16) float m[64];          // minus the running maximum per query (log2 units)
     alignas(16) float alpha[64];      // rescale factors of the current tile
+    alignas(16) float delta[64];      // the raise of m_q of the current tile (log2 units)
     alignas(16) float red[kSoftmaxWG][4][kCols];   // cross-warp reduction scratch, per warpgroup
     alignas(16) float inv_l[64];
     uint64_t bar[NUM_BARS];
@@ -444,9 +445,6 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                 const uint32_t saddr = tmem + lane_off + sb * 64 + col0;
                 float x[kCols];
                 tmem_ld_cols<kCols>(saddr, x);
-                float s_raw[kCols];                            // kept for the rare rescale path
-#pragma unroll
-                for (int q = 0; q < kCols; ++q) s_raw[q] = x[q];
                 fence_before_sync();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(S_EMPTY + sb));  // S^T buffer free for Q K^T(g + 2)
@@ -465,23 +463,21 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
                     for (int q = 0; q < kCols; ++q) x[q] = -INFINITY;
                 }
                 if (bar_red_or(1 + wg, kWGThreads, need)) {
-                    column_reduce<true>(x, sm, wg, wtid, sm.alpha + col0);   // alpha <- column maxima of t
+                    float xr[kCols];                                                // the reduction consumes its input
+#pragma unroll
+                    for (int q = 0; q < kCols; ++q) xr[q] = x[q];
+                    column_reduce<true>(xr, sm, wg, wtid, sm.alpha + col0);   // alpha <- column maxima of t
                     if (wtid < kCols) {
                         const float tmax = sm.alpha[col0 + wtid];
                         const float delta = t == 0 ? tmax : fmaxf(tmax, 0.0f);
                         sm.m[col0 + wtid] -= delta;
                         sm.alpha[col0 + wtid] = fast_exp2(-delta);
+                        sm.delta[col0 + wtid] = delta;
                     }
                     bar_sync(1 + wg, kWGThreads);
-                    if (valid) {                                                     // recompute t against the new m
+                    if (valid) {                                   // t against the new m: t - (m_new - m_old)
 #pragma unroll
-                        for (int q = 0; q < kCols; q += 4) {
-                            const float4 nm = *reinterpret_cast<const float4*>(&sm.m[col0 + q]);
-                            x[q] = fmaf(s_raw[q], c_log2, nm.x);
-                            x[q + 1] = fmaf(s_raw[q + 1], c_log2, nm.y);
-                            x[q + 2] = fmaf(s_raw[q + 2], c_log2, nm.z);
-                            x[q + 3] = fmaf(s_raw[q + 3], c_log2, nm.w);
-                        }
+                        for (int q = 0; q < kCols; ++q) x[q] -= sm.delta[col0 + q];
                     } else {
 #pragma unroll
                         for (int q = 0; q < kCols; ++q) x[q] = -INFINITY;
