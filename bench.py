@@ -83,14 +83,16 @@ def block_sizes(cfg, block=64):
     return [block] * (nB - 1) + [cfg["N"] - (nB - 1) * block]
 
 
-def sparse_flops_from_mask(kv_idx, sizes, d_h=128):
+def sparse_flops_from_mask(kv_idx, sizes, d_h=128, qsizes=None):
     """Algorithmic FLOPs of the sparse branch: 4 d_h sum_{h,i} |Q_i| sum_{j kept} |K_j|
     (QK^T and PV, 2 flops per multiply-add), every block counted at its real size
-    (App. D, C_sparse = 4 B H L^2 (1-S) d_h)."""
+    (App. D, C_sparse = 4 B H L^2 (1-S) d_h).  qsizes: the query blocks' sizes when they
+    differ from the key blocks' (128-token query chunks)."""
     import torch
     sizes = torch.tensor(sizes, dtype=torch.float64, device=kv_idx.device)
+    qs = sizes if qsizes is None else torch.tensor(qsizes, dtype=torch.float64, device=kv_idx.device)
     keys = sizes[kv_idx.long()].sum(dim=-1)            # [B,H,nQB] kept keys per query block
-    return float(4.0 * d_h * (keys * sizes).sum().item())
+    return float(4.0 * d_h * (keys * qs).sum().item())
 
 
 def lowrank_flops(B, H, N, d_h, r):
@@ -402,6 +404,8 @@ def main():
                     help="blocks of the sparse branch: 64-token chunks (default) or 4x4x4 cubes of the latent grid")
     ap.add_argument("--lowrank-act", default=None, choices=["silu", "identity", "tanh", "relu", "gelu"],
                     help="feature map of the low-rank branch (the activation ablation); default SiLU")
+    ap.add_argument("--qblock", type=int, default=None, choices=[64, 128],
+                    help="tokens per query block of the mask (128: the b_q = 128 variant); default 64")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -425,6 +429,8 @@ def main():
         cfg["lowrank_act"] = args.lowrank_act
     if args.geometry is not None:
         cfg["block_geometry"] = args.geometry
+    if args.qblock is not None:
+        cfg["qblock"] = args.qblock
     ws, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, cfg, ws, rank)
@@ -442,7 +448,7 @@ def main():
     wsb = rola.workspace(c, dev)
     nB, nk = rola.num_blocks(c), rola.num_keep(c)
     o = torch.empty_like(x["q"])
-    kv = torch.empty((cfg["B"], cfg["H"], nB, nk), dtype=torch.int32, device=dev)
+    kv = torch.empty((cfg["B"], cfg["H"], rola.num_query_blocks(c), nk), dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     K = args.steps
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
@@ -493,7 +499,8 @@ def main():
     # ---- roofline of the dominant kernel (the sparse branch: tensor-core bound)
     peaks, peak_src = load_peaks()
     geometry = cfg.get("block_geometry", "flat")
-    fl = sparse_flops_from_mask(kv, block_sizes(cfg))
+    fl = sparse_flops_from_mask(kv, block_sizes(cfg),
+                                qsizes=block_sizes(cfg, 128) if cfg.get("qblock", 0) == 128 else None)
     sp_ms = stage_ms["sparse_attn"]
     achieved = fl / (sp_ms * 1e-3) / 1e12
     # burst peak: the timed region is well under a second and ran at full SM clock (the
@@ -664,7 +671,7 @@ def main():
     if not args.no_dense:
         cd = rola.make_config(dict(cfg, keep=1.0))
         wsd = rola.workspace(cd, dev)
-        kvd = torch.empty((cfg["B"], cfg["H"], nB, nB), dtype=torch.int32, device=dev)
+        kvd = torch.empty((cfg["B"], cfg["H"], rola.num_query_blocks(cd), nB), dtype=torch.int32, device=dev)
         rola.forward(cd, x["q"], x["k"], x["v"], x["P_q"], x["P_k"], x["gate"], o, kvd, wsd)
         torch.cuda.synchronize()
         s3, t3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -674,7 +681,9 @@ def main():
         t3.record(stream)
         torch.cuda.synchronize()
         d_ms = s3.elapsed_time(t3) / 2
-        flop_ratio = (sparse_flops_from_mask(kvd, block_sizes(cfg)) + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"])) / \
+        qsz = block_sizes(cfg, 128) if cfg.get("qblock", 0) == 128 else None
+        flop_ratio = (sparse_flops_from_mask(kvd, block_sizes(cfg), qsizes=qsz) +
+                      lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"])) / \
             (fl + lowrank_flops(1, cfg["H"], cfg["N"], 128, cfg["r"]))
         dense = {"dense_ms": d_ms, "speedup": d_ms / ms_step, "flop_ratio": flop_ratio,
                  "target_speedup": 0.85 * flop_ratio}
@@ -693,6 +702,7 @@ def main():
                        "grid": [cfg["T"], cfg["Hh"], cfg["Ww"]], "block": 64, "keep": cfg["keep"],
                        "n_keep": nk, "r": cfg["r"], "d_h": 128, "lowrank_act": cfg.get("lowrank_act", "silu"),
                        "block_geometry": cfg.get("block_geometry", "flat"),
+                       "query_block": cfg.get("qblock", 0) or 64,
                        "l2": "no flush: q, k, v are each larger than L2 (774 MB vs 129 MB)",
                        "parallelism": f"replica per GPU x{ws}"},
             "stage_ms": stage_ms,

@@ -102,6 +102,11 @@ typedef struct {
                                   rola_lowrank_act_t, default ROLA_LOWRANK_ACT_SILU */
     int32_t block_geometry;    /* which tokens form a block of the sparse branch; one of
                                   rola_block_geometry_t, default ROLA_BLOCK_FLAT */
+    int32_t query_block;       /* tokens per query block of the mask, ROLA_BLOCK_FLAT only: 0 or 64
+                                  (the key blocks' size, default) or 128 -- each 128-token query chunk
+                                  is pooled, scored and given its n_keep key blocks as one unit (the
+                                  b_q = 128 / b_kv = 64 tiling of the block-sparse video attentions
+                                  the paper builds on); the forward entry points only */
 } rola_config_t;
 
 #define ROLA_DEBUG_SKIP_FIRST_K_COPY 1
@@ -158,9 +163,13 @@ typedef enum {
 /* Fill *cfg with defaults (shape fields zero).  Returns ROLA_ERR_INVALID_ARG on NULL. */
 rola_status_t rola_config_init(rola_config_t* cfg);
 
-/* The number of query blocks nQB, equal to the number of key blocks nKB: ceil(N / block), or
- * the cube count for ROLA_BLOCK_CUBE; 0 if cfg is invalid. */
+/* The number of key blocks nKB: ceil(N / block), or the cube count for ROLA_BLOCK_CUBE; 0 if cfg
+ * is invalid.  It is also the number of query blocks unless cfg->query_block is 128. */
 int32_t rola_num_blocks(const rola_config_t* cfg);
+
+/* The number of query blocks nQB, the rows of kv_idx: ceil(N / 128) when cfg->query_block is 128,
+ * else rola_num_blocks(cfg); 0 if cfg is invalid. */
+int32_t rola_num_query_blocks(const rola_config_t* cfg);
 
 /* Kept key blocks per query block, clamp(floor(keep_ratio*nKB + 0.5), 1, nKB); 0 if cfg is invalid. */
 int32_t rola_num_keep(const rola_config_t* cfg);
@@ -178,7 +187,12 @@ size_t rola_workspace_bytes(const rola_config_t* cfg);
  * n_keep highest-scoring key blocks of each query block (Alg. 1, "topk
  * ratio"; the pooling / scoring rule is this library's reading of the
  * unspecified selection of the sparse engine).  Ties go to the lower block
- * id.  Pooled means and scores are fp32.
+ * id.  The selection turns floating point into integers, so it is an fp32
+ * decision with every rounding fixed: the fp32 (cos, sin) table,
+ * y0 = fma(x0, c, -fl(x1 s)), y1 = fma(x0, s, fl(x1 c)); a block's slots
+ * (64, or 128 query tokens) summed pairwise in slot order, empty slots +0,
+ * one division by its token count; each score an ascending-d fma chain from
+ * +0 times fl(1/sqrt(d_h)).  Every kernel of this library evaluates it so.
  *   q, k    : [B][H][N][d_h] pre-RoPE, dtype
  *   kv_idx  : out, int32 [B][H][nQB][n_keep], ascending within each row
  */

@@ -27,6 +27,12 @@ int64_t block_rows_of(const rola_config_t& c)
     return c.block_geometry == ROLA_BLOCK_CUBE ? (int64_t)num_blocks_of(c) * c.block : c.N;
 }
 
+int num_qblocks_of(const rola_config_t& c)
+{
+    if (c.query_block == 128) return (int)(((int64_t)c.N + 127) / 128);
+    return num_blocks_of(c);
+}
+
 int num_keep_of(const rola_config_t& c)
 {
     int nkb = num_blocks_of(c);
@@ -63,6 +69,8 @@ rola_status_t validate(const rola_config_t* c)
         return ROLA_ERR_INVALID_ARG;
     if (c->lowrank_act < ROLA_LOWRANK_ACT_SILU || c->lowrank_act > ROLA_LOWRANK_ACT_GELU) return ROLA_ERR_INVALID_ARG;
     if (c->block_geometry != ROLA_BLOCK_FLAT && c->block_geometry != ROLA_BLOCK_CUBE) return ROLA_ERR_INVALID_ARG;
+    if (c->query_block != 0 && c->query_block != kBlock && c->query_block != 128) return ROLA_ERR_INVALID_ARG;
+    if (c->query_block == 128 && c->block_geometry != ROLA_BLOCK_FLAT) return ROLA_ERR_UNSUPPORTED;
     // grid / index limits of the kernels
     if ((int64_t)c->B * c->H > 65535) return ROLA_ERR_UNSUPPORTED;
     // the top-k kernel holds a row of nB keys per warp in shared memory (8 warps, 227 KB)
@@ -81,6 +89,8 @@ Shape make_shape(const rola_config_t& c)
     s.B = c.B; s.H = c.H; s.N = c.N; s.r = c.r;
     s.rp = (c.r + 15) & ~15;
     s.nB = num_blocks_of(c);
+    s.nQ = num_qblocks_of(c);
+    s.qb2 = c.query_block == 128 ? 1 : 0;
     s.nC = (int)(((int64_t)c.N + kBlock - 1) / kBlock);
     s.n_keep = num_keep_of(c);
     s.T = c.T; s.Hh = c.Hh; s.Ww = c.Ww;
@@ -128,8 +138,9 @@ Workspace layout(const rola_config_t& c)
     w.vp = off; off = align_up(off + (s.cube ? esz * bh * s.Np * kDh : 0));   // v in block order (cube)
     w.qbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
     w.kbar = off; off = align_up(off + 4 * bh * s.nB * kDh);
-    w.scores = off; off = align_up(off + 4 * bh * s.nB * s.nB);
-    w.kv_idx = off; off = align_up(off + 4 * bh * s.nB * s.n_keep);
+    w.qbar2 = off; off = align_up(off + (s.qb2 ? 4 * bh * s.nQ * kDh : 0));   // 128-token query means
+    w.scores = off; off = align_up(off + 4 * bh * s.nQ * s.nB);
+    w.kv_idx = off; off = align_up(off + 4 * bh * s.nQ * s.n_keep);
     w.C = off; off = align_up(off + 4 * bh * c.r * kDh);
     w.z = off; off = align_up(off + 4 * bh * c.r);
     w.Cbf = off; off = align_up(off + 2 * bh * s.rp * kDh);           // zero-padded to rp rows
@@ -203,12 +214,23 @@ const void* sparse_v(const Shape& s, const Workspace& w, const void* v, void* ws
     return s.cube ? at<void>(ws, w.vp) : v;
 }
 
+// Block scores and top-k from the pooled means (128-token query means first, when configured).
+cudaError_t select_blocks(const Shape& s, const Workspace& w, int32_t* kv_idx, void* ws, cudaStream_t st)
+{
+    const float* qm = at<float>(ws, w.qbar);
+    if (s.qb2) {
+        cudaError_t e = launch_qpool128(s, at<float>(ws, w.qbar), at<float>(ws, w.qbar2), st);
+        if (e != cudaSuccess) return e;
+        qm = at<float>(ws, w.qbar2);
+    }
+    return launch_block_topk(s, qm, at<float>(ws, w.kbar), at<float>(ws, w.scores), kv_idx, st);
+}
+
 rola_status_t run_mask(const rola_config_t& c, const Shape& s, const Workspace& w, const void* q, const void* k,
                        const void* v, int32_t* kv_idx, void* ws, cudaStream_t st)
 {
     ROLA_TRY(rope_pool(c, s, w, q, k, v, ws, st));
-    ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv_idx,
-                               st));
+    ROLA_TRY(select_blocks(s, w, kv_idx, ws, st));
     return ROLA_OK;
 }
 
@@ -289,8 +311,7 @@ rola_status_t forward_impl(const rola_config_t* cfg, const void* q, const void* 
         ROLA_TRY(launch_prepass(s, ctas, nullptr, k, v, P_k, at<float2>(ws, w.table), nullptr, nullptr, nullptr,
                                 nullptr, at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
         ROLA_TRY(mark(1));
-        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
-                                   st));
+        ROLA_TRY(select_blocks(s, w, kv, ws, st));
         ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
                                         at<__nv_bfloat16>(ws, w.Cbf), st));
     } else if (cfg->dtype == ROLA_BF16) {
@@ -302,8 +323,7 @@ rola_status_t forward_impl(const rola_config_t* cfg, const void* q, const void* 
                                 at<void>(ws, w.kr), at<float>(ws, w.qbar), at<float>(ws, w.kbar),
                                 at<float>(ws, w.partials), at<DeviceStatus>(ws, w.status), st));
         ROLA_TRY(mark(1));
-        ROLA_TRY(launch_block_topk(s, at<float>(ws, w.qbar), at<float>(ws, w.kbar), at<float>(ws, w.scores), kv,
-                                   st));
+        ROLA_TRY(select_blocks(s, w, kv, ws, st));
         ROLA_TRY(launch_prepass_combine(s, ctas, at<float>(ws, w.partials), at<float>(ws, w.C), at<float>(ws, w.z),
                                         at<__nv_bfloat16>(ws, w.Cbf), st));
     } else {
@@ -377,6 +397,12 @@ int32_t rola_num_blocks(const rola_config_t* cfg)
 {
     if (validate(cfg) != ROLA_OK) return 0;
     return num_blocks_of(*cfg);
+}
+
+int32_t rola_num_query_blocks(const rola_config_t* cfg)
+{
+    if (validate(cfg) != ROLA_OK) return 0;
+    return num_qblocks_of(*cfg);
 }
 
 int32_t rola_num_keep(const rola_config_t* cfg)
@@ -471,6 +497,7 @@ rola_status_t rola_forward_train(const rola_config_t* cfg, const void* q, const 
                                  void* o_s, float* lse, float* C, void* ws, size_t ws_bytes, void* stream)
 {
     if (!kv_idx_out || !o_s || !lse || !C) return validate(cfg) == ROLA_OK ? ROLA_ERR_INVALID_ARG : validate(cfg);
+    if (validate(cfg) == ROLA_OK && cfg->query_block == 128) return ROLA_ERR_UNSUPPORTED;   // no backward for it
     return forward_impl(cfg, q, k, v, P_q, P_k, gate, o, kv_idx_out, o_s, lse, C, ws, ws_bytes, stream, nullptr);
 }
 
@@ -493,6 +520,7 @@ rola_status_t rola_backward(const rola_config_t* cfg, const void* q, const void*
                             float* dP_q, float* dP_k, float* dgate, void* ws, size_t ws_bytes, void* stream)
 {
     ROLA_CHECK(validate(cfg));
+    if (cfg->query_block == 128) return ROLA_ERR_UNSUPPORTED;
     const void* in[] = {q, k, v, P_q, P_k, kv_idx, o_s, lse, C, dO, dq, dk, dv, dP_q, dP_k};
     for (const void* p : in)
         if (!p || !aligned16(p)) return ROLA_ERR_INVALID_ARG;

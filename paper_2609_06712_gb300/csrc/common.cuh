@@ -31,7 +31,9 @@ struct DeviceStatus {
 
 // Kernel-side view of a validated configuration.
 struct Shape {
-    int B, H, N, nB, n_keep, r;   // nB: blocks of the sparse branch (chunks or cubes)
+    int B, H, N, nB, n_keep, r;   // nB: key blocks of the sparse branch (chunks or cubes)
+    int nQ;                   // query blocks (rows of the mask): nB, or ceil(N / 128) with 128-token queries
+    int qb2;                  // 1 with 128-token query blocks: the mask row of 64-token block i is i >> 1
     int nC;                   // 64-token chunks ceil(N / 64): the units of the low-rank kernels
     int rp;                   // r rounded up to a multiple of 16: the width the bf16 kernels run at
                               // (rows r .. rp-1 of P are read as zero, so those features are zero)
@@ -157,7 +159,7 @@ __device__ __forceinline__ float2 lowrank_pair(float u0, float u1, float2 cs, in
 
 // Workspace carve-up for one configuration.
 struct Workspace {
-    size_t status, table, qr, kr, vp, qbar, kbar, scores, kv_idx, C, z, Cbf, partials, total;
+    size_t status, table, qr, kr, vp, qbar, kbar, qbar2, scores, kv_idx, C, z, Cbf, partials, total;
     int nsplit;               // fp32 summary splits
     size_t prepass_slots;     // bf16 pre-pass partial slots
 };
@@ -165,12 +167,17 @@ struct Workspace {
 // Host launchers, one per kernel family.  All return cudaGetLastError().
 cudaError_t launch_rope_table(const rola_config_t& cfg, float2* tab, cudaStream_t st);
 // q^r, k^r (rows in block order, Np per head) and the block means; in cube
-// geometry also v copied into block order (vp) when v is given.
+// geometry also v copied into block order (vp) when v is given.  With
+// 128-token query blocks (s.qb2) qbar receives the 64-token blocks' q SUMS,
+// which launch_qpool128 turns into the 128-token means.
 cudaError_t launch_rope_pool(const rola_config_t& cfg, const Shape& s, const void* q, const void* k,
                              const void* v, const float2* tab, void* qr, void* kr, void* vp, float* qbar,
                              float* kbar, cudaStream_t st);
+// qbar [B*H][nQ][128] (query means), kbar [B*H][nB][128]: scores [B*H][nQ][nB], kv_idx [B*H][nQ][n_keep].
 cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
                               int32_t* kv_idx, cudaStream_t st);
+// 128-token query means from the 64-token q sums: (S[2c] + S[2c+1]) / tokens of chunk c.
+cudaError_t launch_qpool128(const Shape& s, const float* qsum64, float* qbar128, cudaStream_t st);
 // lse (nullable): fp32 [B][H][N], log sum_j exp(s_pj) of each query row (natural log).
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr,
                                const void* v, const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status,

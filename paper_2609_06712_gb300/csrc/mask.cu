@@ -27,7 +27,7 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
     __shared__ __align__(16) float qs[2][kSChunk][kSTile + 4];
     __shared__ __align__(16) float ks[2][kSChunk][kSTile + 4];
     const int bh = blockIdx.z, i0 = blockIdx.y * kSTile, j0 = blockIdx.x * kSTile;
-    const float* Q = qbar + (size_t)bh * s.nB * kDh;
+    const float* Q = qbar + (size_t)bh * s.nQ * kDh;
     const float* K = kbar + (size_t)bh * s.nB * kDh;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     // loader: 128 rows x 16 d per operand = 512 float4, two per thread
@@ -38,7 +38,7 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
         for (int h = 0; h < 2; ++h) {
             const int row = lrow + 64 * h;
             const int gi = i0 + row, gj = j0 + row;
-            ra[h] = gi < s.nB ? __ldg(reinterpret_cast<const float4*>(Q + (size_t)gi * kDh + d0) + lq)
+            ra[h] = gi < s.nQ ? __ldg(reinterpret_cast<const float4*>(Q + (size_t)gi * kDh + d0) + lq)
                               : make_float4(0.f, 0.f, 0.f, 0.f);
             rb[h] = gj < s.nB ? __ldg(reinterpret_cast<const float4*>(K + (size_t)gj * kDh + d0) + lq)
                               : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -91,8 +91,8 @@ __global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float*
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
         const int gi = i0 + (u < 4 ? ty * 4 + u : 64 + ty * 4 + u - 4);
-        if (gi >= s.nB) continue;
-        float* out = scores + ((size_t)bh * s.nB + gi) * s.nB;
+        if (gi >= s.nQ) continue;
+        float* out = scores + ((size_t)bh * s.nQ + gi) * s.nB;
 #pragma unroll
         for (int w = 0; w < 8; ++w) {
             const int gj = j0 + (w < 4 ? tx * 4 + w : 64 + tx * 4 + w - 4);
@@ -125,8 +125,8 @@ __global__ void __launch_bounds__(kTopkWarps * 32) block_topk_kernel(Shape s, co
     uint32_t* keys = tk_smem + kTopkWarps * 256 + (size_t)warp * s.nB;
     const int row = blockIdx.x * kTopkWarps + warp;
     const int bh = blockIdx.y;
-    if (row >= s.nB) return;
-    const float* srow = scores + ((size_t)bh * s.nB + row) * s.nB;
+    if (row >= s.nQ) return;
+    const float* srow = scores + ((size_t)bh * s.nQ + row) * s.nB;
     for (int j = lane; j < s.nB; j += 32) keys[j] = order_key(srow[j]);
     __syncwarp();
 
@@ -176,7 +176,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) block_topk_kernel(Shape s, co
     }
     // prefix is now the threshold key; `need` keys equal to it are kept (lowest j first)
     const uint32_t thr = prefix;
-    int32_t* out = kv_idx + ((size_t)bh * s.nB + row) * s.n_keep;
+    int32_t* out = kv_idx + ((size_t)bh * s.nQ + row) * s.n_keep;
     int written = 0, eq_taken = 0;
     for (int j0 = 0; j0 < s.nB; j0 += 32) {
         int j = j0 + lane;
@@ -197,8 +197,8 @@ __global__ void __launch_bounds__(kTopkWarps * 32) block_topk_kernel(Shape s, co
 cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kbar, float* scores,
                               int32_t* kv_idx, cudaStream_t st)
 {
-    int t = (s.nB + kSTile - 1) / kSTile;
-    block_scores_kernel<<<dim3(t, t, s.B * s.H), 256, 0, st>>>(s, qbar, kbar, scores);
+    const int tj = (s.nB + kSTile - 1) / kSTile, ti = (s.nQ + kSTile - 1) / kSTile;
+    block_scores_kernel<<<dim3(tj, ti, s.B * s.H), 256, 0, st>>>(s, qbar, kbar, scores);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     size_t smem = (size_t)kTopkWarps * 256 * 4 + (size_t)kTopkWarps * s.nB * 4;
@@ -206,8 +206,28 @@ cudaError_t launch_block_topk(const Shape& s, const float* qbar, const float* kb
         e = cudaFuncSetAttribute(block_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
-    dim3 grid((s.nB + kTopkWarps - 1) / kTopkWarps, s.B * s.H);
+    dim3 grid((s.nQ + kTopkWarps - 1) / kTopkWarps, s.B * s.H);
     block_topk_kernel<<<grid, kTopkWarps * 32, smem, st>>>(s, scores, kv_idx);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// 128-token query means: the 64-token chunks' fp32 q sums S (each the pairwise
+// tree over its 64 slots) give chunk c of 128 tokens the tree's top node
+// S[2c] + S[2c+1] (an absent right half is the empty tree, +0), divided once by
+// the chunk's token count -- the pairwise sum over 128 slots.
+__global__ void qpool128_kernel(Shape s, const float* __restrict__ qsum, float* __restrict__ qbar)
+{
+    const int c = blockIdx.x, bh = blockIdx.y, d = threadIdx.x;
+    const float* src = qsum + ((size_t)bh * s.nB + 2 * c) * kDh + d;
+    const float right = 2 * c + 1 < s.nB ? src[kDh] : 0.0f;
+    const int cnt = min(128, s.N - 128 * c);
+    qbar[((size_t)bh * s.nQ + c) * kDh + d] = (src[0] + right) / (float)cnt;
+}
+
+cudaError_t launch_qpool128(const Shape& s, const float* qsum64, float* qbar128, cudaStream_t st)
+{
+    qpool128_kernel<<<dim3(s.nQ, s.B * s.H), kDh, 0, st>>>(s, qsum64, qbar128);
     return cudaGetLastError();
 }
 

@@ -435,9 +435,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<R>::kCtasPerSm) prepass_kernel(
                 pool0 = half_sum;
             } else {
                 // the top node: first half + second half, then the mean over the block's tokens
+                // (with 128-token query blocks the query side keeps the sum: one half of the 128-token tree)
                 const int cnt = min(kBlock, s.N - blk * kBlock);
+                const float sum = pool0 + half_sum;
                 (tid < kDh ? p.qbar : p.kbar)[((size_t)bh * s.nC + blk) * kDh + (tid & (kDh - 1))] =
-                    (pool0 + half_sum) / (float)cnt;
+                    (tid < kDh && s.qb2) ? sum : sum / (float)cnt;
             }
         }
         // ---- C^T += V^T k~ : this warp's 16 d columns, all r rows, 32 tokens

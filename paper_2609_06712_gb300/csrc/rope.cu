@@ -165,7 +165,9 @@ __global__ void __launch_bounds__(256) rope_pool_kernel(Shape s, const T* __rest
     __syncthreads();
     if (threadIdx.x < kDh) {
         const int cnt = min(kBlock, s.N - blk * kBlock);
-        xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = pairwise64(&rot[0][threadIdx.x], kDh) / (float)cnt;
+        const float sum = pairwise64(&rot[0][threadIdx.x], kDh);
+        // with 128-token query blocks the query side keeps the sum (the 128-token tree's left or right half)
+        xbar[((size_t)bh * s.nB + blk) * kDh + threadIdx.x] = (blockIdx.z == 0 && s.qb2) ? sum : sum / (float)cnt;
     }
 }
 

@@ -33,7 +33,7 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
     float* Ss = Vs + kBlock * kDh;         // [64][65]
     const int qb = blockIdx.x, bh = blockIdx.y, tid = threadIdx.x;
     const size_t head = (size_t)bh * s.Np * kDh;
-    const int32_t* kept = kv_idx + ((size_t)bh * s.nB + qb) * s.n_keep;
+    const int32_t* kept = kv_idx + ((size_t)bh * s.nQ + (qb >> s.qb2)) * s.n_keep;   // the block's mask row
     for (int e = tid; e < kBlock * kDh; e += kF32Threads) {
         int r = e / kDh, d = e % kDh, n = qb * kBlock + r;
         Qs[r * kPad + d] = n < s.Np ? qr[head + (size_t)n * kDh + d] : 0.0f;

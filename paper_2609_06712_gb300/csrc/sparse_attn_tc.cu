@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
         bool ok = true;
         for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
             const int bh = item / nB, qb = item - bh * nB;
-            const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
+            const int32_t* kept = p.kv_idx + ((size_t)bh * s.nQ + (qb >> s.qb2)) * s.n_keep;
             if (warp == kProducerKWarp) {
                 if (k >= 1) ok = mbar_wait(bar(Q_EMPTY), (k - 1) & 1, abort, s.wait_limit_ns);
                 ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -416,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_tc_kernel(const __gri
         int k = 0;
         for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
             const int bh = item / nB, qb = item - bh * nB;
-            const int32_t* kept = p.kv_idx + (size_t)item * s.n_keep;
+            const int32_t* kept = p.kv_idx + ((size_t)bh * s.nQ + (qb >> s.qb2)) * s.n_keep;
             const int ob = k & 1;
             if (wtid < kCols) sm.m[col0 + wtid] = 0.0f;       // holds -m_q
             float l[kCols];

@@ -39,6 +39,7 @@ class RolaConfig(ctypes.Structure):
         ("lowrank_rope", ctypes.c_int32),
         ("lowrank_act", ctypes.c_int32),
         ("block_geometry", ctypes.c_int32),
+        ("query_block", ctypes.c_int32),
     ]
 
 
@@ -73,6 +74,7 @@ def _load():
         "rola_config_init": (st, [cfgp]),
         "rola_num_blocks": (ctypes.c_int32, [cfgp]),
         "rola_num_keep": (ctypes.c_int32, [cfgp]),
+        "rola_num_query_blocks": (ctypes.c_int32, [cfgp]),
         "rola_workspace_bytes": (S, [cfgp]),
         "rola_block_mask": (st, [cfgp, P, P, P, P, S, P]),
         "rola_sparse_attn": (st, [cfgp, P, P, P, P, P, P, S, P]),
@@ -127,6 +129,7 @@ def make_config(cfg: dict, dtype: int = ROLA_BF16) -> RolaConfig:
     c.lowrank_act = LOWRANK_ACTS[act] if isinstance(act, str) else int(act)
     geom = cfg.get("block_geometry", "flat")
     c.block_geometry = BLOCK_GEOMETRIES[geom] if isinstance(geom, str) else int(geom)
+    c.query_block = int(cfg.get("qblock", 0))
     return c
 
 
@@ -150,6 +153,11 @@ def _check(status: int, where: str):
 
 def num_blocks(c: RolaConfig) -> int:
     return _lib.rola_num_blocks(ctypes.byref(c))
+
+
+def num_query_blocks(c: RolaConfig) -> int:
+    """Rows of kv_idx: 128-token query chunks when c.query_block is 128, else the key blocks."""
+    return _lib.rola_num_query_blocks(ctypes.byref(c))
 
 
 def num_keep(c: RolaConfig) -> int:

@@ -5,6 +5,8 @@ They are checked against independent counts: the oracle's block ids (numpy
 bincount), a brute-force loop over a random mask, the dense closed form
 4 B H L^2 d_h (App. D) when every block is kept, and the layer sizes of the
 Wan2.1-14B 720p layer (75600 tokens, 1182 blocks, the last of 16 tokens)."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -94,17 +96,41 @@ def test_accounting_uses_the_printed_complexity_formulas():
 
 
 def test_sparse_traffic_follows_the_committed_capture(tmp_path, monkeypatch):
-    """roofline.traffic comes from the committed ncu summary only while the kernel's sources
-    are the ones that capture was taken on: a summary recording another source hash, or one
-    without the two fields, gives None (the bench then reports traffic: null)."""
-    tph = bench.sparse_traffic_per_head_token()
-    assert tph is not None and 900.0 < tph < 1100.0      # q^r + k^r + v read, O^s written: ~4 x 256 B
+    """roofline.traffic comes from the committed ncu summary only while the kernel's sources are the
+    ones that capture was taken on: a summary recording the sources' own hash gives its figure, one
+    recording another hash, or lacking the two fields, gives None (the bench then reports
+    traffic: null).  The committed summary carries both fields."""
+    import hashlib
     text = open(bench.SPARSE_PROFILE).read()
+    assert "traffic_bytes_per_head_token: " in text and "kernel_sources_sha256: " in text
+    h = hashlib.sha256()
+    for f in bench.SPARSE_SOURCES:
+        h.update(open(os.path.join(bench.ROOT, "paper_2609_06712_gb300", "csrc", f), "rb").read())
+    current = tmp_path / "current.md"
+    current.write_text("notes\ntraffic_bytes_per_head_token: 996.5\nkernel_sources_sha256: " + h.hexdigest() + "\n")
+    monkeypatch.setattr(bench, "SPARSE_PROFILE", str(current))
+    assert bench.sparse_traffic_per_head_token() == 996.5
     stale = tmp_path / "stale.md"
-    stale.write_text(text.replace("kernel_sources_sha256: ", "kernel_sources_sha256: 0"))
+    stale.write_text("traffic_bytes_per_head_token: 996.5\nkernel_sources_sha256: " + "0" * 64 + "\n")
     monkeypatch.setattr(bench, "SPARSE_PROFILE", str(stale))
     assert bench.sparse_traffic_per_head_token() is None
     bare = tmp_path / "bare.md"
-    bare.write_text("\n".join(l for l in text.splitlines() if not l.startswith("traffic_bytes")))
+    bare.write_text("kernel_sources_sha256: " + h.hexdigest() + "\n")
     monkeypatch.setattr(bench, "SPARSE_PROFILE", str(bare))
     assert bench.sparse_traffic_per_head_token() is None
+
+
+def test_sparse_flops_with_128_token_query_chunks():
+    """With 128-token query chunks each mask row weighs its chunk's size: brute force over a random
+    mask on a ragged 585-token layer (query chunks 128 x 4 + 73, key blocks 64 x 9 ... 9)."""
+    cfg = configs.get("tiny", T=5, Hh=9, Ww=13, H=2)
+    ks, qs = bench.block_sizes(cfg), bench.block_sizes(cfg, 128)
+    assert sum(ks) == sum(qs) == 585 and len(qs) == 5 and qs[-1] == 73
+    rng = np.random.default_rng(3)
+    kv = torch.from_numpy(np.sort(np.stack([[rng.choice(len(ks), 3, replace=False) for _ in qs]
+                                            for _ in range(2)])[None], axis=-1).astype(np.int32))
+    want = 0.0
+    for h in range(2):
+        for i, qsz in enumerate(qs):
+            want += 4 * 128 * qsz * sum(ks[j] for j in kv[0, h, i].tolist())
+    assert bench.sparse_flops_from_mask(kv, ks, qsizes=qs) == want

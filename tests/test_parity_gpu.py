@@ -290,3 +290,85 @@ def test_forward_layer_shapes_sampled(rl, name, r, keep, nsample):
     rl.lowrank_summary(c, dev(x["k"]), dev(x["v"]), dev(x["P_k"]), C, None, ws)
     torch.cuda.synchronize()
     assert_close(to_np(C), res["C"], True, f"C[{cfg['name']}]", unit_rms=True)
+
+
+# ------------------------------------------------------------------ 128-token query blocks
+
+QBLOCK = {
+    # 585 tokens: query chunks of 128, 128, 128, 128, 73 against key blocks of 64 (the last of 9)
+    "q128_ragged_585": layer(T=5, Hh=9, Ww=13, H=2, r=32, keep=0.3, seed=71, qblock=128),
+    # 448 tokens: query chunks of 128 x 3 and 64 (an odd number of key blocks, 7)
+    "q128_odd_448": layer(T=4, Hh=8, Ww=14, H=3, r=16, keep=0.4, seed=72, qblock=128, dist="normal_gate"),
+}
+
+
+@pytest.mark.parametrize("case", sorted(QBLOCK))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_block_mask_query_blocks_of_128(rl, case, dname, tdt):
+    """128-token query chunks against 64-token key blocks: the mask (one row per query chunk) bit for bit
+    against the oracle's fp32 decision, every row."""
+    cfg = QBLOCK[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    nQ, nk = rl.num_query_blocks(c), rl.num_keep(c)
+    assert nQ == O.num_qblocks(cfg) == -(-cfg["N"] // 128) and rl.num_blocks(c) == O.num_blocks(cfg)
+    kv = torch.empty((cfg["B"], cfg["H"], nQ, nk), dtype=torch.int32, device="cuda")
+    rl.block_mask(c, dev(x["q"]), dev(x["k"]), kv, ws)
+    torch.cuda.synchronize()
+    check_mask(cfg, h, kv.cpu().numpy(), f"mask {case} {dname}")
+
+
+@pytest.mark.parametrize("case", sorted(QBLOCK))
+@pytest.mark.parametrize("dname,tdt", dtype_cases())
+def test_forward_query_blocks_of_128(rl, case, dname, tdt):
+    """The module with 128-token query blocks: the fused forward's mask bit for bit, then O on every token
+    against the oracle's forward (qblock = 128) under the GPU's mask."""
+    cfg = QBLOCK[case]
+    x, h = draw(cfg, tdt)
+    c = rl.make_config(cfg, rola_dtype(rl, dname))
+    ws = rl.workspace(c)
+    out = torch.empty_like(dev(x["q"]))
+    kv = torch.empty((cfg["B"], cfg["H"], rl.num_query_blocks(c), rl.num_keep(c)), dtype=torch.int32, device="cuda")
+    rl.forward(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), dev(x["P_q"]), dev(x["P_k"]), dev(x["gate"]), out, kv, ws)
+    torch.cuda.synchronize()
+    assert rl.get_device_status(ws) == rl.ROLA_OK
+    kvn = kv.cpu().numpy()
+    check_mask(cfg, h, kvn, f"forward {case} {dname}")
+    res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], mask_override=kvn)
+    assert_close(to_np(out), res["o"], dname == "bf16", f"O[{case},{dname}]")
+
+
+def test_forward_query_blocks_of_128_720p_sampled(rl):
+    """The Wan2.1-14B 720p layer with 128-token query chunks (591 of them, 118 of 1182 key blocks kept
+    each): the mask in full, O on sampled query chunks of every head (the first and the ragged last)."""
+    cfg = configs.get("wan14b_720p", qblock=128)
+    x, h = draw(cfg, torch.bfloat16)
+    c = rl.make_config(cfg)
+    ws = rl.workspace(c)
+    nQ = rl.num_query_blocks(c)
+    assert nQ == 591
+    out = torch.empty_like(dev(x["q"]))
+    kv = torch.empty((1, cfg["H"], nQ, rl.num_keep(c)), dtype=torch.int32, device="cuda")
+    rl.forward(c, dev(x["q"]), dev(x["k"]), dev(x["v"]), dev(x["P_q"]), dev(x["P_k"]), dev(x["gate"]), out, kv, ws)
+    torch.cuda.synchronize()
+    kvn = kv.cpu().numpy()
+    check_mask(cfg, h, kvn, "forward wan14b_720p qblock128 bf16")
+    chunks = sample_blocks(nQ, 16, seed=cfg["seed"])
+    res = O.forward(cfg, h["q"], h["k"], h["v"], h["P_q"], h["P_k"], h["gate"], mask_override=kvn, qblocks=chunks)
+    rows = rows_of_blocks(chunks, 128, cfg["N"])
+    got = to_np(out)
+    for hh in range(cfg["H"]):
+        assert_close(got[0, hh, rows], res["o"][0, hh, rows], True, f"O[720p q128,h{hh}]")
+
+
+def test_training_refuses_query_blocks_of_128(rl):
+    """The backward pass is built for 64-token query blocks only; the training entry points refuse 128."""
+    cfg = QBLOCK["q128_ragged_585"]
+    c = rl.make_config(cfg)
+    L = rl.library()
+    import ctypes
+    P = ctypes.c_void_p(0x10000)
+    w = ctypes.c_void_p(0x100000)
+    st = L.rola_forward_train(ctypes.byref(c), P, P, P, P, P, None, P, P, P, P, P, w, 1 << 30, None)
+    assert st == rl.ROLA_ERR_UNSUPPORTED
