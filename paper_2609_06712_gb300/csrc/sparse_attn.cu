@@ -4,9 +4,10 @@
 //
 // (Sec. 3 softmax form restricted to the kept blocks, Alg. 1 sparse branch).
 // q^r, k^r are the rotated copies written by the rotate + pool pass.  The
-// bf16 path is a tcgen05 kernel: sparse_attn_tc.cu for 64-token query blocks,
-// sparse_attn_q128.cu for 128-token query chunks; this file holds the fp32
-// validation-mode kernel (online softmax in fp32) and the dispatch.
+// bf16 path is a tcgen05 kernel: sparse_attn_rows.cu for contiguous key
+// blocks (64-token query blocks or 128-token query chunks), sparse_attn_tc.cu
+// for the cube geometry; this file holds the fp32 validation-mode kernel
+// (online softmax in fp32) and the dispatch.
 #include "common.cuh"
 
 namespace rola {
@@ -101,15 +102,15 @@ __global__ void __launch_bounds__(kF32Threads) sparse_attn_f32_kernel(Shape s, c
     }
 }
 
-// 128-token query chunks in bf16 (sparse_attn_q128.cu)
-cudaError_t launch_sparse_attn_q128(const Shape& s, const void* qr, const void* kr, const void* v,
+// bf16 with contiguous key blocks (sparse_attn_rows.cu)
+cudaError_t launch_sparse_attn_rows(const Shape& s, const void* qr, const void* kr, const void* v,
                                     const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status,
                                     cudaStream_t st);
 
 cudaError_t launch_sparse_attn(rola_dtype_t dt, const Shape& s, const void* qr, const void* kr, const void* v,
                                const int32_t* kv_idx, void* o_s, float* lse, DeviceStatus* status, cudaStream_t st)
 {
-    if (dt == ROLA_BF16 && s.qb2) return launch_sparse_attn_q128(s, qr, kr, v, kv_idx, o_s, lse, status, st);
+    if (dt == ROLA_BF16 && !s.cube) return launch_sparse_attn_rows(s, qr, kr, v, kv_idx, o_s, lse, status, st);
     if (dt == ROLA_BF16) return launch_sparse_attn_tc(s, qr, kr, v, kv_idx, o_s, lse, status, st);
     dim3 grid(s.nB, s.B * s.H);
     size_t smem = sizeof(float) * (2 * kBlock * kPad + kBlock * kDh + kBlock * 65);
