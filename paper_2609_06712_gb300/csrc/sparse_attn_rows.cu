@@ -65,7 +65,6 @@ constexpr int kProducerKWarp = 4, kProducerVWarp = 5, kMmaWarp = 6, kPvWarp = 7;
 constexpr int kThreads = 256;
 constexpr uint32_t kKPairBytes = 128 * 128 * 2;      // a pair of key blocks [d-chunk][block][64 rows][64]
 constexpr uint32_t kVBlockBytes = 64 * 128 * 2;      // one key block of v [d-chunk][64 rows][64]
-constexpr int KS = 3;                                // K ring (pairs)
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemS = 0;                       // S buffers at 0, 128
 constexpr uint32_t kTmemO = 256;
@@ -76,6 +75,7 @@ template <int QN>
 struct Cfg {
     static_assert(QN == 64 || QN == 128, "query blocks of 64 or 128 rows");
     static constexpr int QB = QN == 64 ? 2 : 1;                  // Q buffers
+    static constexpr int KS = 3;                                 // K ring (pairs)
     static constexpr int VB = QN == 64 ? 6 : 5;                  // V ring (single blocks)
     static constexpr int kCols = QN == 64 ? 64 : 128;            // keys of a tile per softmax thread
     static constexpr uint32_t kQBytes = QN * 128 * 2;            // [d-chunk][QN rows][64]
@@ -201,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_rows_kernel(const __g
                                                                        const Params p)
 {
     using C = Cfg<QN>;
-    constexpr int QB = C::QB, VB = C::VB, NC = C::kCols;
+    constexpr int QB = C::QB, KS = C::KS, VB = C::VB, NC = C::kCols;
     constexpr uint32_t kQBytes = C::kQBytes, kSmemQ = C::kSmemQ, kSmemK = C::kSmemK, kSmemV = C::kSmemV;
     constexpr int Q_FULL = C::Q_FULL, Q_EMPTY = C::Q_EMPTY, K_FULL = C::K_FULL, K_EMPTY = C::K_EMPTY,
                   V_FULL = C::V_FULL, V_EMPTY = C::V_EMPTY, S_FULL = C::S_FULL, S_EMPTY = C::S_EMPTY,
@@ -267,11 +267,13 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_rows_kernel(const __g
         // ------------------------------------------------------------ TMA producers
         // K warp: lane 0 loads Q (one box); lanes 2h + c load d-chunk c of
         // block h of the K pair (8 KB boxes, [chunk][block][row] so that the
-        // pair is one N = 128 operand).  V warp: lane h loads block h of the
-        // pair (one 16 KB box, [chunk][row]) into a ring of single-block slots.
+        // pair is one N = 128 operand).  V warp: lanes 2h + c load d-chunk c of
+        // block h into its slot of the ring of single blocks ([chunk][row]).
+        // A lane's copies are processed one after another, so every copy of a
+        // tile gets a lane of its own.
         const bool is_v = warp == kProducerVWarp;
-        const int h = is_v ? lane : (lane >> 1);
-        const int kc = lane & 1;
+        const int h = lane >> 1;                        // block of the pair
+        const int kc = lane & 1;                        // d-chunk
         int k = 0, issued_q = 0, issued_k = 0, issued_vb = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < p.total_items && ok; item += gridDim.x, ++k) {
@@ -297,15 +299,15 @@ __global__ void __launch_bounds__(kThreads, 1) sparse_attn_rows_kernel(const __g
                     const int c = k * s.n_keep + 2 * t + h;       // cumulative block index of block h
                     const int slot = c % VB;
                     bool okl = true;
-                    if (lane < 2 && h < nblk && c >= VB)
+                    if (lane < 4 && kc == 0 && h < nblk && c >= VB)
                         okl = mbar_wait(bar(V_EMPTY + slot), ((c / VB) - 1) & 1, abort, s.wait_limit_ns);
-                    ok = __shfl_sync(0xffffffffu, okl, 0) && __shfl_sync(0xffffffffu, okl, 1);
+                    ok = __shfl_sync(0xffffffffu, okl, 0) && __shfl_sync(0xffffffffu, okl, 2);
                     if (!ok) break;
-                    if (lane < 2 && h < nblk) {
-                        mbar_expect_tx(bar(V_FULL + slot), kVBlockBytes);
-                        tma_load_4d(sbase + kSmemV + slot * kVBlockBytes, &map_v, bar(V_FULL + slot), 0,
-                                    (h ? jb : ja) * 64, 0, bh);
-                    }
+                    if (lane < 4 && kc == 0 && h < nblk) mbar_expect_tx(bar(V_FULL + slot), kVBlockBytes);
+                    __syncwarp();
+                    if (lane < 4 && h < nblk)
+                        tma_load_3d(sbase + kSmemV + slot * kVBlockBytes + kc * 8192, &map_v, bar(V_FULL + slot),
+                                    kc * 64, (h ? jb : ja) * 64, bh);
                     issued_vb += nblk;
                 } else {
                     const int st = g % KS;
@@ -567,7 +569,7 @@ cudaError_t launch_rows(const Shape& s, const void* qr, const void* kr, const vo
                         void* o_s, float* lse, DeviceStatus* status, cudaStream_t st)
 {
     CUtensorMap mq, mk, mv;
-    if (!make_block_map(&mq, qr, s, QN) || !make_chunk_map(&mk, kr, s) || !make_block_map(&mv, v, s))
+    if (!make_block_map(&mq, qr, s, QN) || !make_chunk_map(&mk, kr, s) || !make_chunk_map(&mv, v, s))
         return cudaErrorInvalidValue;
     int dev = 0, nsm = 0;
     cudaError_t e = cudaGetDevice(&dev);
