@@ -36,8 +36,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 
 # The ncu summary that carries the sparse kernel's DRAM traffic per (head, token), and
 # the sources its capture was taken on.
-SPARSE_PROFILE = os.path.join(ROOT, "profiles", "sparse_attn_tc_wan13b_480p.md")
-SPARSE_SOURCES = ["sparse_attn_tc.cu", "common.cuh", "tcgen05.cuh", "tensor_map.cuh"]
+SPARSE_PROFILE = os.path.join(ROOT, "profiles", "sparse_attn_rows_wan13b_480p.md")
+SPARSE_SOURCES = ["sparse_attn_rows.cu", "common.cuh", "tcgen05.cuh", "tensor_map.cuh"]
 
 
 def sparse_traffic_per_head_token():
@@ -507,14 +507,15 @@ def main():
     # sustained figure was measured over 4 s under the power cap, at a lower clock)
     peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-    tph = sparse_traffic_per_head_token() if geometry == "flat" else None
+    # the capture is of the 64-token query blocks on contiguous key blocks
+    tph = sparse_traffic_per_head_token() if geometry == "flat" and cfg.get("qblock", 0) in (0, 64) else None
     traffic = None if tph is None else tph * cfg["B"] * cfg["H"] * cfg["N"]
     roofline = {"bound": "tensor", "kernel": "sparse_attn", "achieved": achieved, "peak": peak,
                 "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                 "peak_source": f"{peak_src} bf16_tflops (burst: sub-second timed region at full clock)",
                 "frac_of_sustained": achieved / peak_sus,
                 "traffic_source": (None if traffic is None else
-                                   "profiles/sparse_attn_tc_wan13b_480p.md, per (head, token) x B*H*N"),
+                                   "profiles/sparse_attn_rows_wan13b_480p.md, per (head, token) x B*H*N"),
                 "algorithmic_flops_per_launch": fl, "ms_per_launch": sp_ms}
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     tensor_bytes = summary_bytes(cfg["B"], cfg["H"], cfg["N"], 128) / 2      # one [B,H,N,128] bf16 tensor

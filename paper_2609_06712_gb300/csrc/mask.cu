@@ -20,9 +20,10 @@ namespace rola {
 
 constexpr int kSTile = 128, kSChunk = 16;
 
-__global__ void __launch_bounds__(256) block_scores_kernel(Shape s, const float* __restrict__ qbar,
-                                                           const float* __restrict__ kbar,
-                                                           float* __restrict__ scores)
+// (two CTAs per SM: the 128-register budget keeps both resident)
+__global__ void __launch_bounds__(256, 2) block_scores_kernel(Shape s, const float* __restrict__ qbar,
+                                                              const float* __restrict__ kbar,
+                                                              float* __restrict__ scores)
 {
     __shared__ __align__(16) float qs[2][kSChunk][kSTile + 4];
     __shared__ __align__(16) float ks[2][kSChunk][kSTile + 4];

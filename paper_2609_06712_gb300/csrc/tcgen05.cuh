@@ -265,22 +265,5 @@ __device__ __forceinline__ void bar_sync(int id, int count)
     asm volatile("barrier.cta.sync %0, %1;\n" ::"r"(id), "r"(count) : "memory");
 }
 
-// Per-warpgroup register budget (every warp of a warpgroup executes the same
-// form).  The launch's registers (threads x registers per thread) are the pool:
-// the decreases and increases of a kernel must add up within it, or an
-// increase waits for registers that never come.
-template <uint32_t R>
-__device__ __forceinline__ void setmaxnreg_dec()
-{
-    static_assert(R % 8 == 0 && R >= 24 && R <= 256, "setmaxnreg takes multiples of 8 in [24, 256]");
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(R));
-}
-template <uint32_t R>
-__device__ __forceinline__ void setmaxnreg_inc()
-{
-    static_assert(R % 8 == 0 && R >= 24 && R <= 256, "setmaxnreg takes multiples of 8 in [24, 256]");
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(R));
-}
-
 }  // namespace tc
 }  // namespace rola
