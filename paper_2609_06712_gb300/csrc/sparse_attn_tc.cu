@@ -4,6 +4,10 @@
 //
 // (Sec. 3 softmax form restricted to the kept key blocks, Alg. 1 sparse branch.)
 //
+// This transposed form serves the 4 x 4 x 4 cube geometry, where a thread per
+// key keeps the slot-validity test and the scatter of O^s rows local;
+// contiguous key blocks run the row-wise kernel of sparse_attn_rows.cu.
+//
 // Mapping to tcgen05.  A query block has only 64 rows, but every MMA here
 // has M = 128: the kernel works on the TRANSPOSED problem, with a pair of
 // kept 64-key blocks as the 128-row operand.
@@ -656,7 +660,9 @@ cudaError_t launch_sparse_attn_tc(const Shape& s, const void* qr, const void* kr
     p.tiles = (s.n_keep + 1) / 2;
     const size_t smem = kSmemTiles + sizeof(Smem);
     const int grid = p.total_items < nsm ? p.total_items : nsm;
-    auto kernel = s.cube ? sparse_attn_tc_kernel<true> : sparse_attn_tc_kernel<false>;
+    // contiguous key blocks run the row-wise kernel (sparse_attn_rows.cu); this one serves cubes
+    if (!s.cube) return cudaErrorInvalidValue;
+    auto kernel = sparse_attn_tc_kernel<true>;
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     kernel<<<grid, kThreads, smem, st>>>(mq, mk, mv, p);
