@@ -656,14 +656,29 @@ def main():
             torch.cuda.synchronize()
             return reduce_max(a.elapsed_time(z) / n, ws)
 
+        # the host link on its own: one step's inputs in and one output back, each timed alone
+        torch.cuda.synchronize()
+        l0, l1, l2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        with torch.cuda.stream(s_in):
+            l0.record(s_in)
+            copy_in(0)
+            l1.record(s_in)
+            o_host[0].copy_(obuf[0], non_blocking=True)
+            l2.record(s_in)
+        torch.cuda.synchronize()
+        link = {"h2d_gbs": h2d / (l0.elapsed_time(l1) * 1e-3) / 1e9, "d2h_gbs": d2h / (l1.elapsed_time(l2) * 1e-3) / 1e9}
         ke = max(4, K)
         serial_ms = timed(serial_steps, max(2, K // 2))
-        e_ms = timed(pipelined_steps, ke)
+        # three timed windows of ke pipelined steps; the median window is reported (the host link's
+        # speed varied between processes on one box, so one window alone is a noisy sample)
+        windows = [timed(pipelined_steps, ke) for _ in range(3)]
+        e_ms = sorted(windows)[1]
         assert rola.get_device_status(wsb) == rola.ROLA_OK
         e2e = {"value": job_throughput(tokens, e_ms, ws), "unit": "tokens/s", "ms_per_step": e_ms,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke,
+               "windows_ms_per_step": windows, "link": link,
                "mode": "pipelined: step i+1's host-to-device copies and step i's device-to-host read overlap "
-                       "step i's layer on two copy streams",
+                       "step i's layer on two copy streams; median of three timed windows",
                "serial": {"value": job_throughput(tokens, serial_ms, ws), "ms_per_step": serial_ms}}
         del dbuf, obuf
 
