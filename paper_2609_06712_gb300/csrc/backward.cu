@@ -954,8 +954,9 @@ __global__ void __launch_bounds__(kMT) lr_bwd_k_mma_kernel(Shape s, const __nv_b
 {
     extern __shared__ __align__(128) uint8_t msm[];
     const uint32_t b0 = smem_u32(msm);
-    // layout: X (k) [64] | V [64] | P [R rows] | dC [R rows] | dU [64]
-    const uint32_t sX = b0, sV = b0 + kTile, sP = b0 + 2 * kTile, sC = sP + R * 256, sU = sC + R * 256;
+    // layout: X (k) [64] | V [64] | P [R rows] | dC [R rows]; dU takes V's place: a warp reads only its
+    // own 16 rows of V (dk~ = dC v) and writes dU to the same rows, so 48 KB at r = 32 and four CTAs an SM
+    const uint32_t sX = b0, sV = b0 + kTile, sP = b0 + 2 * kTile, sC = sP + R * 256, sU = sV;
     const int chunk = blockIdx.x, bh = blockIdx.y, h = bh % s.H;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, tig = lane & 3;
     const int n0 = chunk * 64, t0 = 16 * warp + g;
@@ -989,6 +990,7 @@ __global__ void __launch_bounds__(kMT) lr_bwd_k_mma_kernel(Shape s, const __nv_b
     float df[R / 8][4] = {};
     mma_rows_x_w<R>(df, sV, 16 * warp, sC, lane);
     frag_features_bwd<R>(s, tab, u, df, n0, t0, tig, act);
+    __syncwarp();                                 // this warp's V rows are read: dU goes in their place
 #pragma unroll
     for (int nt = 0; nt < R / 8; ++nt) {
         put_pair(msm, sU - b0, t0, 8 * nt + 2 * tig, df[nt][0], df[nt][1]);
@@ -1011,15 +1013,15 @@ __global__ void __launch_bounds__(kMT) lr_bwd_k_mma_kernel(Shape s, const __nv_b
     mma_outer<R>(sU, sX, s.r, partPk + ((size_t)bh * s.nC + chunk) * s.r * kDh, warp, lane);
 }
 
-// three 64-row tiles and the two R-row weight tiles (both kernels)
+// 64-row tiles (three on the query side, two on the key side) and the two R-row weight tiles
 template <int R>
-size_t lr_mma_smem() { return 3 * (size_t)kTile + 2 * (size_t)R * 256; }
+size_t lr_mma_smem(bool key_side) { return (key_side ? 2 : 3) * (size_t)kTile + 2 * (size_t)R * 256; }
 
 template <int R>
 cudaError_t launch_lr_mma_r(const Shape& s, const BackwardArgs& a, bool key_side, cudaStream_t st)
 {
     const dim3 chunks(s.nC, s.B * s.H);
-    const size_t smem = lr_mma_smem<R>();
+    const size_t smem = lr_mma_smem<R>(key_side);
     using bf = __nv_bfloat16;
     if (!key_side) {
         cudaError_t e = cudaFuncSetAttribute(lr_bwd_q_mma_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
