@@ -213,6 +213,39 @@ def test_fp32_pooling_is_pairwise_in_slot_order(oracle):
     assert np.float32(262144.0625 / 4) * scale != np.float32(262144.03125 / 4) * scale
 
 
+def test_fp32_pooling_of_128_token_query_chunks(oracle):
+    """A 128-token query chunk pools its 128 slots pairwise in slot order -- the top node of the two
+    64-slot trees -- and divides once by its token count.  Frame 0 only (coordinate 0 of pair 0 is
+    not rotated), every other coordinate 0, key block 0's mean in coordinate 0 is 1."""
+    O = oracle
+    scale = np.float32(1.0 / math.sqrt(128.0))
+    # 128 tokens of frame 0: token 0 holds 2^24, tokens 1..127 hold 1.  The first 64-slot tree gives
+    # 2^24 + 62 (its first pair rounds 2^24 + 1 to 2^24), the second 64 exactly, the top node
+    # 2^24 + 126 (even, exact); divided by 128: 131072.984375, exact.  The sequential sum would keep
+    # 2^24 (131072) and the exact sum 2^24 + 127 would round differently.
+    cfg = small_cfg(T=2, Hh=8, Ww=16, H=1, keep=0.5, qblock=128)
+    assert O.num_qblocks(cfg) == 2 and O.num_blocks(cfg) == 4
+    q = np.zeros((1, 1, cfg["N"], 128), np.float32)
+    k = np.zeros_like(q)
+    q[0, 0, :128, 0] = 1.0
+    q[0, 0, 0, 0] = 2.0 ** 24
+    k[0, 0, :64, 0] = 1.0
+    _, s32 = O.block_mask_f32(cfg, q, k)
+    assert s32[0, 0, 0, 0] == np.float32(np.float32(2.0 ** 24 + 126) / np.float32(128)) * scale
+    assert s32[0, 0, 0, 0] == np.float32(131072.984375) * scale
+    assert np.float32(131072.0) * scale != np.float32(131072.984375) * scale
+    # a ragged last chunk: 128 + 73 tokens in one frame; chunk 1 holds 73 tokens of value 1, so its
+    # pooled value is 73 / 73 = 1 (a divisor of 128 would give 0.5703125)
+    cfg = small_cfg(T=1, Hh=3, Ww=67, H=1, keep=0.5, qblock=128)
+    assert cfg["N"] == 201 and O.num_qblocks(cfg) == 2
+    q = np.zeros((1, 1, 201, 128), np.float32)
+    k = np.zeros_like(q)
+    q[0, 0, 128:, 0] = 1.0
+    k[0, 0, :64, 0] = 1.0
+    _, s32 = O.block_mask_f32(cfg, q, k)
+    assert s32[0, 0, 1, 0] == np.float32(1.0) * scale
+
+
 def test_fp32_decision_ties_and_brute_force(oracle):
     """The fp32 decision keeps, per row, the n_keep-subset with the largest fp32 score sum (brute
     force over all subsets on the tiny layer, whose fp32 scores are distinct), and breaks an exact
