@@ -77,6 +77,7 @@ MUTATIONS = {
                             "return x[0] + pairwise_f32(x + 1, n - 1);"),
     "f32_rotation_sign": ("yr[2 * m] = fmaf(x0, cm, -p1);", "yr[2 * m] = fmaf(x0, cm, p1);"),
     "f32_pool_divisor": ("pairwise_f32(vals, slots) / (float)cnt;", "pairwise_f32(vals, slots) / (float)slots;"),
+    "f32_query_chunk_slots": ("int qslots = c->geometry == 1 ? kslots : qblock_size(c);", "int qslots = kslots;"),
     "f32_tie_order": ("return (x->j > y->j) - (x->j < y->j);", "return (x->j < y->j) - (x->j > y->j);"),
     "f32_scale_dropped": ("row[j].s = acc * scale;", "row[j].s = acc;"),
     "f32_cube_slot_order": ("x = CUBE * cx + (i / CUBE) % CUBE, y = CUBE * cy + i % CUBE;",
