@@ -45,6 +45,8 @@ SMALL = {
     # ranks that are not multiples of 16 (the paper's sweep starts at r = 8)
     "r8_ragged": layer(T=3, Hh=7, Ww=11, H=2, r=8, keep=0.25, seed=28),
     "r24": layer(T=2, Hh=8, Ww=12, H=2, r=24, keep=0.3, seed=29, dist="normal_gate"),
+    # the whole sequence is one partial block (40 tokens): one query block, one kept key block, a half tile
+    "one_partial_block": layer(T=1, Hh=5, Ww=8, H=2, r=16, keep=0.5, seed=30),
 }
 
 
